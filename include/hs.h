@@ -1,0 +1,187 @@
+/*
+ * hs.h — C ABI of the GB300 embed-and-retrieve hot path of HeraSys'
+ * cross-workflow node merging.
+ *
+ * The stage has four steps, each one call:
+ *   hs_fingerprint      hash every input row (chunk tokens or query vectors)
+ *   hs_unique_inverse   merge exactly-equal rows into unique nodes + inverse map
+ *   hs_retrieve_topk    score merged queries against a corpus, keep top-k
+ *   hs_scatter_results  fan each kept result back out to every merged row
+ *
+ * Conventions shared by every call
+ *   - Pointers named *_dev or documented as device pointers must be device
+ *     memory of the current CUDA device; the caller owns all of them
+ *     (inputs, outputs and workspace).  The library allocates no device
+ *     memory in any call.
+ *   - Every call enqueues its kernels on `stream` (a cudaStream_t; NULL is
+ *     the legacy default stream) and returns without synchronising.
+ *   - Argument errors that the host can see are returned at once and nothing
+ *     is enqueued; hs_last_error() then describes them.  Errors that only the
+ *     device can see (a row length outside [0, row_stride], a map entry out
+ *     of range, a bounded wait that ran out) set a per-device error word;
+ *     hs_get_device_error() synchronises the stream and reports and clears it.
+ *   - Unless stated otherwise, device pointers must be 16-byte aligned.
+ *   - Calls on one stream run in order; calls on different streams that
+ *     share an output or a workspace race.
+ */
+#ifndef HS_H_
+#define HS_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t / CUstream, without including CUDA headers. */
+typedef struct CUstream_st* hs_stream_t;
+
+typedef enum {
+  HS_OK = 0,
+  HS_ERR_INVALID_ARG = 1, /* bad size, pointer, alignment or (device) data  */
+  HS_ERR_UNSUPPORTED = 2, /* valid request this build does not handle       */
+  HS_ERR_CUDA = 3,        /* a CUDA runtime/driver call failed              */
+  HS_ERR_WORKSPACE = 4,   /* workspace pointer NULL/misaligned or too small */
+  HS_ERR_TIMEOUT = 5      /* a bounded device-side wait ran out             */
+} hs_status;
+
+/* FNV-1a 64-bit offset basis: the seed of a plain (unseeded) hash. */
+#define HS_FNV64_OFFSET_BASIS 0xcbf29ce484222325ULL
+
+/* Largest k accepted by hs_retrieve_topk. */
+#define HS_TOPK_MAX_K 1024
+
+/* Human-readable description of the last error returned on this host
+ * thread ("" if none).  The string stays valid until the next hs_* call on
+ * the same thread. */
+const char* hs_last_error(void);
+
+/* Library version string. */
+const char* hs_version(void);
+
+/*
+ * hs_fingerprint — per-row node signature over the input data.
+ *
+ * Paper: Section 3.3, Eq. 2: Sig(v) = H(tau_v, Theta_p, D_in, ordered
+ * combination of predecessor signatures).  This call computes the D_in part
+ * with H = 64-bit FNV-1a over octets: for row i,
+ *   fp[i] = FNV-1a(seed_state, little-endian octets of tokens[i, 0:len_i])
+ * i.e. h = seed_state; for each octet b: h = (h xor b) * 1099511628211 mod 2^64.
+ * tau_v, Theta_p and the predecessor signatures are folded in by the caller:
+ * hash their canonical bytes first and pass the result as seed_state (FNV-1a
+ * continues a byte stream exactly).  Pass HS_FNV64_OFFSET_BASIS for the
+ * plain hash.
+ *
+ * tokens      device, int32 [n_rows, row_stride] row-major.  Query vectors are
+ *             hashed by viewing their bf16 bits as int32 words (dim/2 words).
+ * n_rows      >= 0 (0: nothing is enqueued).
+ * row_stride  >= 0, words between consecutive rows.
+ * lens        device int32 [n_rows] or NULL (every row has row_stride words).
+ *             A length outside [0, row_stride] sets the device error word
+ *             (HS_ERR_INVALID_ARG) and that row's fp is written as 0.
+ * fp_out      device uint64 [n_rows], 8-byte aligned.
+ * tokens needs only 4-byte alignment; 16-byte aligned tokens with
+ * row_stride % 4 == 0 take the vector path.
+ */
+hs_status hs_fingerprint(const int32_t* tokens, int64_t n_rows, int32_t row_stride,
+                         const int32_t* lens, uint64_t seed_state, uint64_t* fp_out,
+                         hs_stream_t stream);
+
+/*
+ * hs_unique_inverse — exact merge of equal rows (node fusion).
+ *
+ * Paper: Section 3.3, "Dynamic Fusion and Reuse Mechanism" (I): a node that
+ * matches a node already in the window is removed and its downstream edges
+ * are redirected to the kept node; Appendix A.2, "Redundancy Elimination &
+ * Result Sharing": merge sets M(v*) executed once.
+ *
+ * Rows i and j are equal iff len_i == len_j and tokens[i, 0:len] ==
+ * tokens[j, 0:len] (words beyond len are ignored).  Outputs:
+ *   *n_unique_dev      number of groups,
+ *   unique_idx_out[u]  index of group u's first occurrence, ascending in u,
+ *   inverse_out[i]     group ordinal of row i (the redirected edge),
+ * so rows[unique_idx[inverse[i]]] == rows[i].  fp must hold fingerprints of
+ * these rows that are equal for equal rows (as hs_fingerprint produces with
+ * one seed); different rows may share a fingerprint (a collision): they are
+ * told apart by a full row comparison, never merged.  Cost is linear in the
+ * row bytes plus a radix sort of the fingerprints; rows whose fingerprints
+ * collide are resolved by an extra pass that is quadratic in the number of
+ * distinct rows sharing one fingerprint.
+ *
+ * fp              device uint64 [n_rows], 8-byte aligned.
+ * tokens, n_rows, row_stride, lens   as for hs_fingerprint;
+ *                 1 <= ... n_rows <= 2^30 - 1 (0 writes *n_unique_dev = 0).
+ * n_unique_dev    device int32 scalar.
+ * unique_idx_out  device int32 [n_rows] (only the first *n_unique_dev used).
+ * inverse_out     device int32 [n_rows].
+ * workspace       device, >= hs_unique_inverse_workspace(n_rows) bytes,
+ *                 256-byte aligned; contents on entry are ignored.
+ */
+size_t hs_unique_inverse_workspace(int64_t n_rows);
+hs_status hs_unique_inverse(const uint64_t* fp, const int32_t* tokens, int64_t n_rows,
+                            int32_t row_stride, const int32_t* lens, int32_t* n_unique_dev,
+                            int32_t* unique_idx_out, int32_t* inverse_out, void* workspace,
+                            size_t workspace_bytes, hs_stream_t stream);
+
+/*
+ * hs_retrieve_topk — dense retrieval of the merged queries, fused top-k.
+ *
+ * Paper: Section 4.1, "Workloads": queries and documents are embedded and
+ * the top-k (k = 12 in the paper) chunks are retrieved per query; the merged
+ * queries of Section 3.3 share one retrieval.  Here:
+ *   S[q, j] = sum_t queries[q, t] * corpus[j, t]   (bf16 inputs, fp32 sums)
+ * and for each q the k pairs (S[q, j], j) that come first in the order
+ * (score descending, ties to the lower j), written in that order.  The
+ * Q x N score matrix is never stored.  For unit-norm rows S is the cosine.
+ *
+ * queries     device bf16 bits (uint16) [n_queries, dim] row-major.
+ * corpus      device bf16 bits (uint16) [n_corpus, dim] row-major.
+ * n_queries   >= 0 (0: nothing enqueued); n_corpus >= 1, < 2^31.
+ * dim         >= 8, dim % 8 == 0.
+ * k           1 <= k <= min(n_corpus, HS_TOPK_MAX_K).
+ * scores_out  device float [n_queries, k]; ids_out device int32 [n_queries, k].
+ * workspace   device, >= hs_retrieve_topk_workspace(...) bytes, 256-byte
+ *             aligned; contents on entry are ignored.
+ * Inputs must be finite; a NaN score is never selected.
+ */
+size_t hs_retrieve_topk_workspace(int64_t n_queries, int64_t n_corpus, int32_t dim, int32_t k);
+hs_status hs_retrieve_topk(const uint16_t* queries, int64_t n_queries, const uint16_t* corpus,
+                           int64_t n_corpus, int32_t dim, int32_t k, float* scores_out,
+                           int32_t* ids_out, void* workspace, size_t workspace_bytes,
+                           hs_stream_t stream);
+
+/*
+ * hs_scatter_results — row gather/scatter: dst[i, :] = src[map[i], :].
+ *
+ * Paper: Section 3.3 (I): upon completion the output of the kept node flows
+ * to the downstream nodes of all merged queries; Appendix A.2: nodes in
+ * M(v*) depend on the output of v*.  With map = inverse from
+ * hs_unique_inverse this fans results back to every originating row; with
+ * map = unique_idx it gathers the unique rows.
+ *
+ * src        device [n_src, row_bytes] bytes; dst device [n_rows, row_bytes].
+ * map        device int32 [n_rows]; an entry outside [0, n_src) sets the device
+ *            error word (HS_ERR_INVALID_ARG) and leaves that dst row unwritten.
+ * row_bytes  >= 1.  Any alignment is accepted; src/dst 16-byte aligned with
+ *            row_bytes % 16 == 0 take the 16-byte vector path, 4-byte aligned
+ *            with row_bytes % 4 == 0 the word path, otherwise bytes.
+ * n_rows     >= 0 (0: nothing enqueued).  src and dst must not overlap.
+ */
+hs_status hs_scatter_results(const void* src, int64_t n_src, int64_t row_bytes,
+                             const int32_t* map, int64_t n_rows, void* dst,
+                             hs_stream_t stream);
+
+/*
+ * hs_get_device_error — synchronise `stream`, then read and clear the
+ * current device's error word.  Returns HS_OK if no kernel reported a
+ * problem since the last call, else the recorded status (HS_ERR_TIMEOUT
+ * takes precedence over HS_ERR_INVALID_ARG).
+ */
+hs_status hs_get_device_error(hs_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* HS_H_ */

@@ -1,0 +1,204 @@
+"""Thin ctypes binding of libhs.so with the C ABI's names.
+
+Argument marshalling only: every function passes device pointers
+(``tensor.data_ptr()``), sizes and the current torch CUDA stream to the
+library and returns the tensors it wrote.  Workspaces and outputs are torch
+allocations when the caller does not pass them.  Every step of the path runs
+in the library's kernels; if the library cannot be built or loaded, these
+functions raise instead of computing anything another way.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+from . import build as _build
+
+HS_OK = 0
+HS_ERR_INVALID_ARG = 1
+HS_ERR_UNSUPPORTED = 2
+HS_ERR_CUDA = 3
+HS_ERR_WORKSPACE = 4
+HS_ERR_TIMEOUT = 5
+HS_FNV64_OFFSET_BASIS = 0xCBF29CE484222325
+HS_TOPK_MAX_K = 1024
+
+_STATUS = {0: "HS_OK", 1: "HS_ERR_INVALID_ARG", 2: "HS_ERR_UNSUPPORTED", 3: "HS_ERR_CUDA",
+           4: "HS_ERR_WORKSPACE", 5: "HS_ERR_TIMEOUT"}
+
+_lock = threading.Lock()
+_lib = None
+
+
+class HsError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__("%s: %s" % (_STATUS.get(status, str(status)), msg))
+        self.status = status
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load(build_if_missing: bool = True) -> ctypes.CDLL:
+    """Load libhs.so (building it first if it is missing or stale)."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if build_if_missing:
+                _build.build()
+            if not os.path.exists(_build.LIB):
+                raise RuntimeError("libhs.so is missing: run paper_2607_22578_gb300.build.build()")
+            lib = ctypes.CDLL(_build.LIB)
+            P, i64, i32, u64, sz = (ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32,
+                                    ctypes.c_uint64, ctypes.c_size_t)
+            st = ctypes.c_int
+            lib.hs_last_error.restype = ctypes.c_char_p
+            lib.hs_version.restype = ctypes.c_char_p
+            lib.hs_fingerprint.argtypes = [P, i64, i32, P, u64, P, P]
+            lib.hs_fingerprint.restype = st
+            lib.hs_unique_inverse_workspace.argtypes = [i64]
+            lib.hs_unique_inverse_workspace.restype = sz
+            lib.hs_unique_inverse.argtypes = [P, P, i64, i32, P, P, P, P, P, sz, P]
+            lib.hs_unique_inverse.restype = st
+            lib.hs_retrieve_topk_workspace.argtypes = [i64, i64, i32, i32]
+            lib.hs_retrieve_topk_workspace.restype = sz
+            lib.hs_retrieve_topk.argtypes = [P, i64, P, i64, i32, i32, P, P, P, sz, P]
+            lib.hs_retrieve_topk.restype = st
+            lib.hs_scatter_results.argtypes = [P, i64, i64, P, i64, P, P]
+            lib.hs_scatter_results.restype = st
+            lib.hs_get_device_error.argtypes = [P]
+            lib.hs_get_device_error.restype = st
+            _lib = lib
+    return _lib
+
+
+def _check(status: int) -> None:
+    if status != HS_OK:
+        raise HsError(status, load().hs_last_error().decode())
+
+
+def _stream(stream) -> int:
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, torch.cuda.Stream):
+        return stream.cuda_stream
+    return int(stream)
+
+
+def _ptr(t):
+    return None if t is None else t.data_ptr()
+
+
+def _cuda(t: torch.Tensor, name: str) -> torch.Tensor:
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError("%s must be a CUDA tensor" % name)
+    if not t.is_contiguous():
+        raise ValueError("%s must be contiguous" % name)
+    return t
+
+
+def hs_version() -> str:
+    return load().hs_version().decode()
+
+
+def hs_fingerprint(tokens: torch.Tensor, lens: torch.Tensor | None = None,
+                   seed_state: int = HS_FNV64_OFFSET_BASIS, fp_out: torch.Tensor | None = None,
+                   stream=None) -> torch.Tensor:
+    """fp[i] = FNV-1a-64 over row i's little-endian token octets (int64 tensor
+    holding the uint64 bit patterns)."""
+    _cuda(tokens, "tokens")
+    if tokens.dtype != torch.int32 or tokens.dim() != 2:
+        raise TypeError("tokens must be a 2-D int32 tensor")
+    n, stride = tokens.shape
+    if lens is not None:
+        _cuda(lens, "lens")
+        if lens.dtype != torch.int32 or lens.numel() != n:
+            raise TypeError("lens must be int32 [n_rows]")
+    if fp_out is None:
+        fp_out = torch.empty(n, dtype=torch.int64, device=tokens.device)
+    _check(load().hs_fingerprint(_ptr(tokens), n, stride, _ptr(lens), seed_state & (2**64 - 1),
+                                 _ptr(fp_out), _stream(stream)))
+    return fp_out
+
+
+def hs_unique_inverse_workspace(n_rows: int) -> int:
+    return int(load().hs_unique_inverse_workspace(n_rows))
+
+
+def hs_unique_inverse(fp: torch.Tensor, tokens: torch.Tensor, lens: torch.Tensor | None = None,
+                      workspace: torch.Tensor | None = None, out: tuple | None = None,
+                      stream=None):
+    """Exact unique rows.  Returns (n_unique_dev [1] int32, unique_idx [n]
+    int32, inverse [n] int32); only the first n_unique entries of unique_idx
+    are meaningful."""
+    _cuda(fp, "fp")
+    _cuda(tokens, "tokens")
+    n, stride = tokens.shape
+    dev = tokens.device
+    if out is None:
+        out = (torch.empty(1, dtype=torch.int32, device=dev),
+               torch.empty(max(n, 1), dtype=torch.int32, device=dev),
+               torch.empty(max(n, 1), dtype=torch.int32, device=dev))
+    nu, uidx, inv = out
+    need = hs_unique_inverse_workspace(n)
+    if workspace is None:
+        workspace = torch.empty(need, dtype=torch.uint8, device=dev)
+    _check(load().hs_unique_inverse(_ptr(fp), _ptr(tokens), n, stride, _ptr(lens), _ptr(nu),
+                                    _ptr(uidx), _ptr(inv), _ptr(workspace), workspace.numel(),
+                                    _stream(stream)))
+    return nu, uidx[:n], inv[:n]
+
+
+def hs_retrieve_topk_workspace(n_queries: int, n_corpus: int, dim: int, k: int) -> int:
+    return int(load().hs_retrieve_topk_workspace(n_queries, n_corpus, dim, k))
+
+
+def hs_retrieve_topk(queries: torch.Tensor, corpus: torch.Tensor, k: int,
+                     workspace: torch.Tensor | None = None, out: tuple | None = None,
+                     stream=None):
+    """Top-k inner products of bf16 query rows against bf16 corpus rows.
+    Returns (scores fp32 [Q, k], ids int32 [Q, k])."""
+    _cuda(queries, "queries")
+    _cuda(corpus, "corpus")
+    if queries.element_size() != 2 or corpus.element_size() != 2:
+        raise TypeError("queries and corpus must hold bf16 (2-byte) elements")
+    Q, d = queries.shape
+    N, d2 = corpus.shape
+    if d != d2:
+        raise ValueError("dimension mismatch")
+    dev = queries.device
+    if out is None:
+        out = (torch.empty((Q, k), dtype=torch.float32, device=dev),
+               torch.empty((Q, k), dtype=torch.int32, device=dev))
+    scores, ids = out
+    if workspace is None:
+        workspace = torch.empty(hs_retrieve_topk_workspace(Q, N, d, k), dtype=torch.uint8,
+                                device=dev)
+    _check(load().hs_retrieve_topk(_ptr(queries), Q, _ptr(corpus), N, d, k, _ptr(scores),
+                                   _ptr(ids), _ptr(workspace), workspace.numel(), _stream(stream)))
+    return scores, ids
+
+
+def hs_scatter_results(src: torch.Tensor, mapping: torch.Tensor, dst: torch.Tensor | None = None,
+                       stream=None) -> torch.Tensor:
+    """dst[i] = src[mapping[i]] row-wise (rows are the first dimension)."""
+    _cuda(src, "src")
+    _cuda(mapping, "map")
+    if mapping.dtype != torch.int32:
+        raise TypeError("map must be int32")
+    n = mapping.numel()
+    row_bytes = src[0].numel() * src.element_size() if src.dim() > 1 else src.element_size()
+    if dst is None:
+        dst = torch.empty((n,) + tuple(src.shape[1:]), dtype=src.dtype, device=src.device)
+    _check(load().hs_scatter_results(_ptr(src), src.shape[0], row_bytes, _ptr(mapping), n,
+                                     _ptr(dst), _stream(stream)))
+    return dst
+
+
+def hs_get_device_error(stream=None) -> None:
+    """Synchronise the stream; raise HsError if a kernel reported a problem."""
+    _check(load().hs_get_device_error(_stream(stream)))

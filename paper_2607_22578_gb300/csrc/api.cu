@@ -1,0 +1,201 @@
+// C-ABI entry points (include/hs.h): argument validation, workspace checks,
+// the per-device error word, and dispatch to the kernels.
+#include <stdarg.h>
+#include <stdio.h>
+
+#include <mutex>
+
+#include "hs_internal.cuh"
+
+namespace hs {
+
+hs_status launch_fingerprint(const int32_t*, int64_t, int32_t, const int32_t*, uint64_t,
+                             uint64_t*, cudaStream_t);
+size_t unique_inverse_workspace(int64_t);
+hs_status launch_unique_inverse(const uint64_t*, const int32_t*, int64_t, int32_t,
+                                const int32_t*, int32_t*, int32_t*, int32_t*, void*,
+                                cudaStream_t);
+size_t retrieve_topk_workspace(int64_t, int64_t, int32_t, int32_t);
+hs_status launch_retrieve_topk(const uint16_t*, int64_t, const uint16_t*, int64_t, int32_t,
+                               int32_t, float*, int32_t*, void*, size_t, cudaStream_t);
+hs_status launch_scatter(const void*, int64_t, int64_t, const int32_t*, int64_t, void*,
+                         cudaStream_t);
+
+namespace {
+thread_local char g_msg[512] = "";
+constexpr int kMaxDevices = 64;
+__device__ unsigned g_device_error;  // one word per device (module-scope variable)
+unsigned* g_err_addr[kMaxDevices] = {};
+int g_sms[kMaxDevices] = {};
+std::mutex g_mu;
+
+int current_device() {
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return -1;
+  return dev;
+}
+
+bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+void clear_msg() { g_msg[0] = '\0'; }
+}  // namespace
+
+hs_status fail(hs_status s, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_msg, sizeof g_msg, fmt, ap);
+  va_end(ap);
+  return s;
+}
+
+hs_status cuda_fail(cudaError_t e, const char* what) {
+  if (e == cudaSuccess) return HS_OK;
+  return fail(HS_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+unsigned* device_error_word() {
+  const int dev = current_device();
+  if (dev < 0) return nullptr;
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (!g_err_addr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_device_error) != cudaSuccess) return nullptr;
+    g_err_addr[dev] = static_cast<unsigned*>(p);
+  }
+  return g_err_addr[dev];
+}
+
+int num_sms() {
+  const int dev = current_device();
+  if (dev < 0) return 1;
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (!g_sms[dev]) {
+    int v = 0;
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || v < 1)
+      v = 1;
+    g_sms[dev] = v;
+  }
+  return g_sms[dev];
+}
+
+}  // namespace hs
+
+using namespace hs;
+
+extern "C" {
+
+const char* hs_last_error(void) { return g_msg; }
+
+const char* hs_version(void) { return "hs 0.1 (sm_103a)"; }
+
+hs_status hs_fingerprint(const int32_t* tokens, int64_t n_rows, int32_t row_stride,
+                         const int32_t* lens, uint64_t seed_state, uint64_t* fp_out,
+                         hs_stream_t stream) {
+  clear_msg();
+  if (n_rows < 0) return fail(HS_ERR_INVALID_ARG, "n_rows < 0");
+  if (row_stride < 0) return fail(HS_ERR_INVALID_ARG, "row_stride < 0");
+  if (n_rows == 0) return HS_OK;
+  if (!tokens && row_stride > 0) return fail(HS_ERR_INVALID_ARG, "tokens is NULL");
+  if (!fp_out) return fail(HS_ERR_INVALID_ARG, "fp_out is NULL");
+  if (!aligned(tokens, 4) || !aligned(fp_out, 8) || (lens && !aligned(lens, 4)))
+    return fail(HS_ERR_INVALID_ARG, "misaligned pointer (tokens/lens 4 B, fp_out 8 B)");
+  return launch_fingerprint(tokens, n_rows, row_stride, lens, seed_state, fp_out,
+                            reinterpret_cast<cudaStream_t>(stream));
+}
+
+size_t hs_unique_inverse_workspace(int64_t n_rows) { return unique_inverse_workspace(n_rows); }
+
+hs_status hs_unique_inverse(const uint64_t* fp, const int32_t* tokens, int64_t n_rows,
+                            int32_t row_stride, const int32_t* lens, int32_t* n_unique_dev,
+                            int32_t* unique_idx_out, int32_t* inverse_out, void* workspace,
+                            size_t workspace_bytes, hs_stream_t stream) {
+  clear_msg();
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (n_rows < 0 || n_rows > (int64_t)((1u << 30) - 1))
+    return fail(HS_ERR_INVALID_ARG, "n_rows outside [0, 2^30 - 1]");
+  if (row_stride < 0) return fail(HS_ERR_INVALID_ARG, "row_stride < 0");
+  if (!n_unique_dev) return fail(HS_ERR_INVALID_ARG, "n_unique_dev is NULL");
+  if (!aligned(n_unique_dev, 4)) return fail(HS_ERR_INVALID_ARG, "n_unique_dev misaligned");
+  if (n_rows == 0) return cuda_fail(cudaMemsetAsync(n_unique_dev, 0, sizeof(int32_t), s),
+                                    "n_unique clear");
+  if (!fp || !unique_idx_out || !inverse_out || (!tokens && row_stride > 0))
+    return fail(HS_ERR_INVALID_ARG, "NULL input or output pointer");
+  if (!aligned(fp, 8) || !aligned(tokens, 4) || (lens && !aligned(lens, 4)) ||
+      !aligned(unique_idx_out, 4) || !aligned(inverse_out, 4))
+    return fail(HS_ERR_INVALID_ARG, "misaligned pointer");
+  const size_t need = unique_inverse_workspace(n_rows);
+  if (!workspace || !aligned(workspace, 256))
+    return fail(HS_ERR_WORKSPACE, "workspace NULL or not 256-byte aligned");
+  if (workspace_bytes < need)
+    return fail(HS_ERR_WORKSPACE, "unique workspace too small: %zu < %zu", workspace_bytes, need);
+  return launch_unique_inverse(fp, tokens, n_rows, row_stride, lens, n_unique_dev,
+                               unique_idx_out, inverse_out, workspace, s);
+}
+
+size_t hs_retrieve_topk_workspace(int64_t n_queries, int64_t n_corpus, int32_t dim, int32_t k) {
+  return retrieve_topk_workspace(n_queries, n_corpus, dim, k);
+}
+
+hs_status hs_retrieve_topk(const uint16_t* queries, int64_t n_queries, const uint16_t* corpus,
+                           int64_t n_corpus, int32_t dim, int32_t k, float* scores_out,
+                           int32_t* ids_out, void* workspace, size_t workspace_bytes,
+                           hs_stream_t stream) {
+  clear_msg();
+  if (n_queries < 0) return fail(HS_ERR_INVALID_ARG, "n_queries < 0");
+  if (n_corpus < 1 || n_corpus > 0x7fffffffLL)
+    return fail(HS_ERR_INVALID_ARG, "n_corpus outside [1, 2^31 - 1]");
+  if (dim < 8 || dim % 8 != 0) return fail(HS_ERR_INVALID_ARG, "dim must be >= 8 and a multiple of 8");
+  if (k < 1 || (int64_t)k > n_corpus || k > HS_TOPK_MAX_K)
+    return fail(HS_ERR_INVALID_ARG, "k outside [1, min(n_corpus, %d)]", HS_TOPK_MAX_K);
+  if (n_queries == 0) return HS_OK;
+  if (n_queries > 0x7fffffffLL) return fail(HS_ERR_INVALID_ARG, "n_queries >= 2^31");
+  if (!queries || !corpus || !scores_out || !ids_out)
+    return fail(HS_ERR_INVALID_ARG, "NULL input or output pointer");
+  if (!aligned(queries, 16) || !aligned(corpus, 16))
+    return fail(HS_ERR_INVALID_ARG, "queries/corpus must be 16-byte aligned");
+  if (!aligned(scores_out, 4) || !aligned(ids_out, 4))
+    return fail(HS_ERR_INVALID_ARG, "scores_out/ids_out misaligned");
+  if (!workspace || !aligned(workspace, 256))
+    return fail(HS_ERR_WORKSPACE, "workspace NULL or not 256-byte aligned");
+  return launch_retrieve_topk(queries, n_queries, corpus, n_corpus, dim, k, scores_out, ids_out,
+                              workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream));
+}
+
+hs_status hs_scatter_results(const void* src, int64_t n_src, int64_t row_bytes,
+                             const int32_t* map, int64_t n_rows, void* dst, hs_stream_t stream) {
+  clear_msg();
+  if (n_rows < 0 || n_src < 0) return fail(HS_ERR_INVALID_ARG, "negative row count");
+  if (row_bytes < 1 || row_bytes > 0x7fffffffLL)
+    return fail(HS_ERR_INVALID_ARG, "row_bytes outside [1, 2^31 - 1]");
+  if (n_rows == 0) return HS_OK;
+  if (!src || !map || !dst) return fail(HS_ERR_INVALID_ARG, "NULL pointer");
+  if (!aligned(map, 4)) return fail(HS_ERR_INVALID_ARG, "map misaligned");
+  const uintptr_t s0 = reinterpret_cast<uintptr_t>(src), d0 = reinterpret_cast<uintptr_t>(dst);
+  const uintptr_t s1 = s0 + (uintptr_t)(n_src * row_bytes), d1 = d0 + (uintptr_t)(n_rows * row_bytes);
+  if (s0 < d1 && d0 < s1) return fail(HS_ERR_INVALID_ARG, "src and dst overlap");
+  return launch_scatter(src, n_src, row_bytes, map, n_rows, dst,
+                        reinterpret_cast<cudaStream_t>(stream));
+}
+
+hs_status hs_get_device_error(hs_stream_t stream) {
+  clear_msg();
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return cuda_fail(e, "stream synchronize");
+  unsigned* addr = device_error_word();
+  if (!addr) return fail(HS_ERR_CUDA, "could not resolve the device error word");
+  unsigned v = 0;
+  e = cudaMemcpy(&v, addr, sizeof v, cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e, "error word read");
+  if (v) {
+    const unsigned zero = 0;
+    e = cudaMemcpy(addr, &zero, sizeof zero, cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return cuda_fail(e, "error word clear");
+  }
+  if (v & kErrTimeout) return fail(HS_ERR_TIMEOUT, "a bounded device wait ran out");
+  if (v & kErrInvalidArg)
+    return fail(HS_ERR_INVALID_ARG, "a kernel saw invalid data (row length or map entry)");
+  return HS_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,529 @@
+// K6/K7: dense retrieval with a fused per-query top-k — the vector-retrieval
+// node shared by merged queries (Section 4.1, "Workloads": embed, retrieve the
+// top-k chunks; Section 3.3: merged nodes execute once).
+//
+//   S = Q * C^T   (bf16 x bf16 -> fp32), per query keep the k best (S, j),
+//   ordered by score descending, ties to the lower corpus index j.
+//
+// K6 (retrieve_kernel) is a persistent, warp-specialised tcgen05 kernel:
+//   warp 0      TMA producer: 128x64 query tile + 256x64 corpus tile per
+//               stage, 128-byte swizzle, 4-stage mbarrier ring;
+//   warp 1      MMA issuer: 4 x tcgen05.mma (M=128, N=256, K=16) per stage
+//               into a double-buffered fp32 accumulator in tensor memory
+//               (2 x 256 columns), tcgen05.commit releases smem stages;
+//   warps 2-5   epilogue: tcgen05.ld of the 128 x 256 score tile, one thread
+//               per query (TMEM lane), threshold filter + per-query top-k.
+// The Q x N score matrix never leaves the SM.  Work is split into units
+// (query block, corpus split); units that share a corpus split run at the
+// same time on different SMs, so each corpus tile is read from HBM about once
+// and served to the other query blocks from L2.
+//
+// Top-k state per query: for k <= 32 a sorted list in registers (KREG = 16
+// or 32 slots); for larger k a 32-entry candidate buffer in shared memory
+// that is sorted and merged into a sorted list in global scratch whenever a
+// query's buffer fills.  Each unit writes its k best per query; K7 merges the
+// splits of each query with a bitonic sort of packed (score, index) keys.
+#include <float.h>
+
+#include "hs_internal.cuh"
+
+namespace hs {
+namespace {
+
+constexpr int BM = 128;               // queries per tile: UMMA M = TMEM lanes
+constexpr int BN = 256;               // corpus rows per tile: UMMA N
+constexpr int BK = 64;                // K per stage: one 128-byte swizzle row
+constexpr int UK = 16;                // K per tcgen05.mma, kind::f16
+constexpr int kStages = 4;
+constexpr int kThreads = 192;
+constexpr int kEpi = 128;
+constexpr uint32_t kABytes = BM * BK * 2;
+constexpr uint32_t kBBytes = BN * BK * 2;
+constexpr uint32_t kStageBytes = kABytes + kBBytes;
+constexpr uint32_t kTmemCols = 2 * BN;
+constexpr int kCap = 32;              // candidate buffer per query (large-k path)
+constexpr int kMergeMax = 16384;      // nsplit * k bound for K7
+constexpr size_t kBarBytes = 256;
+constexpr size_t kSmemKReg = 1024 + (size_t)kStages * kStageBytes + kBarBytes;
+constexpr size_t kSmemLarge = kSmemKReg + (size_t)kCap * kEpi * 8;
+
+struct Params {
+  int64_t Q, N, tiles;
+  int32_t k, kb_count, qblocks, nsplit;
+  float* part_s;     // [Q][nsplit][k]
+  int32_t* part_i;
+  float* list_s;     // large-k: [grid][kEpi][2][k]
+  int32_t* list_i;
+  unsigned* err;
+};
+
+__device__ __forceinline__ void unit_coords(const Params& p, int64_t u, int& qb, int& split,
+                                            int64_t& t0, int64_t& t1) {
+  qb = (int)(u % p.qblocks);
+  split = (int)(u / p.qblocks);
+  t0 = (int64_t)split * p.tiles / p.nsplit;
+  t1 = (int64_t)(split + 1) * p.tiles / p.nsplit;
+}
+
+// ---- large-k helpers (per thread, serial) ---------------------------------------------
+__device__ void flush_candidates(float* cs, int32_t* ci, int et, int& cnt, float* Ls, int32_t* Li,
+                                 int k, int& cur, float& theta) {
+  if (cnt == 0) return;
+  // Stable insertion sort of the buffer, score descending (buffer order is
+  // ascending corpus index, so ties keep the lower index first).
+  for (int a = 1; a < cnt; ++a) {
+    const float s = cs[a * kEpi + et];
+    const int32_t i = ci[a * kEpi + et];
+    int b = a - 1;
+    while (b >= 0 && s > cs[b * kEpi + et]) {
+      cs[(b + 1) * kEpi + et] = cs[b * kEpi + et];
+      ci[(b + 1) * kEpi + et] = ci[b * kEpi + et];
+      --b;
+    }
+    cs[(b + 1) * kEpi + et] = s;
+    ci[(b + 1) * kEpi + et] = i;
+  }
+  // Merge with the current list (all of whose entries have lower corpus
+  // indices: on equal scores the list entry wins).
+  const float* As = Ls + (size_t)cur * k;
+  const int32_t* Ai = Li + (size_t)cur * k;
+  float* Os = Ls + (size_t)(cur ^ 1) * k;
+  int32_t* Oi = Li + (size_t)(cur ^ 1) * k;
+  int a = 0, b = 0;
+  for (int o = 0; o < k; ++o) {
+    const float sb = b < cnt ? cs[b * kEpi + et] : -FLT_MAX;
+    const float sa = As[a];
+    if (b < cnt && sb > sa) {
+      Os[o] = sb;
+      Oi[o] = ci[b * kEpi + et];
+      ++b;
+    } else {
+      Os[o] = sa;
+      Oi[o] = Ai[a];
+      ++a;
+    }
+  }
+  cur ^= 1;
+  theta = Os[k - 1];
+  cnt = 0;
+}
+
+template <int KREG>
+__global__ void __launch_bounds__(kThreads, 1)
+    retrieve_kernel(const __grid_constant__ CUtensorMap tmap_q,
+                    const __grid_constant__ CUtensorMap tmap_c, const Params p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + kStages * kABytes;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kStages * kStageBytes);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + kStages;
+  uint64_t* tfull = bars + 2 * kStages;
+  uint64_t* tempty = tfull + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + 2);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  float* cand_s = reinterpret_cast<float*>(smem + kStages * kStageBytes + kBarBytes);
+  int32_t* cand_i = reinterpret_cast<int32_t*>(cand_s + kCap * kEpi);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(full + s, 1);
+      mbar_init(empty + s, 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(tfull + a, 1);
+      mbar_init(tempty + a, 4);
+    }
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    prefetch_tmap(&tmap_q);
+    prefetch_tmap(&tmap_c);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const int64_t units = (int64_t)p.qblocks * p.nsplit;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      const uint64_t pol_c = policy_evict_first();
+      const uint64_t pol_q = policy_evict_last();
+      uint32_t stage = 0, phase = 0;
+      for (int64_t u = blockIdx.x; u < units; u += gridDim.x) {
+        int qb, split;
+        int64_t t0, t1;
+        unit_coords(p, u, qb, split, t0, t1);
+        for (int64_t t = t0; t < t1; ++t) {
+          for (int kb = 0; kb < p.kb_count; ++kb) {
+            if (!mbar_wait(empty + stage, phase ^ 1u, abort_flag)) goto producer_done;
+            mbar_arrive_expect_tx(full + stage, kStageBytes);
+            tma_load_2d_hint(sA + stage * kABytes, &tmap_q, full + stage, kb * BK, qb * BM, pol_q);
+            tma_load_2d_hint(sB + stage * kBBytes, &tmap_c, full + stage, kb * BK,
+                             (int32_t)(t * BN), pol_c);
+            if (++stage == kStages) {
+              stage = 0;
+              phase ^= 1u;
+            }
+          }
+        }
+      }
+    producer_done:;
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_bf16_f32(BM, BN);
+      uint32_t stage = 0, phase = 0, tile_i = 0;
+      for (int64_t u = blockIdx.x; u < units; u += gridDim.x) {
+        int qb, split;
+        int64_t t0, t1;
+        unit_coords(p, u, qb, split, t0, t1);
+        for (int64_t t = t0; t < t1; ++t, ++tile_i) {
+          const uint32_t acc = tile_i & 1u, aphase = (tile_i >> 1) & 1u;
+          if (!mbar_wait(tempty + acc, aphase ^ 1u, abort_flag)) goto mma_done;
+          tc_fence_after();
+          const uint32_t d_tmem = tmem_base + acc * BN;
+          for (int kb = 0; kb < p.kb_count; ++kb) {
+            if (!mbar_wait(full + stage, phase, abort_flag)) goto mma_done;
+            tc_fence_after();
+            const uint64_t a0 = smem_desc_k_sw128(smem_u32(sA + stage * kABytes));
+            const uint64_t b0 = smem_desc_k_sw128(smem_u32(sB + stage * kBBytes));
+#pragma unroll
+            for (int kk = 0; kk < BK / UK; ++kk)
+              umma_bf16(d_tmem, a0 + (uint64_t)(kk * UK * 2 / 16), b0 + (uint64_t)(kk * UK * 2 / 16),
+                        idesc, (kb | kk) != 0 ? 1u : 0u);
+            umma_commit(empty + stage);
+            if (++stage == kStages) {
+              stage = 0;
+              phase ^= 1u;
+            }
+          }
+          umma_commit(tfull + acc);
+        }
+      }
+    mma_done:;
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int quarter = warp & 3;  // TMEM lanes [32*quarter, 32*quarter+32)
+    const int et = quarter * 32 + lane;
+    const uint32_t lane_addr = (uint32_t)(quarter * 32) << 16;
+    const int k = p.k;
+    uint32_t tile_i = 0;
+    float* Ls = p.list_s + ((size_t)blockIdx.x * kEpi + et) * 2 * (size_t)k;
+    int32_t* Li = p.list_i + ((size_t)blockIdx.x * kEpi + et) * 2 * (size_t)k;
+    for (int64_t u = blockIdx.x; u < units; u += gridDim.x) {
+      int qb, split;
+      int64_t t0, t1;
+      unit_coords(p, u, qb, split, t0, t1);
+      const int64_t q = (int64_t)qb * BM + et;
+      const bool valid_q = q < p.Q;
+      float theta = -FLT_MAX;
+      float ls[KREG > 0 ? KREG : 1];
+      int32_t li[KREG > 0 ? KREG : 1];
+      int cnt = 0, cur = 0;
+      if (KREG > 0) {
+#pragma unroll
+        for (int i = 0; i < (KREG > 0 ? KREG : 1); ++i) {
+          ls[i] = -FLT_MAX;
+          li[i] = -1;
+        }
+      } else if (valid_q) {
+        for (int i = 0; i < k; ++i) {
+          Ls[i] = -FLT_MAX;
+          Li[i] = -1;
+        }
+      }
+      for (int64_t t = t0; t < t1; ++t, ++tile_i) {
+        const uint32_t acc = tile_i & 1u, aphase = (tile_i >> 1) & 1u;
+        if (!mbar_wait(tfull + acc, aphase, abort_flag)) goto epi_done;
+        tc_fence_after();
+        const int64_t col0 = t * BN;
+        const bool tail = col0 + BN > p.N;
+#pragma unroll 1
+        for (int c = 0; c < BN / 32; ++c) {
+          uint32_t r[32];
+          tmem_ld_32x32b_x32(tmem_base + lane_addr + acc * BN + c * 32, r);
+          tmem_ld_wait();
+          const int32_t cbase = (int32_t)(col0 + c * 32);
+          if (KREG > 0) {
+            if (valid_q) {
+#pragma unroll
+              for (int j = 0; j < 32; ++j) {
+                const float s = __uint_as_float(r[j]);
+                if (s > theta && (!tail || (int64_t)(cbase + j) < p.N)) {
+                  const int32_t idx = cbase + j;
+#pragma unroll
+                  for (int i = (KREG > 0 ? KREG : 1) - 1; i > 0; --i) {
+                    const bool up = s > ls[i - 1];
+                    const bool here = !up && s > ls[i];
+                    ls[i] = up ? ls[i - 1] : (here ? s : ls[i]);
+                    li[i] = up ? li[i - 1] : (here ? idx : li[i]);
+                  }
+                  if (s > ls[0]) {
+                    ls[0] = s;
+                    li[0] = idx;
+                  }
+                  theta = ls[(KREG > 0 ? KREG : 1) - 1];
+                }
+              }
+            }
+          } else {
+#pragma unroll
+            for (int j0 = 0; j0 < 32; j0 += 8) {
+              if (valid_q) {
+#pragma unroll
+                for (int j = j0; j < j0 + 8; ++j) {
+                  const float s = __uint_as_float(r[j]);
+                  if (s > theta && (!tail || (int64_t)(cbase + j) < p.N)) {
+                    cand_s[cnt * kEpi + et] = s;
+                    cand_i[cnt * kEpi + et] = cbase + j;
+                    ++cnt;
+                  }
+                }
+              }
+              if (__any_sync(0xffffffffu, cnt > kCap - 8))
+                flush_candidates(cand_s, cand_i, et, cnt, Ls, Li, k, cur, theta);
+            }
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(tempty + acc);
+      }
+      if (valid_q) {
+        float* os = p.part_s + ((size_t)q * p.nsplit + split) * k;
+        int32_t* oi = p.part_i + ((size_t)q * p.nsplit + split) * k;
+        if (KREG > 0) {
+#pragma unroll
+          for (int i = 0; i < (KREG > 0 ? KREG : 1); ++i)
+            if (i < k) {
+              os[i] = ls[i];
+              oi[i] = li[i];
+            }
+        } else {
+          flush_candidates(cand_s, cand_i, et, cnt, Ls, Li, k, cur, theta);
+          for (int i = 0; i < k; ++i) {
+            os[i] = Ls[(size_t)cur * k + i];
+            oi[i] = Li[(size_t)cur * k + i];
+          }
+        }
+      }
+    }
+  epi_done:;
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem_base, kTmemCols);
+  }
+  if (threadIdx.x == 0 && *abort_flag) set_error(p.err, kErrTimeout);
+}
+
+// ---- K7: merge of the per-split lists ----------------------------------------------------
+__device__ __forceinline__ uint64_t pack_key(float s, int32_t idx) {
+  uint32_t u = __float_as_uint(s);
+  u = (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+  return ((uint64_t)u << 32) | (uint64_t)(0xffffffffu - (uint32_t)idx);
+}
+
+__device__ __forceinline__ void unpack_key(uint64_t key, float& s, int32_t& idx) {
+  uint32_t u = (uint32_t)(key >> 32);
+  u = (u & 0x80000000u) ? (u ^ 0x80000000u) : ~u;
+  s = __uint_as_float(u);
+  idx = (int32_t)(0xffffffffu - (uint32_t)key);
+}
+
+__global__ void __launch_bounds__(256) merge_kernel(const float* __restrict__ part_s,
+                                                    const int32_t* __restrict__ part_i, int64_t Q,
+                                                    int32_t nsplit, int32_t k, int32_t p2,
+                                                    float* __restrict__ out_s,
+                                                    int32_t* __restrict__ out_i) {
+  extern __shared__ uint64_t keys[];
+  const int m = nsplit * k;
+  for (int64_t q = blockIdx.x; q < Q; q += gridDim.x) {
+    const float* ps = part_s + (size_t)q * m;
+    const int32_t* pi = part_i + (size_t)q * m;
+    for (int e = threadIdx.x; e < p2; e += blockDim.x) keys[e] = e < m ? pack_key(ps[e], pi[e]) : 0ull;
+    __syncthreads();
+    // Bitonic sort, descending.
+    for (int size = 2; size <= p2; size <<= 1) {
+      for (int stride = size >> 1; stride > 0; stride >>= 1) {
+        for (int t = threadIdx.x; t < (p2 >> 1); t += blockDim.x) {
+          const int lo = 2 * t - (t & (stride - 1));
+          const int hi = lo + stride;
+          const bool desc = (lo & size) == 0;
+          const uint64_t a = keys[lo], b = keys[hi];
+          if ((a < b) == desc) {
+            keys[lo] = b;
+            keys[hi] = a;
+          }
+        }
+        __syncthreads();
+      }
+    }
+    for (int j = threadIdx.x; j < k; j += blockDim.x) {
+      float s;
+      int32_t idx;
+      unpack_key(keys[j], s, idx);
+      out_s[(size_t)q * k + j] = s;
+      out_i[(size_t)q * k + j] = idx;
+    }
+    __syncthreads();
+  }
+}
+
+// ---- host side ---------------------------------------------------------------------------
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+bool make_map(CUtensorMap* map, const uint16_t* base, int64_t rows, int32_t d, uint32_t box_rows) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  const cuuint64_t dims[2] = {(cuuint64_t)d, (cuuint64_t)rows};
+  const cuuint64_t strides[1] = {(cuuint64_t)d * 2};
+  const cuuint32_t box[2] = {(cuuint32_t)BK, box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<uint16_t*>(base), dims, strides,
+            box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+int64_t gcd64(int64_t a, int64_t b) {
+  while (b) {
+    const int64_t t = a % b;
+    a = b;
+    b = t;
+  }
+  return a;
+}
+
+struct Plan {
+  int32_t qblocks, nsplit, kreg, p2;
+  int64_t tiles, grid;
+  size_t part_bytes, list_bytes, total;
+};
+
+Plan plan(int64_t Q, int64_t N, int32_t d, int32_t k) {
+  Plan pl{};
+  const int64_t sms = num_sms();
+  pl.qblocks = (int32_t)((Q + BM - 1) / BM);
+  pl.tiles = (N + BN - 1) / BN;
+  int64_t ns = sms / gcd64(sms, pl.qblocks > 0 ? pl.qblocks : 1);
+  if (ns > pl.tiles) ns = pl.tiles;
+  if (ns > kMergeMax / k) ns = kMergeMax / k;
+  if (ns < 1) ns = 1;
+  pl.nsplit = (int32_t)ns;
+  pl.kreg = k <= 16 ? 16 : (k <= 32 ? 32 : 0);
+  int p2 = 1;
+  while (p2 < pl.nsplit * k) p2 <<= 1;
+  pl.p2 = p2;
+  const int64_t units = (int64_t)pl.qblocks * pl.nsplit;
+  pl.grid = units < sms ? units : sms;
+  pl.part_bytes = (((size_t)Q * pl.nsplit * k * 4) + 255) & ~(size_t)255;
+  pl.list_bytes = pl.kreg ? 0 : ((((size_t)pl.grid * kEpi * 2 * k * 4) + 255) & ~(size_t)255);
+  pl.total = 2 * pl.part_bytes + 2 * pl.list_bytes + 256;
+  return pl;
+}
+
+template <int KREG>
+hs_status launch_kernel(const CUtensorMap& mq, const CUtensorMap& mc, const Params& prm,
+                        int64_t grid, cudaStream_t stream) {
+  const size_t smem = KREG > 0 ? kSmemKReg : kSmemLarge;
+  static bool configured = false;
+  if (!configured) {
+    cudaError_t e = cudaFuncSetAttribute(retrieve_kernel<KREG>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return cuda_fail(e, "retrieve smem attribute");
+    configured = true;
+  }
+  retrieve_kernel<KREG><<<(unsigned)grid, kThreads, smem, stream>>>(mq, mc, prm);
+  return cuda_fail(cudaGetLastError(), "retrieve launch");
+}
+
+}  // namespace
+
+size_t retrieve_topk_workspace(int64_t Q, int64_t N, int32_t d, int32_t k) {
+  if (Q <= 0 || N <= 0 || k <= 0) return 256;
+  return plan(Q, N, d, k).total;
+}
+
+hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Q, const uint16_t* corpus,
+                               int64_t N, int32_t d, int32_t k, float* scores_out,
+                               int32_t* ids_out, void* ws, size_t ws_bytes,
+                               cudaStream_t stream) {
+  unsigned* err = device_error_word();
+  if (!err) return fail(HS_ERR_CUDA, "could not resolve the device error word");
+  const Plan pl = plan(Q, N, d, k);
+  if (ws_bytes < pl.total)
+    return fail(HS_ERR_WORKSPACE, "retrieve workspace too small: %zu < %zu", ws_bytes, pl.total);
+  CUtensorMap mq, mc;
+  if (!make_map(&mq, queries, Q, d, BM) || !make_map(&mc, corpus, N, d, BN))
+    return fail(HS_ERR_CUDA, "cuTensorMapEncodeTiled failed (driver entry point or arguments)");
+  char* w = static_cast<char*>(ws);
+  Params prm{};
+  prm.Q = Q;
+  prm.N = N;
+  prm.tiles = pl.tiles;
+  prm.k = k;
+  prm.kb_count = (d + BK - 1) / BK;
+  prm.qblocks = pl.qblocks;
+  prm.nsplit = pl.nsplit;
+  prm.part_s = reinterpret_cast<float*>(w);
+  prm.part_i = reinterpret_cast<int32_t*>(w + pl.part_bytes);
+  prm.list_s = reinterpret_cast<float*>(w + 2 * pl.part_bytes);
+  prm.list_i = reinterpret_cast<int32_t*>(w + 2 * pl.part_bytes + pl.list_bytes);
+  prm.err = err;
+  hs_status st;
+  if (pl.kreg == 16)
+    st = launch_kernel<16>(mq, mc, prm, pl.grid, stream);
+  else if (pl.kreg == 32)
+    st = launch_kernel<32>(mq, mc, prm, pl.grid, stream);
+  else
+    st = launch_kernel<0>(mq, mc, prm, pl.grid, stream);
+  if (st != HS_OK) return st;
+  const size_t msmem = (size_t)pl.p2 * 8;
+  static size_t merge_configured = 0;
+  if (msmem > 48 * 1024 && msmem > merge_configured) {
+    cudaError_t e = cudaFuncSetAttribute(merge_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)msmem);
+    if (e != cudaSuccess) return cuda_fail(e, "merge smem attribute");
+    merge_configured = msmem;
+  }
+  int64_t mgrid = Q < (int64_t)num_sms() * 8 ? Q : (int64_t)num_sms() * 8;
+  merge_kernel<<<(unsigned)mgrid, 256, msmem, stream>>>(prm.part_s, prm.part_i, Q, pl.nsplit, k,
+                                                        pl.p2, scores_out, ids_out);
+  return cuda_fail(cudaGetLastError(), "merge launch");
+}
+
+}  // namespace hs

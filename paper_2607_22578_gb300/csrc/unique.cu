@@ -1,0 +1,521 @@
+// K2-K4: exact unique-with-inverse over fingerprinted rows — the merge step of
+// topological fusion within a time window (Section 3.3, "Dynamic Fusion and
+// Reuse Mechanism" (I)) and the merge sets M(v*) of Appendix A.2.
+//
+// Pipeline (all on the caller's stream, no host synchronisation):
+//   1. histogram of all eight 8-bit digits of the fingerprints (one pass);
+//   2. eight stable LSD radix passes over (fingerprint, row index), each a
+//      single kernel with decoupled look-back across tiles (bounded spins);
+//      stability keeps equal fingerprints in ascending row order, so each
+//      run of equal fingerprints starts with its smallest row index;
+//   3. segment heads: inclusive max-scan of "fingerprint differs from the
+//      previous one" positions;
+//   4. verify: every non-head row is compared in full (length + tokens) with
+//      its segment head by one warp; equal rows take the head as their
+//      representative, a mismatch marks the segment as collided;
+//   5. collided segments only: exact regrouping by repeated peeling (the
+//      first unassigned row becomes a representative, all rows equal to it
+//      join it);
+//   6. exclusive sum-scan of "row is its own representative" gives each
+//      group its ordinal in first-occurrence order; the final kernel writes
+//      unique_idx and inverse.
+#include "hs_internal.cuh"
+
+namespace hs {
+namespace {
+
+constexpr int kSortThreads = 256;
+constexpr int kSortItems = 16;
+constexpr int kSortTile = kSortThreads * kSortItems;  // 4096 keys per tile
+constexpr int kPasses = 8;
+constexpr uint32_t kFlagA = 1u << 30;  // tile aggregate published
+constexpr uint32_t kFlagP = 2u << 30;  // inclusive prefix published
+constexpr uint32_t kValMask = (1u << 30) - 1u;
+
+constexpr int kScanThreads = 256;
+constexpr int kScanItems = 16;
+constexpr int kScanTile = kScanThreads * kScanItems;
+
+constexpr size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+struct Layout {
+  // zero-initialised region first
+  size_t hist, status, ctr, coll_flag, coll_count, scan_status0, scan_status1, zero_end;
+  size_t keys0, keys1, vals0, vals1, seg_head, rep, uid, coll_list, total;
+};
+
+Layout layout(int64_t n) {
+  Layout L{};
+  const int64_t sort_tiles = (n + kSortTile - 1) / kSortTile;
+  const int64_t scan_tiles = (n + kScanTile - 1) / kScanTile;
+  size_t o = 0;
+  L.hist = o;          o += align256(sizeof(uint32_t) * kPasses * 256);
+  L.status = o;        o += align256(sizeof(uint32_t) * kPasses * 256 * (size_t)sort_tiles);
+  L.ctr = o;           o += align256(sizeof(uint32_t) * 16);
+  L.coll_flag = o;     o += align256(sizeof(int32_t) * (size_t)n);
+  L.coll_count = o;    o += align256(sizeof(uint32_t));
+  L.scan_status0 = o;  o += align256(sizeof(uint64_t) * (size_t)scan_tiles);
+  L.scan_status1 = o;  o += align256(sizeof(uint64_t) * (size_t)scan_tiles);
+  L.zero_end = o;
+  L.keys0 = o;         o += align256(sizeof(uint64_t) * (size_t)n);
+  L.keys1 = o;         o += align256(sizeof(uint64_t) * (size_t)n);
+  L.vals0 = o;         o += align256(sizeof(uint32_t) * (size_t)n);
+  L.vals1 = o;         o += align256(sizeof(uint32_t) * (size_t)n);
+  L.seg_head = o;      o += align256(sizeof(int32_t) * (size_t)n);
+  L.rep = o;           o += align256(sizeof(int32_t) * (size_t)n);
+  L.uid = o;           o += align256(sizeof(int32_t) * (size_t)n);
+  L.coll_list = o;     o += align256(sizeof(int32_t) * (size_t)n);
+  L.total = o;
+  return L;
+}
+
+// Bounded spin on a 32-bit status word until its flag bits are non-zero.
+__device__ __forceinline__ uint32_t wait_flag32(const volatile uint32_t* p, unsigned* err) {
+  uint32_t s = *p;
+  if (s & ~kValMask) return s;
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t it = 1;; ++it) {
+    s = *p;
+    if (s & ~kValMask) return s;
+    if ((it & 31u) == 0) {
+      __nanosleep(64);
+      if (globaltimer_ns() - t0 > kWaitLimitNs) {
+        set_error(err, kErrTimeout);
+        return kFlagP;  // give up: treat as a zero prefix
+      }
+    }
+  }
+}
+
+__device__ __forceinline__ uint64_t wait_flag64(const volatile unsigned long long* p,
+                                                unsigned* err) {
+  unsigned long long s = *p;
+  if (s >> 32) return s;
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t it = 1;; ++it) {
+    s = *p;
+    if (s >> 32) return s;
+    if ((it & 31u) == 0) {
+      __nanosleep(64);
+      if (globaltimer_ns() - t0 > kWaitLimitNs) {
+        set_error(err, kErrTimeout);
+        return 2ull << 32;
+      }
+    }
+  }
+}
+
+// ---- 1. digit histograms ---------------------------------------------------------------
+__global__ void __launch_bounds__(256) sort_hist_kernel(const uint64_t* __restrict__ fp, int64_t n,
+                                                        uint32_t* __restrict__ hist) {
+  __shared__ uint32_t h[kPasses * 256];
+  for (int i = threadIdx.x; i < kPasses * 256; i += blockDim.x) h[i] = 0;
+  __syncthreads();
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    const uint64_t k = __ldg(fp + e);
+#pragma unroll
+    for (int p = 0; p < kPasses; ++p) atomicAdd(&h[p * 256 + ((k >> (8 * p)) & 0xff)], 1u);
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < kPasses * 256; i += blockDim.x)
+    if (h[i]) atomicAdd(&hist[i], h[i]);
+}
+
+// ---- 2. one stable radix pass ----------------------------------------------------------------
+// Tile t holds keys [t*4096, (t+1)*4096); warp w of the tile owns the 512 keys
+// [w*512, (w+1)*512), read striped (item i of lane l is key w*512 + i*32 + l),
+// so processing items in order with lanes in order follows the input order.
+__global__ void __launch_bounds__(kSortThreads) onesweep_kernel(
+    int pass, const uint64_t* __restrict__ keys_in, const uint32_t* __restrict__ vals_in,
+    uint64_t* __restrict__ keys_out, uint32_t* __restrict__ vals_out, int64_t n,
+    const uint32_t* __restrict__ hist, uint32_t* status, uint32_t* tile_ctr, unsigned* err) {
+  __shared__ uint32_t s_tile;
+  __shared__ uint32_t warp_cnt[kSortThreads / 32][256];
+  __shared__ uint32_t digit_base[256];
+  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+  if (tid == 0) s_tile = atomicAdd(tile_ctr + pass, 1u);
+  for (int i = tid; i < (kSortThreads / 32) * 256; i += kSortThreads) (&warp_cnt[0][0])[i] = 0;
+  // Exclusive scan of this pass's global digit counts (thread = digit).
+  {
+    const uint32_t c = hist[pass * 256 + tid];
+    uint32_t x = c;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t y = __shfl_up_sync(0xffffffffu, x, o);
+      if (lane >= o) x += y;
+    }
+    __shared__ uint32_t wsum[8];
+    if (lane == 31) wsum[w] = x;
+    __syncthreads();
+    uint32_t add = 0;
+    for (int i = 0; i < w; ++i) add += wsum[i];
+    digit_base[tid] = add + x - c;
+  }
+  __syncthreads();
+  const uint32_t tile = s_tile;
+  const int64_t base = (int64_t)tile * kSortTile + w * (kSortItems * 32);
+  const int shift = 8 * pass;
+
+  uint64_t k[kSortItems];
+  uint32_t v[kSortItems];
+  uint32_t rank[kSortItems];
+#pragma unroll
+  for (int i = 0; i < kSortItems; ++i) {
+    const int64_t e = base + i * 32 + lane;
+    if (e < n) {
+      k[i] = keys_in[e];
+      v[i] = vals_in ? vals_in[e] : (uint32_t)e;
+    } else {
+      k[i] = 0;
+      v[i] = 0;
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < kSortItems; ++i) {
+    const int64_t e = base + i * 32 + lane;
+    const bool valid = e < n;
+    const uint32_t d = valid ? (uint32_t)((k[i] >> shift) & 0xff) : 256u + lane;
+    const uint32_t peers = __match_any_sync(0xffffffffu, d);
+    const uint32_t before = valid ? warp_cnt[w][d] : 0u;
+    rank[i] = before + __popc(peers & lanemask_lt());
+    __syncwarp();
+    if (valid && (__ffs(peers) - 1) == lane) warp_cnt[w][d] = before + __popc(peers);
+    __syncwarp();
+  }
+  __syncthreads();
+  // Thread = digit: turn per-warp counts into per-warp exclusive offsets.
+  uint32_t tile_count = 0;
+#pragma unroll
+  for (int ww = 0; ww < kSortThreads / 32; ++ww) {
+    const uint32_t c = warp_cnt[ww][tid];
+    warp_cnt[ww][tid] = tile_count;
+    tile_count += c;
+  }
+  // Publish, look back, publish the inclusive prefix.
+  volatile uint32_t* st = status + (size_t)pass * 256 * gridDim.x;
+  uint32_t prefix = 0;
+  if (tile == 0) {
+    st[tid] = kFlagP | tile_count;
+  } else {
+    st[(size_t)tile * 256 + tid] = kFlagA | tile_count;
+    for (int64_t j = (int64_t)tile - 1; j >= 0; --j) {
+      const uint32_t s = wait_flag32(st + (size_t)j * 256 + tid, err);
+      prefix += s & kValMask;
+      if ((s & ~kValMask) == kFlagP) break;
+    }
+    st[(size_t)tile * 256 + tid] = kFlagP | ((prefix + tile_count) & kValMask);
+  }
+  digit_base[tid] += prefix;
+  __syncthreads();
+#pragma unroll
+  for (int i = 0; i < kSortItems; ++i) {
+    const int64_t e = base + i * 32 + lane;
+    if (e < n) {
+      const uint32_t d = (uint32_t)((k[i] >> shift) & 0xff);
+      const uint32_t pos = digit_base[d] + warp_cnt[w][d] + rank[i];
+      keys_out[pos] = k[i];
+      vals_out[pos] = v[i];
+    }
+  }
+}
+
+// ---- 3./6. single-pass scans with decoupled look-back ---------------------------------------
+struct HeadPos {  // value(p) = p if the sorted fingerprint changes at p, else 0
+  const uint64_t* keys;
+  __device__ int32_t operator()(int64_t p) const {
+    return (p == 0 || keys[p] != keys[p - 1]) ? (int32_t)p : 0;
+  }
+};
+struct IsRep {  // value(i) = 1 if row i represents its group
+  const int32_t* rep;
+  __device__ int32_t operator()(int64_t i) const { return rep[i] == (int32_t)i ? 1 : 0; }
+};
+struct OpMax {
+  __device__ int32_t operator()(int32_t a, int32_t b) const { return a > b ? a : b; }
+  static constexpr int32_t identity = 0;
+};
+struct OpSum {
+  __device__ int32_t operator()(int32_t a, int32_t b) const { return a + b; }
+  static constexpr int32_t identity = 0;
+};
+
+template <class Src, class Op, bool kExclusive>
+__global__ void __launch_bounds__(kScanThreads) scan_kernel(Src src, int64_t n, int32_t* out,
+                                                            unsigned long long* status,
+                                                            uint32_t* tile_ctr,
+                                                            int32_t* total_out, unsigned* err) {
+  __shared__ uint32_t s_tile;
+  __shared__ int32_t s_warp[kScanThreads / 32];
+  __shared__ int32_t s_prefix;
+  const Op op;
+  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+  if (tid == 0) s_tile = atomicAdd(tile_ctr, 1u);
+  __syncthreads();
+  const uint32_t tile = s_tile;
+  const int64_t base = (int64_t)tile * kScanTile + (int64_t)tid * kScanItems;
+  int32_t x[kScanItems];
+  int32_t run = Op::identity;
+#pragma unroll
+  for (int i = 0; i < kScanItems; ++i) {
+    const int64_t e = base + i;
+    x[i] = e < n ? src(e) : Op::identity;
+    run = op(run, x[i]);
+  }
+  // Warp-level inclusive scan of thread totals.
+  int32_t incl = run;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl = op(y, incl);
+  }
+  if (lane == 31) s_warp[w] = incl;
+  __syncthreads();
+  int32_t warp_prefix = Op::identity, tile_total = Op::identity;
+  for (int i = 0; i < kScanThreads / 32; ++i) {
+    if (i < w) warp_prefix = op(warp_prefix, s_warp[i]);
+    tile_total = op(tile_total, s_warp[i]);
+  }
+  int32_t thread_prefix = __shfl_up_sync(0xffffffffu, incl, 1);
+  if (lane == 0) thread_prefix = Op::identity;
+  thread_prefix = op(warp_prefix, thread_prefix);
+  if (tid == 0) {
+    volatile unsigned long long* st = status;
+    int32_t prefix = Op::identity;
+    if (tile == 0) {
+      st[0] = (2ull << 32) | (uint32_t)tile_total;
+    } else {
+      st[tile] = (1ull << 32) | (uint32_t)tile_total;
+      for (int64_t j = (int64_t)tile - 1; j >= 0; --j) {
+        const unsigned long long s = wait_flag64(st + j, err);
+        prefix = op((int32_t)(uint32_t)s, prefix);
+        if ((s >> 32) == 2ull) break;
+      }
+      st[tile] = (2ull << 32) | (uint32_t)op(prefix, tile_total);
+    }
+    s_prefix = prefix;
+    const int64_t tiles = (n + kScanTile - 1) / kScanTile;
+    if (total_out && (int64_t)tile == tiles - 1) *total_out = op(prefix, tile_total);
+  }
+  __syncthreads();
+  int32_t acc = op(s_prefix, thread_prefix);
+#pragma unroll
+  for (int i = 0; i < kScanItems; ++i) {
+    const int64_t e = base + i;
+    if (kExclusive) {
+      if (e < n) out[e] = acc;
+      acc = op(acc, x[i]);
+    } else {
+      acc = op(acc, x[i]);
+      if (e < n) out[e] = acc;
+    }
+  }
+}
+
+// ---- 4./5. full-row comparison -------------------------------------------------------------------
+__device__ __forceinline__ int32_t clamp_len(const int32_t* lens, int64_t r, int32_t stride,
+                                             unsigned* err) {
+  int32_t L = lens ? __ldg(lens + r) : stride;
+  if (L < 0 || L > stride) {
+    set_error(err, kErrInvalidArg);
+    L = L < 0 ? 0 : stride;
+  }
+  return L;
+}
+
+// Whole warp: are rows a and b equal (same length, same tokens below it)?
+template <bool VEC>
+__device__ bool rows_equal_warp(const int32_t* __restrict__ tokens, int32_t stride,
+                                const int32_t* __restrict__ lens, int64_t a, int64_t b,
+                                unsigned* err) {
+  const int lane = threadIdx.x & 31;
+  const int32_t la = clamp_len(lens, a, stride, err);
+  const int32_t lb = clamp_len(lens, b, stride, err);
+  if (la != lb) return false;
+  const int32_t* ra = tokens + a * (int64_t)stride;
+  const int32_t* rb = tokens + b * (int64_t)stride;
+  bool diff = false;
+  int32_t done = 0;
+  if (VEC) {
+    const int32_t pieces = la >> 2;
+    for (int32_t j = lane; j < pieces; j += 32) {
+      const int4 x = __ldg(reinterpret_cast<const int4*>(ra) + j);
+      const int4 y = __ldg(reinterpret_cast<const int4*>(rb) + j);
+      diff |= (x.x != y.x) | (x.y != y.y) | (x.z != y.z) | (x.w != y.w);
+    }
+    done = pieces << 2;
+  }
+  for (int32_t t = done + lane; t < la; t += 32) diff |= (__ldg(ra + t) != __ldg(rb + t));
+  return !__any_sync(0xffffffffu, diff);
+}
+
+template <bool VEC>
+__global__ void __launch_bounds__(256) verify_kernel(
+    const uint32_t* __restrict__ vals, const int32_t* __restrict__ seg_head, int64_t n,
+    const int32_t* __restrict__ tokens, int32_t stride, const int32_t* __restrict__ lens,
+    int32_t* __restrict__ rep, int32_t* coll_flag, int32_t* coll_list, uint32_t* coll_count,
+    unsigned* err) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t p = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; p < n; p += warps) {
+    const int32_t h = seg_head[p];
+    const int64_t a = vals[p];
+    if (h == (int32_t)p) {
+      if (lane == 0) rep[a] = (int32_t)a;
+      continue;
+    }
+    const int64_t b = vals[h];
+    const bool eq = rows_equal_warp<VEC>(tokens, stride, lens, a, b, err);
+    if (lane == 0) {
+      rep[a] = eq ? (int32_t)b : (int32_t)a;
+      if (!eq && atomicCAS(coll_flag + h, 0, 1) == 0) coll_list[atomicAdd(coll_count, 1u)] = h;
+    }
+  }
+}
+
+// Regroup the rows of each collided segment exactly.  Within a segment,
+// positions are in ascending row order (stable sort), so the first
+// unassigned position is the smallest unassigned row index.
+template <bool VEC>
+__global__ void __launch_bounds__(256) resolve_kernel(
+    const uint32_t* __restrict__ vals, const int32_t* __restrict__ seg_head, int64_t n,
+    const int32_t* __restrict__ tokens, int32_t stride, const int32_t* __restrict__ lens,
+    int32_t* rep, const int32_t* __restrict__ coll_list, const uint32_t* coll_count,
+    unsigned* err) {
+  __shared__ int64_t s_end;
+  __shared__ int32_t s_first;
+  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5, nw = blockDim.x >> 5;
+  const uint32_t count = *coll_count;
+  for (uint32_t c = blockIdx.x; c < count; c += gridDim.x) {
+    const int32_t h = coll_list[c];
+    if (tid == 0) s_end = n;
+    __syncthreads();
+    for (int64_t p = (int64_t)h + 1 + tid; p < n; p += blockDim.x) {
+      if (p >= s_end) break;
+      if (seg_head[p] != h) {
+        atomicMin(reinterpret_cast<unsigned long long*>(&s_end), (unsigned long long)p);
+        break;
+      }
+    }
+    __syncthreads();
+    const int64_t end = s_end;
+    for (int64_t p = (int64_t)h + tid; p < end; p += blockDim.x) rep[vals[p]] = -1;
+    __syncthreads();
+    for (;;) {
+      if (tid == 0) s_first = 0x7fffffff;
+      __syncthreads();
+      for (int64_t p = (int64_t)h + tid; p < end; p += blockDim.x)
+        if (rep[vals[p]] == -1) {
+          atomicMin(&s_first, (int32_t)(p - h));
+          break;
+        }
+      __syncthreads();
+      const int32_t first = s_first;
+      if (first == 0x7fffffff) break;
+      const int64_t r = vals[h + first];
+      for (int64_t p = (int64_t)h + first + w; p < end; p += nw) {
+        const int64_t a = vals[p];
+        const int32_t cur = __shfl_sync(0xffffffffu, lane == 0 ? rep[a] : 0, 0);
+        if (cur != -1) continue;
+        const bool eq = (a == r) || rows_equal_warp<VEC>(tokens, stride, lens, a, r, err);
+        if (eq && lane == 0) rep[a] = (int32_t)r;
+      }
+      __syncthreads();
+    }
+  }
+}
+
+__global__ void __launch_bounds__(256) finalize_kernel(const int32_t* __restrict__ rep,
+                                                       const int32_t* __restrict__ uid, int64_t n,
+                                                       int32_t* __restrict__ unique_idx,
+                                                       int32_t* __restrict__ inverse) {
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    const int32_t r = rep[i];
+    inverse[i] = uid[r];
+    if (r == (int32_t)i) unique_idx[uid[i]] = (int32_t)i;
+  }
+}
+
+unsigned grid_for(int64_t items, int per_block, int max_blocks) {
+  int64_t b = (items + per_block - 1) / per_block;
+  if (b < 1) b = 1;
+  if (b > max_blocks) b = max_blocks;
+  return (unsigned)b;
+}
+
+}  // namespace
+
+size_t unique_inverse_workspace(int64_t n) { return n <= 0 ? 256 : layout(n).total; }
+
+hs_status launch_unique_inverse(const uint64_t* fp, const int32_t* tokens, int64_t n,
+                                int32_t stride, const int32_t* lens, int32_t* n_unique_dev,
+                                int32_t* unique_idx, int32_t* inverse, void* ws,
+                                cudaStream_t stream) {
+  unsigned* err = device_error_word();
+  if (!err) return fail(HS_ERR_CUDA, "could not resolve the device error word");
+  const Layout L = layout(n);
+  char* w = static_cast<char*>(ws);
+  uint32_t* hist = reinterpret_cast<uint32_t*>(w + L.hist);
+  uint32_t* status = reinterpret_cast<uint32_t*>(w + L.status);
+  uint32_t* ctr = reinterpret_cast<uint32_t*>(w + L.ctr);
+  int32_t* coll_flag = reinterpret_cast<int32_t*>(w + L.coll_flag);
+  uint32_t* coll_count = reinterpret_cast<uint32_t*>(w + L.coll_count);
+  auto* scan0 = reinterpret_cast<unsigned long long*>(w + L.scan_status0);
+  auto* scan1 = reinterpret_cast<unsigned long long*>(w + L.scan_status1);
+  uint64_t* keys[2] = {reinterpret_cast<uint64_t*>(w + L.keys0),
+                       reinterpret_cast<uint64_t*>(w + L.keys1)};
+  uint32_t* vals[2] = {reinterpret_cast<uint32_t*>(w + L.vals0),
+                       reinterpret_cast<uint32_t*>(w + L.vals1)};
+  int32_t* seg_head = reinterpret_cast<int32_t*>(w + L.seg_head);
+  int32_t* rep = reinterpret_cast<int32_t*>(w + L.rep);
+  int32_t* uid = reinterpret_cast<int32_t*>(w + L.uid);
+  int32_t* coll_list = reinterpret_cast<int32_t*>(w + L.coll_list);
+
+  cudaError_t e = cudaMemsetAsync(w, 0, L.zero_end, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "workspace clear");
+  const int sms = num_sms();
+  const int64_t sort_tiles = (n + kSortTile - 1) / kSortTile;
+  const int64_t scan_tiles = (n + kScanTile - 1) / kScanTile;
+
+  sort_hist_kernel<<<grid_for(n, 256 * 8, sms * 4), 256, 0, stream>>>(fp, n, hist);
+  // Eight passes; pass 0 reads the caller's fingerprints and implicit indices.
+  const uint64_t* kin = fp;
+  const uint32_t* vin = nullptr;
+  int out = 0;
+  for (int pass = 0; pass < kPasses; ++pass) {
+    onesweep_kernel<<<(unsigned)sort_tiles, kSortThreads, 0, stream>>>(
+        pass, kin, vin, keys[out], vals[out], n, hist, status, ctr, err);
+    kin = keys[out];
+    vin = vals[out];
+    out ^= 1;
+  }
+  const uint64_t* skeys = kin;
+  const uint32_t* svals = vin;
+
+  scan_kernel<HeadPos, OpMax, false><<<(unsigned)scan_tiles, kScanThreads, 0, stream>>>(
+      HeadPos{skeys}, n, seg_head, scan0, ctr + 8, nullptr, err);
+
+  const bool vec = ((reinterpret_cast<uintptr_t>(tokens) & 15u) == 0) && (stride % 4 == 0);
+  const unsigned vgrid = grid_for(n * 32, 256, sms * 16);
+  if (vec)
+    verify_kernel<true><<<vgrid, 256, 0, stream>>>(svals, seg_head, n, tokens, stride, lens, rep,
+                                                   coll_flag, coll_list, coll_count, err);
+  else
+    verify_kernel<false><<<vgrid, 256, 0, stream>>>(svals, seg_head, n, tokens, stride, lens,
+                                                    rep, coll_flag, coll_list, coll_count, err);
+  if (vec)
+    resolve_kernel<true><<<(unsigned)sms, 256, 0, stream>>>(svals, seg_head, n, tokens, stride,
+                                                            lens, rep, coll_list, coll_count, err);
+  else
+    resolve_kernel<false><<<(unsigned)sms, 256, 0, stream>>>(svals, seg_head, n, tokens, stride,
+                                                             lens, rep, coll_list, coll_count,
+                                                             err);
+  scan_kernel<IsRep, OpSum, true><<<(unsigned)scan_tiles, kScanThreads, 0, stream>>>(
+      IsRep{rep}, n, uid, scan1, ctr + 9, n_unique_dev, err);
+  finalize_kernel<<<grid_for(n, 256, sms * 8), 256, 0, stream>>>(rep, uid, n, unique_idx,
+                                                                 inverse);
+  return cuda_fail(cudaGetLastError(), "unique_inverse launch");
+}
+
+}  // namespace hs

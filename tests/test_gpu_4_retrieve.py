@@ -1,0 +1,191 @@
+"""hs_retrieve_topk vs the oracle (the retrieval node shared by merged
+queries, Section 4.1 "Workloads"; merged execution, Section 3.3).
+
+Scores must be within 2e-2 of the oracle's fp64 scores (and within 1e-3, the
+fp32-accumulation bound for unit-norm rows with d <= 1024); ids must match
+except where the oracle's k-th and (k+1)-th scores are closer than 2e-2 (the
+parity rule in hs_testutil.check_topk).  Full-size workloads are checked on
+sampled queries with the oracle, and on every query for the properties that
+hold at any size."""
+import gc
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2607_22578_gb300 as hs
+import synth
+from hs_testutil import check_topk, to_dev
+from synth import configs
+
+pytestmark = pytest.mark.gpu
+
+
+def gpu_topk(Qd, Cd, k):
+    s, i = hs.hs_retrieve_topk(Qd, Cd, k)
+    hs.hs_get_device_error()
+    return s.cpu().numpy(), i.cpu().numpy()
+
+
+def parity(Q, C, k, gs, gi, rows):
+    rows = np.asarray(rows)
+    N = C.shape[0]
+    kk = min(k + 1, N)
+    os_, oi = oracle.topk(Q[rows], C, kk)
+    exact = oracle.pair_scores(Q, C, np.repeat(rows, k), gi[rows].reshape(-1)).reshape(-1, k)
+    worst = 0.0
+    for r, q in enumerate(rows):
+        worst = max(worst, check_topk(gs[q], gi[q], os_[r], oi[r], exact[r], N, k))
+    return worst
+
+
+def all_rows_properties(Q, C, k, gs, gi):
+    """(i) and (ii) of the parity rule on every query."""
+    N = C.shape[0]
+    nq = Q.shape[0]
+    assert (gi >= 0).all() and (gi < N).all()
+    assert (np.diff(gs, axis=1) <= 0).all()
+    srt = np.sort(gi, axis=1)
+    assert (np.diff(srt, axis=1) > 0).all(), "duplicate ids within a query"
+    exact = oracle.pair_scores(Q, C, np.repeat(np.arange(nq), k), gi.reshape(-1)).reshape(nq, k)
+    err = np.abs(exact - gs).max()
+    assert err <= 1e-3, err
+    return err
+
+
+def unit_pair(nq, N, d, seed):
+    return synth.unit_rows(nq, d, seed, stream=901), synth.unit_rows(N, d, seed, stream=902)
+
+
+def test_single_tile_single_kblock():
+    Q, C = unit_pair(128, 256, 64, 1)
+    gs, gi = gpu_topk(to_dev(Q), to_dev(C), 10)
+    parity(Q, C, 10, gs, gi, range(128))
+
+
+def test_tiny_config():
+    w = configs.build_retrieval_mix(configs.TINY)
+    uidx, _ = oracle.unique_inverse(w["queries"].view(np.int32))
+    Q, C = w["queries"][uidx], w["corpus"]
+    gs, gi = gpu_topk(to_dev(Q), to_dev(C), 10)
+    parity(Q, C, 10, gs, gi, range(len(uidx)))
+
+
+@pytest.mark.parametrize("nq,N,d,k", [
+    (1, 1000, 384, 10),       # one query, ragged last corpus tile
+    (130, 777, 72, 5),        # two query blocks, d not a multiple of 64
+    (3, 300, 1024, 1),        # k = 1
+    (257, 4096, 768, 16),     # largest register-list k
+    (64, 40, 128, 40),        # k = N (full sort)
+    (33, 5000, 256, 20),      # 32-slot register list
+    (17, 3000, 256, 100),     # candidate-buffer path
+    (5, 2000, 64, 33),        # smallest buffered k
+    (40, 20000, 128, 1024),   # HS_TOPK_MAX_K
+])
+def test_shapes(nq, N, d, k):
+    Q, C = unit_pair(nq, N, d, nq * 7 + N)
+    gs, gi = gpu_topk(to_dev(Q), to_dev(C), k)
+    parity(Q, C, k, gs, gi, range(nq))
+
+
+def test_exact_ties_resolve_to_lower_index():
+    Q, C = unit_pair(4, 3000, 256, 11)
+    for q in range(4):               # three exact copies of each query
+        for j in (2900 - q, 1500 + q, 10 + q):
+            C[j] = Q[q]
+    gs, gi = gpu_topk(to_dev(Q), to_dev(C), 5)
+    for q in range(4):
+        assert gi[q, :3].tolist() == [10 + q, 1500 + q, 2900 - q]
+        assert gs[q, 0] == gs[q, 1] == gs[q, 2]
+    parity(Q, C, 5, gs, gi, range(4))
+
+
+def test_integer_valued_exact_scores():
+    # Small integers: bf16 products and fp32 sums are exact, so the GPU
+    # scores must equal the oracle's exactly and ids must match exactly.
+    rng = np.random.default_rng(2)
+    Qf = rng.integers(-2, 3, size=(70, 128)).astype(np.float32)
+    Cf = rng.integers(-2, 3, size=(900, 128)).astype(np.float32)
+    Q = (Qf.view(np.uint32) >> 16).astype(np.uint16)
+    C = (Cf.view(np.uint32) >> 16).astype(np.uint16)
+    gs, gi = gpu_topk(to_dev(Q), to_dev(C), 12)
+    os_, oi = oracle.topk(Q, C, 12)
+    assert (gs == os_).all() and (gi == oi).all()
+
+
+def test_rag_mix_full_size():
+    w = configs.build_retrieval_mix(configs.RAG_MIX)
+    uidx, _ = oracle.unique_inverse(w["queries"].view(np.int32))
+    Q, C = w["queries"][uidx], w["corpus"]
+    assert Q.shape == (1434, 768) and C.shape == (1048576, 768)
+    Cd = to_dev(C)
+    gs, gi = gpu_topk(to_dev(Q), Cd, 10)
+    del Cd
+    all_rows_properties(Q, C, 10, gs, gi)
+    sample = np.random.default_rng(0).choice(len(Q), size=24, replace=False)
+    sample = np.union1d(sample, [0, len(Q) - 1])
+    parity(Q, C, 10, gs, gi, sample)
+    gc.collect()
+    torch.cuda.empty_cache()
+
+
+def test_batch_sweep_corpus():
+    C = configs.sweep_corpus()
+    assert C.shape == (2097152, 768)
+    Cd = to_dev(C)
+    for B in configs.BATCH_SWEEP["batches"]:
+        b = configs.build_sweep_batch(B, seed=B)
+        uidx, _ = oracle.unique_inverse(b["queries"].view(np.int32))
+        Q = b["queries"][uidx]
+        gs, gi = gpu_topk(to_dev(Q), Cd, 10)
+        all_rows_properties(Q, C, 10, gs, gi)
+        sample = np.unique(np.random.default_rng(B).choice(len(Q), size=min(len(Q), 6),
+                                                           replace=False))
+        parity(Q, C, 10, gs, gi, sample)
+    del Cd
+    gc.collect()
+    torch.cuda.empty_cache()
+
+
+def test_large_corpus_planted_clusters():
+    w = configs.build_large_corpus()
+    C, Q = w["corpus"], w["queries"]
+    assert C.shape == (8388608, 1024) and Q.shape == (4096, 1024)
+    Cd = to_dev(C)
+    gs, gi = gpu_topk(to_dev(Q), Cd, 100)
+    del Cd
+    # Structure at full size: every query's top-100 lies inside its own
+    # cluster's 128 planted near-duplicates.
+    members = w["members"]
+    cl = w["query_cluster"]
+    for q in range(Q.shape[0]):
+        own = members[cl[q]]
+        assert np.isin(gi[q], own).all()
+    all_rows_properties(Q[:256], C, 100, gs[:256], gi[:256])
+    parity(Q, C, 100, gs, gi, [0, 1234, 4095])
+    gc.collect()
+    torch.cuda.empty_cache()
+
+
+def test_argument_errors():
+    C = torch.zeros((100, 64), dtype=torch.bfloat16, device="cuda")
+    Q = torch.zeros((4, 64), dtype=torch.bfloat16, device="cuda")
+    for k in (0, 101, 2000):
+        with pytest.raises(hs.HsError):
+            hs.hs_retrieve_topk(Q, C, k)
+    ws = torch.empty(256, dtype=torch.uint8, device="cuda")
+    with pytest.raises(hs.HsError) as e:
+        hs.hs_retrieve_topk(Q, C, 5, workspace=ws)
+    assert e.value.status == hs.HS_ERR_WORKSPACE
+    s, i = hs.hs_retrieve_topk(Q[:0], C, 5)
+    assert s.shape == (0, 5)
+
+
+def test_deterministic():
+    Q, C = unit_pair(300, 20000, 256, 5)
+    Qd, Cd = to_dev(Q), to_dev(C)
+    a = hs.hs_retrieve_topk(Qd, Cd, 10)
+    b = hs.hs_retrieve_topk(Qd, Cd, 10)
+    hs.hs_get_device_error()
+    assert torch.equal(a[0], b[0]) and torch.equal(a[1], b[1])

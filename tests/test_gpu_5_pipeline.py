@@ -1,0 +1,43 @@
+"""The whole stage through the public API: merged queries get exactly their
+representative's results (the kept node's output flows to every merged node,
+Section 3.3 (I)), and those results match the oracle."""
+import numpy as np
+import pytest
+
+import oracle
+import paper_2607_22578_gb300 as hs
+from hs_testutil import check_topk, to_dev
+from synth import configs
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.mark.parametrize("cfg", [configs.TINY, configs.RAG_MIX])
+def test_stage_matches_oracle(cfg):
+    w = configs.build_retrieval_mix(cfg)
+    stage = hs.EmbedRetrieveStage(to_dev(w["corpus"]), w["k"], max_queries=len(w["queries"]),
+                                  max_chunk_rows=w["tokens"].shape[0])
+    nu, uidx, inv, fp = stage.dedup_chunks(to_dev(w["tokens"]))
+    hs.hs_get_device_error()
+    ou, oi = oracle.unique_inverse(w["tokens"])
+    n = int(nu.item())
+    assert n == len(ou)
+    assert (uidx[:n].cpu().numpy() == ou).all() and (inv.cpu().numpy() == oi).all()
+    assert (fp.cpu().numpy().view(np.uint64) == oracle.fingerprint(w["tokens"])).all()
+
+    Q = w["queries"]
+    scores, ids, n_unique = stage.retrieve(to_dev(Q))
+    hs.hs_get_device_error()
+    quidx, qinv = oracle.unique_inverse(Q.view(np.int32))
+    assert n_unique == len(quidx)
+    s, i = scores.cpu().numpy(), ids.cpu().numpy()
+    # Every query equals its representative's row of the result.
+    rep = quidx[qinv]
+    assert (s == s[rep]).all() and (i == i[rep]).all()
+    k = w["k"]
+    sample = quidx[: min(len(quidx), 16)]
+    os_, oi_ = oracle.topk(Q[sample], w["corpus"], k + 1)
+    exact = oracle.pair_scores(Q, w["corpus"], np.repeat(sample, k),
+                               i[sample].reshape(-1)).reshape(-1, k)
+    for r, q in enumerate(sample):
+        check_topk(s[q], i[q], os_[r], oi_[r], exact[r], w["corpus"].shape[0], k)
