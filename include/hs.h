@@ -180,6 +180,13 @@ hs_status hs_scatter_results(const void* src, int64_t n_src, int64_t row_bytes,
  */
 hs_status hs_get_device_error(hs_stream_t stream);
 
+/*
+ * hs_launch_count — diagnostics: number of kernels this library has launched
+ * in this process (all devices, all threads) since it was loaded.  Takes no
+ * part in the method; callers use it to count device work per call.
+ */
+uint64_t hs_launch_count(void);
+
 #ifdef __cplusplus
 }
 #endif

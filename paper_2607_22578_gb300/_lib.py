@@ -72,6 +72,7 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
             lib.hs_scatter_results.restype = st
             lib.hs_get_device_error.argtypes = [P]
             lib.hs_get_device_error.restype = st
+            lib.hs_launch_count.restype = ctypes.c_uint64
             _lib = lib
     return _lib
 
@@ -197,6 +198,11 @@ def hs_scatter_results(src: torch.Tensor, mapping: torch.Tensor, dst: torch.Tens
     _check(load().hs_scatter_results(_ptr(src), src.shape[0], row_bytes, _ptr(mapping), n,
                                      _ptr(dst), _stream(stream)))
     return dst
+
+
+def hs_launch_count() -> int:
+    """Kernels launched by the library in this process (diagnostics)."""
+    return int(load().hs_launch_count())
 
 
 def hs_get_device_error(stream=None) -> None:

@@ -3,6 +3,7 @@
 #include <stdarg.h>
 #include <stdio.h>
 
+#include <atomic>
 #include <mutex>
 
 #include "hs_internal.cuh"
@@ -28,6 +29,7 @@ __device__ unsigned g_device_error;  // one word per device (module-scope variab
 unsigned* g_err_addr[kMaxDevices] = {};
 int g_sms[kMaxDevices] = {};
 std::mutex g_mu;
+std::atomic<uint64_t> g_launches{0};
 
 int current_device() {
   int dev = -1;
@@ -65,6 +67,8 @@ unsigned* device_error_word() {
   return g_err_addr[dev];
 }
 
+void count_launches(unsigned n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
+
 int num_sms() {
   const int dev = current_device();
   if (dev < 0) return 1;
@@ -87,6 +91,8 @@ extern "C" {
 const char* hs_last_error(void) { return g_msg; }
 
 const char* hs_version(void) { return "hs 0.1 (sm_103a)"; }
+
+uint64_t hs_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
 
 hs_status hs_fingerprint(const int32_t* tokens, int64_t n_rows, int32_t row_stride,
                          const int32_t* lens, uint64_t seed_state, uint64_t* fp_out,

@@ -204,6 +204,7 @@ hs_status launch_fingerprint(const int32_t* tokens, int64_t n, int32_t stride,
   else
     fingerprint_kernel<false><<<(unsigned)blocks, 256, 0, stream>>>(tokens, n, stride, lens,
                                                                      seed, fp_out, rpw, err);
+  count_launches(1);
   return cuda_fail(cudaGetLastError(), "fingerprint launch");
 }
 

@@ -523,6 +523,7 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Q, const uint16_
   int64_t mgrid = Q < (int64_t)num_sms() * 8 ? Q : (int64_t)num_sms() * 8;
   merge_kernel<<<(unsigned)mgrid, 256, msmem, stream>>>(prm.part_s, prm.part_i, Q, pl.nsplit, k,
                                                         pl.p2, scores_out, ids_out);
+  count_launches(2);  // retrieve_kernel + merge_kernel
   return cuda_fail(cudaGetLastError(), "merge launch");
 }
 

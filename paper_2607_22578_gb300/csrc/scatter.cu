@@ -71,6 +71,7 @@ hs_status launch_typed(const void* src, int64_t n_src, int64_t row_bytes, const 
   if (blocks < 1) blocks = 1;
   scatter_kernel<T, U><<<(unsigned)blocks, 256, 0, stream>>>(
       static_cast<const T*>(src), n_src, map, n_rows, (uint32_t)cpr, static_cast<T*>(dst), err);
+  count_launches(1);
   return cuda_fail(cudaGetLastError(), "scatter launch");
 }
 

@@ -515,6 +515,7 @@ hs_status launch_unique_inverse(const uint64_t* fp, const int32_t* tokens, int64
       IsRep{rep}, n, uid, scan1, ctr + 9, n_unique_dev, err);
   finalize_kernel<<<grid_for(n, 256, sms * 8), 256, 0, stream>>>(rep, uid, n, unique_idx,
                                                                  inverse);
+  count_launches(14);  // hist, 8 radix passes, 2 scans, verify, resolve, finalize
   return cuda_fail(cudaGetLastError(), "unique_inverse launch");
 }
 

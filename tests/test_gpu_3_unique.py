@@ -114,11 +114,14 @@ def test_deterministic_and_workspace_reuse():
     f = hs.hs_fingerprint(t, L)
     ws = torch.empty(hs.hs_unique_inverse_workspace(t.shape[0]), dtype=torch.uint8, device="cuda")
     ws.fill_(0xAB)                                    # stale contents must not matter
-    a = [x.clone() for x in hs.hs_unique_inverse(f, t, L, workspace=ws)]
-    b = [x.clone() for x in hs.hs_unique_inverse(f, t, L, workspace=ws)]
+    runs = []
+    for _ in range(2):
+        nu, uidx, inv = hs.hs_unique_inverse(f, t, L, workspace=ws)
+        n = int(nu.item())
+        runs.append((n, uidx[:n].clone(), inv.clone()))   # entries past n_unique are unspecified
     hs.hs_get_device_error()
-    for x, y in zip(a, b):
-        assert torch.equal(x, y)
+    assert runs[0][0] == runs[1][0]
+    assert torch.equal(runs[0][1], runs[1][1]) and torch.equal(runs[0][2], runs[1][2])
 
 
 def test_workspace_too_small_is_rejected():
