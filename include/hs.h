@@ -142,7 +142,9 @@ hs_status hs_unique_inverse(const uint64_t* fp, const int32_t* tokens, int64_t n
  * k           1 <= k <= min(n_corpus, HS_TOPK_MAX_K).
  * scores_out  device float [n_queries, k]; ids_out device int32 [n_queries, k].
  * workspace   device, >= hs_retrieve_topk_workspace(...) bytes, 256-byte
- *             aligned; contents on entry are ignored.
+ *             aligned; contents on entry are ignored.  The size returned for
+ *             (n_queries, n_corpus, dim, k) suffices for every call with at
+ *             most n_queries queries and the same n_corpus, dim and k.
  * Inputs must be finite; a NaN score is never selected.
  */
 size_t hs_retrieve_topk_workspace(int64_t n_queries, int64_t n_corpus, int32_t dim, int32_t k);

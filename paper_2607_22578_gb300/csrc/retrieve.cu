@@ -473,9 +473,21 @@ hs_status launch_kernel(const CUtensorMap& mq, const CUtensorMap& mc, const Para
 
 }  // namespace
 
+// Upper bound over every query count up to Q: the split count of a plan is at
+// most min(#SMs, corpus tiles, kMergeMax / k) and its grid at most #SMs, so
+// one workspace serves every batch of at most Q queries.
 size_t retrieve_topk_workspace(int64_t Q, int64_t N, int32_t d, int32_t k) {
   if (Q <= 0 || N <= 0 || k <= 0) return 256;
-  return plan(Q, N, d, k).total;
+  (void)d;
+  const int64_t sms = num_sms();
+  int64_t ns = sms;
+  const int64_t tiles = (N + BN - 1) / BN;
+  if (ns > tiles) ns = tiles;
+  if (ns > kMergeMax / k) ns = kMergeMax / k;
+  if (ns < 1) ns = 1;
+  const size_t part = (((size_t)Q * ns * k * 4) + 255) & ~(size_t)255;
+  const size_t list = k <= 32 ? 0 : ((((size_t)sms * kEpi * 2 * k * 4) + 255) & ~(size_t)255);
+  return 2 * part + 2 * list + 256;
 }
 
 hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Q, const uint16_t* corpus,

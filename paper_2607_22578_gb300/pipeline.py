@@ -51,9 +51,11 @@ class EmbedRetrieveStage:
                                                out=self.c_out)
         return nu, uidx, inv, fp
 
-    def retrieve(self, queries: torch.Tensor):
+    def retrieve(self, queries: torch.Tensor, events: tuple | None = None):
         """Merged retrieval of a query batch.  Returns (scores [Q, k],
-        ids [Q, k], n_unique) for every original query."""
+        ids [Q, k], n_unique) for every original query.  If ``events`` is a
+        pair of CUDA events they are recorded on the current stream around
+        the hs_retrieve_topk launch (kernel timing for the roofline)."""
         Q, d = queries.shape
         if Q > self.max_queries:
             raise ValueError("batch larger than max_queries")
@@ -62,7 +64,11 @@ class EmbedRetrieveStage:
         nu, uidx, inv = _lib.hs_unique_inverse(fp, qi32, workspace=self.ws_q, out=self.q_out)
         n_unique = int(nu.item())                     # the one host synchronisation
         uq = _lib.hs_scatter_results(queries, uidx[:n_unique])
+        if events is not None:
+            events[0].record()
         s_u, i_u = _lib.hs_retrieve_topk(uq, self.corpus, self.k, workspace=self.ws_r)
+        if events is not None:
+            events[1].record()
         scores = _lib.hs_scatter_results(s_u, inv)
         ids = _lib.hs_scatter_results(i_u, inv)
         return scores, ids, n_unique
