@@ -2,8 +2,9 @@
 // part of the node semantic signature Sig(v) (Section 3.3, Eq. 2).
 //
 // FNV-1a is a serial chain over the octets of one row, so parallelism comes
-// from rows: each lane of a warp owns one row at a time and streams it with
-// 16-byte loads (4 tokens), 64 bytes in flight per lane.  Rows have
+// from rows: each lane of a warp owns one row at a time and streams it in
+// 128-byte blocks of 16-byte loads, the next block in flight while the current
+// one is hashed.  Rows have
 // different lengths; a lane that finishes its row claims the next unclaimed
 // row of its warp's range (warp-synchronous ballot, no atomics), so the
 // lanes of a warp stay busy until the range is drained.
@@ -87,8 +88,18 @@ __device__ __forceinline__ int4 ld_stream16(const int32_t* p) {
   return v;
 }
 
+__device__ __forceinline__ void hash_partial(uint32_t& lo, uint32_t& hi, const int4 v, int w) {
+  hash_word(lo, hi, (uint32_t)v.x);
+  if (w > 1) hash_word(lo, hi, (uint32_t)v.y);
+  if (w > 2) hash_word(lo, hi, (uint32_t)v.z);
+}
+
+constexpr int kBlockPieces = 8;  // 8 x 16 B = 32 tokens per block
+
 // VEC: tokens 16-byte aligned and row_stride % 4 == 0, so every row starts
-// on a 16-byte boundary.
+// on a 16-byte boundary and its ceil(len/4) 16-byte pieces lie inside the
+// row.  A lane hashes one 128-byte block of its row while the next block is
+// already in flight.
 template <bool VEC>
 __global__ void __launch_bounds__(256) fingerprint_kernel(
     const int32_t* __restrict__ tokens, int64_t n, int32_t stride,
@@ -102,15 +113,24 @@ __global__ void __launch_bounds__(256) fingerprint_kernel(
 
   bool busy = false;
   int64_t row = 0;
-  int32_t len = 0, pos = 0;
+  int32_t len = 0, pos = 0, pieces = 0, full = 0, blk = 0;
   uint32_t lo = seed_lo, hi = seed_hi;
   const int32_t* src = tokens;
+  int4 buf[kBlockPieces];
+
+  auto load_block = [&](int b, int4 (&dst)[kBlockPieces]) {
+    const int4* base = reinterpret_cast<const int4*>(src) + kBlockPieces * b;
+#pragma unroll
+    for (int i = 0; i < kBlockPieces; ++i)
+      if (kBlockPieces * b + i < pieces) dst[i] = ld_stream16(reinterpret_cast<const int32_t*>(base + i));
+  };
 
   // Start row r on this lane.  Rows of length 0 are finished at once; rows
   // with an invalid length are reported and written as 0.
   auto begin_row = [&](int64_t r) {
     row = r;
     pos = 0;
+    blk = 0;
     lo = seed_lo;
     hi = seed_hi;
     src = tokens + r * (int64_t)stride;
@@ -127,6 +147,9 @@ __global__ void __launch_bounds__(256) fingerprint_kernel(
       busy = false;
       return;
     }
+    pieces = (L + 3) >> 2;
+    full = L >> 2;
+    if (VEC) load_block(0, buf);
     busy = true;
   };
 
@@ -143,28 +166,37 @@ __global__ void __launch_bounds__(256) fingerprint_kernel(
     }
     if (!__any_sync(0xffffffffu, busy)) break;
     if (busy) {
-      const int32_t rem = len - pos;
-      if (VEC && rem >= 16) {
-        const int32_t* p = src + pos;
-        const int4 v0 = ld_stream16(p);
-        const int4 v1 = ld_stream16(p + 4);
-        const int4 v2 = ld_stream16(p + 8);
-        const int4 v3 = ld_stream16(p + 12);
-        hash4(lo, hi, v0);
-        hash4(lo, hi, v1);
-        hash4(lo, hi, v2);
-        hash4(lo, hi, v3);
-        pos += 16;
+      if (VEC) {
+        int4 nxt[kBlockPieces];
+        const bool more = kBlockPieces * (blk + 1) < pieces;
+        if (more) load_block(blk + 1, nxt);
+#pragma unroll
+        for (int i = 0; i < kBlockPieces; ++i) {
+          const int pi = kBlockPieces * blk + i;
+          if (pi < full)
+            hash4(lo, hi, buf[i]);
+          else if (pi < pieces)
+            hash_partial(lo, hi, buf[i], len & 3);
+        }
+        if (more) {
+#pragma unroll
+          for (int i = 0; i < kBlockPieces; ++i) buf[i] = nxt[i];
+          ++blk;
+        } else {
+          fp_out[row] = ((uint64_t)hi << 32) | lo;
+          busy = false;
+        }
       } else {
+        const int32_t rem = len - pos;
         const int32_t m = rem < 16 ? rem : 16;
 #pragma unroll
         for (int j = 0; j < 16; ++j)
           if (j < m) hash_word(lo, hi, (uint32_t)__ldg(src + pos + j));
         pos += m;
-      }
-      if (pos >= len) {
-        fp_out[row] = ((uint64_t)hi << 32) | lo;
-        busy = false;
+        if (pos >= len) {
+          fp_out[row] = ((uint64_t)hi << 32) | lo;
+          busy = false;
+        }
       }
     }
   }
@@ -192,8 +224,9 @@ hs_status launch_fingerprint(const int32_t* tokens, int64_t n, int32_t stride,
   const void* kfn = vec ? (const void*)fingerprint_kernel<true>
                         : (const void*)fingerprint_kernel<false>;
   const int64_t warps_target = resident_warps(kfn);
+  // At least one row per lane; more rows per warp once the grid is full.
   int64_t rpw = (n + warps_target - 1) / warps_target;
-  if (rpw < 1) rpw = 1;
+  if (rpw < 32) rpw = 32;
   const int64_t warps = (n + rpw - 1) / rpw;
   const int64_t blocks = (warps + 7) / 8;
   unsigned* err = device_error_word();

@@ -11,18 +11,23 @@
 //   warp 1      MMA issuer: 4 x tcgen05.mma (M=128, N=256, K=16) per stage
 //               into a double-buffered fp32 accumulator in tensor memory
 //               (2 x 256 columns), tcgen05.commit releases smem stages;
-//   warps 2-5   epilogue: tcgen05.ld of the 128 x 256 score tile, one thread
-//               per query (TMEM lane), threshold filter + per-query top-k.
+//   warps 2-9   epilogue: two warps per TMEM lane quarter, each reading half
+//               of the 128 x 256 score tile with tcgen05.ld; thread = (query,
+//               column half); threshold filter + per-query top-k.
 // The Q x N score matrix never leaves the SM.  Work is split into units
 // (query block, corpus split); units that share a corpus split run at the
 // same time on different SMs, so each corpus tile is read from HBM about once
 // and served to the other query blocks from L2.
 //
-// Top-k state per query: for k <= 32 a sorted list in registers (KREG = 16
-// or 32 slots); for larger k a 32-entry candidate buffer in shared memory
-// that is sorted and merged into a sorted list in global scratch whenever a
-// query's buffer fills.  Each unit writes its k best per query; K7 merges the
-// splits of each query with a bitonic sort of packed (score, index) keys.
+// Top-k state per (query, half): for k <= 32 a sorted list in registers
+// (KREG = 16 or 32 slots).  A 32-column chunk whose maximum beats no lane's
+// threshold costs one max-reduction; otherwise the chunk is staged in shared
+// memory and every lane inserts its candidates in one converged loop, so the
+// warp pays for the largest candidate count of a lane, not for the sum over
+// lanes.  For k > 32 a 16-entry candidate buffer per thread in shared memory
+// is sorted and merged into a sorted list in global scratch whenever a
+// buffer fills.  Each unit writes its k best per (query, half); K7 merges the
+// lists of each query with a bitonic sort of packed (score, index) keys.
 #include <float.h>
 
 #include "hs_internal.cuh"
@@ -35,22 +40,25 @@ constexpr int BN = 256;               // corpus rows per tile: UMMA N
 constexpr int BK = 64;                // K per stage: one 128-byte swizzle row
 constexpr int UK = 16;                // K per tcgen05.mma, kind::f16
 constexpr int kStages = 4;
-constexpr int kThreads = 192;
-constexpr int kEpi = 128;
+constexpr int kEpiWarps = 8;
+constexpr int kEpi = kEpiWarps * 32;  // epilogue threads
+constexpr int kThreads = 64 + kEpi;
+constexpr int kHalfCols = BN / 2;     // columns per epilogue thread per tile
 constexpr uint32_t kABytes = BM * BK * 2;
 constexpr uint32_t kBBytes = BN * BK * 2;
 constexpr uint32_t kStageBytes = kABytes + kBBytes;
 constexpr uint32_t kTmemCols = 2 * BN;
-constexpr int kCap = 32;              // candidate buffer per query (large-k path)
-constexpr int kMergeMax = 16384;      // nsplit * k bound for K7
+constexpr int kCap = 16;              // candidate buffer per thread (large-k path)
+constexpr int kMergeMax = 16384;      // lists * k bound for K7
 constexpr size_t kBarBytes = 256;
-constexpr size_t kSmemKReg = 1024 + (size_t)kStages * kStageBytes + kBarBytes;
-constexpr size_t kSmemLarge = kSmemKReg + (size_t)kCap * kEpi * 8;
+constexpr size_t kEpiSmem = (size_t)kEpi * 32 * 4;  // 32 KB: staging or candidate buffer
+static_assert((size_t)kCap * kEpi * 8 == kEpiSmem, "candidate buffer size");
+constexpr size_t kSmem = 1024 + (size_t)kStages * kStageBytes + kBarBytes + kEpiSmem;
 
 struct Params {
   int64_t Q, N, tiles;
   int32_t k, kb_count, qblocks, nsplit;
-  float* part_s;     // [Q][nsplit][k]
+  float* part_s;     // [Q][2 * nsplit][k]: one list per (split, column half)
   int32_t* part_i;
   float* list_s;     // large-k: [grid][kEpi][2][k]
   int32_t* list_i;
@@ -63,6 +71,24 @@ __device__ __forceinline__ void unit_coords(const Params& p, int64_t u, int& qb,
   split = (int)(u / p.qblocks);
   t0 = (int64_t)split * p.tiles / p.nsplit;
   t1 = (int64_t)(split + 1) * p.tiles / p.nsplit;
+}
+
+// Insert (s, idx) into a list sorted by score descending.  idx is larger than
+// every index already present, so on equal scores it goes after them.
+template <int KREG>
+__device__ __forceinline__ void list_insert(float (&ls)[KREG], int32_t (&li)[KREG], float s,
+                                            int32_t idx) {
+#pragma unroll
+  for (int i = KREG - 1; i > 0; --i) {
+    const bool up = s > ls[i - 1];
+    const bool here = !up && s > ls[i];
+    ls[i] = up ? ls[i - 1] : (here ? s : ls[i]);
+    li[i] = up ? li[i - 1] : (here ? idx : li[i]);
+  }
+  if (s > ls[0]) {
+    ls[0] = s;
+    li[0] = idx;
+  }
 }
 
 // ---- large-k helpers (per thread, serial) ---------------------------------------------
@@ -124,8 +150,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* tempty = tfull + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  float* cand_s = reinterpret_cast<float*>(smem + kStages * kStageBytes + kBarBytes);
-  int32_t* cand_i = reinterpret_cast<int32_t*>(cand_s + kCap * kEpi);
+  uint8_t* epi_smem = smem + kStages * kStageBytes + kBarBytes;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -135,7 +160,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(tfull + a, 1);
-      mbar_init(tempty + a, 4);
+      mbar_init(tempty + a, kEpiWarps);
     }
     *abort_flag = 0;
     fence_mbar_init();
@@ -216,30 +241,36 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     // ------------------------------------------------------------ epilogue
-    const int quarter = warp & 3;  // TMEM lanes [32*quarter, 32*quarter+32)
-    const int et = quarter * 32 + lane;
+    const int ew = warp - 2;                  // 0..7
+    const int quarter = warp & 3;             // TMEM lanes [32*quarter, 32*quarter+32)
+    const int half = ew >> 2;                 // columns [half*128, half*128+128) of a tile
+    const int row = quarter * 32 + lane;      // query within the block
+    const int et = ew * 32 + lane;            // epilogue thread index, 0..255
     const uint32_t lane_addr = (uint32_t)(quarter * 32) << 16;
     const int k = p.k;
+    const int lists = 2 * p.nsplit;
     uint32_t tile_i = 0;
+    float* stage_f = reinterpret_cast<float*>(epi_smem);            // KREG: [8][kEpi][4]
+    float* cand_s = reinterpret_cast<float*>(epi_smem);             // large k: [kCap][kEpi]
+    int32_t* cand_i = reinterpret_cast<int32_t*>(epi_smem + (size_t)kCap * kEpi * 4);
     float* Ls = p.list_s + ((size_t)blockIdx.x * kEpi + et) * 2 * (size_t)k;
     int32_t* Li = p.list_i + ((size_t)blockIdx.x * kEpi + et) * 2 * (size_t)k;
     for (int64_t u = blockIdx.x; u < units; u += gridDim.x) {
       int qb, split;
       int64_t t0, t1;
       unit_coords(p, u, qb, split, t0, t1);
-      const int64_t q = (int64_t)qb * BM + et;
+      const int64_t q = (int64_t)qb * BM + row;
       const bool valid_q = q < p.Q;
       float theta = -FLT_MAX;
       float ls[KREG > 0 ? KREG : 1];
       int32_t li[KREG > 0 ? KREG : 1];
       int cnt = 0, cur = 0;
-      if (KREG > 0) {
 #pragma unroll
-        for (int i = 0; i < (KREG > 0 ? KREG : 1); ++i) {
-          ls[i] = -FLT_MAX;
-          li[i] = -1;
-        }
-      } else if (valid_q) {
+      for (int i = 0; i < (KREG > 0 ? KREG : 1); ++i) {
+        ls[i] = -FLT_MAX;
+        li[i] = -1;
+      }
+      if (KREG == 0 && valid_q) {
         for (int i = 0; i < k; ++i) {
           Ls[i] = -FLT_MAX;
           Li[i] = -1;
@@ -249,48 +280,60 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t acc = tile_i & 1u, aphase = (tile_i >> 1) & 1u;
         if (!mbar_wait(tfull + acc, aphase, abort_flag)) goto epi_done;
         tc_fence_after();
-        const int64_t col0 = t * BN;
-        const bool tail = col0 + BN > p.N;
+        const int64_t col0 = t * BN + half * kHalfCols;
+        const bool tail = col0 + kHalfCols > p.N;
 #pragma unroll 1
-        for (int c = 0; c < BN / 32; ++c) {
+        for (int c = 0; c < kHalfCols / 32; ++c) {
           uint32_t r[32];
-          tmem_ld_32x32b_x32(tmem_base + lane_addr + acc * BN + c * 32, r);
+          tmem_ld_32x32b_x32(tmem_base + lane_addr + acc * BN + half * kHalfCols + c * 32, r);
           tmem_ld_wait();
           const int32_t cbase = (int32_t)(col0 + c * 32);
+          if (tail) {                           // zero-filled rows past N never qualify
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+              if ((int64_t)cbase + j >= p.N) r[j] = __float_as_uint(-FLT_MAX);
+          }
+          if (!valid_q) {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) r[j] = __float_as_uint(-FLT_MAX);
+          }
           if (KREG > 0) {
-            if (valid_q) {
+            float mx = __uint_as_float(r[0]);
 #pragma unroll
-              for (int j = 0; j < 32; ++j) {
-                const float s = __uint_as_float(r[j]);
-                if (s > theta && (!tail || (int64_t)(cbase + j) < p.N)) {
-                  const int32_t idx = cbase + j;
+            for (int j = 1; j < 32; ++j) mx = fmaxf(mx, __uint_as_float(r[j]));
+            const bool any = mx > theta;
+            if (__any_sync(0xffffffffu, any)) {
+              uint32_t m = 0;
+              if (any) {
 #pragma unroll
-                  for (int i = (KREG > 0 ? KREG : 1) - 1; i > 0; --i) {
-                    const bool up = s > ls[i - 1];
-                    const bool here = !up && s > ls[i];
-                    ls[i] = up ? ls[i - 1] : (here ? s : ls[i]);
-                    li[i] = up ? li[i - 1] : (here ? idx : li[i]);
-                  }
-                  if (s > ls[0]) {
-                    ls[0] = s;
-                    li[0] = idx;
-                  }
+                for (int j = 0; j < 32; ++j) m |= (__uint_as_float(r[j]) > theta ? 1u : 0u) << j;
+#pragma unroll
+                for (int v = 0; v < 8; ++v)
+                  reinterpret_cast<uint4*>(stage_f)[v * kEpi + et] =
+                      make_uint4(r[4 * v], r[4 * v + 1], r[4 * v + 2], r[4 * v + 3]);
+              }
+              const int most = __reduce_max_sync(0xffffffffu, (unsigned)__popc(m));
+              for (int it = 0; it < most; ++it) {
+                const int j = m ? __ffs(m) - 1 : 0;
+                const float s = m ? stage_f[((j >> 2) * kEpi + et) * 4 + (j & 3)] : -FLT_MAX;
+                m &= m - 1;
+                if (s > theta) {
+                  list_insert<(KREG > 0 ? KREG : 1)>(ls, li, s, cbase + j);
                   theta = ls[(KREG > 0 ? KREG : 1) - 1];
                 }
               }
+              __syncwarp();
             }
           } else {
 #pragma unroll
             for (int j0 = 0; j0 < 32; j0 += 8) {
-              if (valid_q) {
 #pragma unroll
-                for (int j = j0; j < j0 + 8; ++j) {
-                  const float s = __uint_as_float(r[j]);
-                  if (s > theta && (!tail || (int64_t)(cbase + j) < p.N)) {
-                    cand_s[cnt * kEpi + et] = s;
-                    cand_i[cnt * kEpi + et] = cbase + j;
-                    ++cnt;
-                  }
+              for (int j = j0; j < j0 + 8; ++j) {
+                const float s = __uint_as_float(r[j]);
+                if (s > theta) {
+                  cand_s[cnt * kEpi + et] = s;
+                  cand_i[cnt * kEpi + et] = cbase + j;
+                  ++cnt;
                 }
               }
               if (__any_sync(0xffffffffu, cnt > kCap - 8))
@@ -303,8 +346,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) mbar_arrive(tempty + acc);
       }
       if (valid_q) {
-        float* os = p.part_s + ((size_t)q * p.nsplit + split) * k;
-        int32_t* oi = p.part_i + ((size_t)q * p.nsplit + split) * k;
+        const size_t o = ((size_t)q * lists + 2 * split + half) * k;
+        float* os = p.part_s + o;
+        int32_t* oi = p.part_i + o;
         if (KREG > 0) {
 #pragma unroll
           for (int i = 0; i < (KREG > 0 ? KREG : 1); ++i)
@@ -350,11 +394,11 @@ __device__ __forceinline__ void unpack_key(uint64_t key, float& s, int32_t& idx)
 
 __global__ void __launch_bounds__(256) merge_kernel(const float* __restrict__ part_s,
                                                     const int32_t* __restrict__ part_i, int64_t Q,
-                                                    int32_t nsplit, int32_t k, int32_t p2,
+                                                    int32_t lists, int32_t k, int32_t p2,
                                                     float* __restrict__ out_s,
                                                     int32_t* __restrict__ out_i) {
   extern __shared__ uint64_t keys[];
-  const int m = nsplit * k;
+  const int m = lists * k;
   for (int64_t q = blockIdx.x; q < Q; q += gridDim.x) {
     const float* ps = part_s + (size_t)q * m;
     const int32_t* pi = part_i + (size_t)q * m;
@@ -428,6 +472,15 @@ int64_t gcd64(int64_t a, int64_t b) {
   return a;
 }
 
+// Largest split count a plan may use: every split needs a corpus tile, and
+// the merge sorts 2 * nsplit * k candidates per query.
+int64_t max_splits(int64_t sms, int64_t tiles, int32_t k) {
+  int64_t ns = sms;
+  if (ns > tiles) ns = tiles;
+  if (ns > kMergeMax / (2 * k)) ns = kMergeMax / (2 * k);
+  return ns < 1 ? 1 : ns;
+}
+
 struct Plan {
   int32_t qblocks, nsplit, kreg, p2;
   int64_t tiles, grid;
@@ -436,21 +489,22 @@ struct Plan {
 
 Plan plan(int64_t Q, int64_t N, int32_t d, int32_t k) {
   Plan pl{};
+  (void)d;
   const int64_t sms = num_sms();
   pl.qblocks = (int32_t)((Q + BM - 1) / BM);
   pl.tiles = (N + BN - 1) / BN;
+  // Units = qblocks * nsplit is a multiple of the SM count when possible.
   int64_t ns = sms / gcd64(sms, pl.qblocks > 0 ? pl.qblocks : 1);
-  if (ns > pl.tiles) ns = pl.tiles;
-  if (ns > kMergeMax / k) ns = kMergeMax / k;
-  if (ns < 1) ns = 1;
+  const int64_t cap = max_splits(sms, pl.tiles, k);
+  if (ns > cap) ns = cap;
   pl.nsplit = (int32_t)ns;
   pl.kreg = k <= 16 ? 16 : (k <= 32 ? 32 : 0);
   int p2 = 1;
-  while (p2 < pl.nsplit * k) p2 <<= 1;
+  while (p2 < 2 * pl.nsplit * k) p2 <<= 1;
   pl.p2 = p2;
   const int64_t units = (int64_t)pl.qblocks * pl.nsplit;
   pl.grid = units < sms ? units : sms;
-  pl.part_bytes = (((size_t)Q * pl.nsplit * k * 4) + 255) & ~(size_t)255;
+  pl.part_bytes = (((size_t)Q * 2 * pl.nsplit * k * 4) + 255) & ~(size_t)255;
   pl.list_bytes = pl.kreg ? 0 : ((((size_t)pl.grid * kEpi * 2 * k * 4) + 255) & ~(size_t)255);
   pl.total = 2 * pl.part_bytes + 2 * pl.list_bytes + 256;
   return pl;
@@ -459,33 +513,28 @@ Plan plan(int64_t Q, int64_t N, int32_t d, int32_t k) {
 template <int KREG>
 hs_status launch_kernel(const CUtensorMap& mq, const CUtensorMap& mc, const Params& prm,
                         int64_t grid, cudaStream_t stream) {
-  const size_t smem = KREG > 0 ? kSmemKReg : kSmemLarge;
   static bool configured = false;
   if (!configured) {
     cudaError_t e = cudaFuncSetAttribute(retrieve_kernel<KREG>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmem);
     if (e != cudaSuccess) return cuda_fail(e, "retrieve smem attribute");
     configured = true;
   }
-  retrieve_kernel<KREG><<<(unsigned)grid, kThreads, smem, stream>>>(mq, mc, prm);
+  retrieve_kernel<KREG><<<(unsigned)grid, kThreads, kSmem, stream>>>(mq, mc, prm);
   return cuda_fail(cudaGetLastError(), "retrieve launch");
 }
 
 }  // namespace
 
-// Upper bound over every query count up to Q: the split count of a plan is at
-// most min(#SMs, corpus tiles, kMergeMax / k) and its grid at most #SMs, so
-// one workspace serves every batch of at most Q queries.
+// Upper bound over every query count up to Q: a plan's split count is at most
+// max_splits() and its grid at most the SM count, so one workspace serves
+// every batch of at most Q queries.
 size_t retrieve_topk_workspace(int64_t Q, int64_t N, int32_t d, int32_t k) {
   if (Q <= 0 || N <= 0 || k <= 0) return 256;
   (void)d;
   const int64_t sms = num_sms();
-  int64_t ns = sms;
-  const int64_t tiles = (N + BN - 1) / BN;
-  if (ns > tiles) ns = tiles;
-  if (ns > kMergeMax / k) ns = kMergeMax / k;
-  if (ns < 1) ns = 1;
-  const size_t part = (((size_t)Q * ns * k * 4) + 255) & ~(size_t)255;
+  const int64_t ns = max_splits(sms, (N + BN - 1) / BN, k);
+  const size_t part = (((size_t)Q * 2 * ns * k * 4) + 255) & ~(size_t)255;
   const size_t list = k <= 32 ? 0 : ((((size_t)sms * kEpi * 2 * k * 4) + 255) & ~(size_t)255);
   return 2 * part + 2 * list + 256;
 }
@@ -533,8 +582,8 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Q, const uint16_
     merge_configured = msmem;
   }
   int64_t mgrid = Q < (int64_t)num_sms() * 8 ? Q : (int64_t)num_sms() * 8;
-  merge_kernel<<<(unsigned)mgrid, 256, msmem, stream>>>(prm.part_s, prm.part_i, Q, pl.nsplit, k,
-                                                        pl.p2, scores_out, ids_out);
+  merge_kernel<<<(unsigned)mgrid, 256, msmem, stream>>>(prm.part_s, prm.part_i, Q, 2 * pl.nsplit,
+                                                        k, pl.p2, scores_out, ids_out);
   count_launches(2);  // retrieve_kernel + merge_kernel
   return cuda_fail(cudaGetLastError(), "merge launch");
 }
