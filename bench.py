@@ -45,7 +45,7 @@ WORKLOAD = ("rag_mix: 64 workflows x 32 queries (30% cross-workflow exact duplic
             "corpus 1,048,576 x 768 bf16 unit-norm; top-10")
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 KERNELS_PER_STEP = {  # kernels the library launches per call (hs_launch_count agrees)
-    "hs_fingerprint": 1, "hs_unique_inverse": 14, "hs_scatter_results": 1, "hs_retrieve_topk": 2}
+    "hs_fingerprint": 1, "hs_unique_inverse": 10, "hs_scatter_results": 1, "hs_retrieve_topk": 2}
 
 
 # ---------------------------------------------------------------- host logic
@@ -296,6 +296,8 @@ def gpu_arm(args, rank: int, local_rank: int, world: int) -> int:
     rows_total = (n_chunk + n_q) * K * world
     ret_ms = statistics.mean(a.elapsed_time(b) for a, b in rev)
 
+    breakdown = rag_mix_breakdown(stage, tokens, queries, min(K, 50)) if args.breakdown else None
+
     # End to end through the public API: pinned host inputs in, results out.
     h_tokens = torch.from_numpy(w["tokens"]).pin_memory()
     h_queries = torch.from_numpy(w["queries"].view(np.int16)).pin_memory()
@@ -367,6 +369,8 @@ def gpu_arm(args, rank: int, local_rank: int, world: int) -> int:
             "gpu_launches": int(launches),
             "clocks": clk,
         }
+        if breakdown is not None:
+            line["breakdown_ms"] = breakdown
         if world == 1 and not args.no_cpu_baseline:
             del corpus, tokens, queries, stage
             torch.cuda.empty_cache()
@@ -384,6 +388,232 @@ def gpu_arm(args, rank: int, local_rank: int, world: int) -> int:
     return 0
 
 
+# ---------------------------------------------------------------- per-row measurements
+# These print one JSON line per workload for the other rows of the hot-path
+# table (dedup-heavy dedup + scatter, the batch sweep, the large corpus) and a
+# per-phase breakdown of the RAG-mix step.  They are measurement aids beside
+# the contract line above, not the headline.
+def _dev_array(a, dev):
+    import numpy as np
+    import torch
+    a = np.ascontiguousarray(a)
+    if a.dtype == np.uint16:
+        return torch.from_numpy(a.view(np.int16)).to(dev).view(torch.bfloat16)
+    return torch.from_numpy(a).to(dev)
+
+
+def _ev():
+    import torch
+    return torch.cuda.Event(enable_timing=True)
+
+
+def _roof(bytes_=None, flops=None, ms=None, peaks=None):
+    out = {"ms": ms}
+    if bytes_ is not None:
+        gbs = bytes_ / (ms / 1e3) / 1e9
+        out.update(bytes=bytes_, gbs=gbs, frac_hbm=gbs / peaks["hbm_gbs"])
+    if flops is not None:
+        tf = flops / (ms / 1e3) / 1e12
+        out.update(flops=flops, tflops=tf, frac_tensor=tf / peaks["bf16_tflops"])
+    return out
+
+
+def row_dedup_heavy(args, dev, peaks) -> dict:
+    """Dedup-heavy: fingerprint + unique/inverse + scatter of a 1536-byte
+    payload per unique row back to all 400,000 rows."""
+    import numpy as np
+    import torch
+
+    import paper_2607_22578_gb300 as hs
+    import synth
+    from synth import configs
+    w = configs.build_dedup_heavy(seed=args.seed)
+    n = w["tokens"].shape[0]
+    tokens, lens = _dev_array(w["tokens"], dev), _dev_array(w["lens"], dev)
+    gu, gi = synth.partition_of(w["chunk_root"])
+    n_u = len(gu)
+    W = w["payload_bytes"]
+    payload = torch.randint(0, 255, (n_u, W), dtype=torch.uint8, device=dev)
+    fp = torch.empty(n, dtype=torch.int64, device=dev)
+    ws = torch.empty(hs.hs_unique_inverse_workspace(n), dtype=torch.uint8, device=dev)
+    outs = (torch.empty(1, dtype=torch.int32, device=dev),
+            torch.empty(n, dtype=torch.int32, device=dev),
+            torch.empty(n, dtype=torch.int32, device=dev))
+    dst = torch.empty((n, W), dtype=torch.uint8, device=dev)
+    K = max(1, args.steps)
+    evs = [[_ev() for _ in range(4)] for _ in range(K)]
+
+    def step(e=None):
+        if e: e[0].record()
+        hs.hs_fingerprint(tokens, lens, fp_out=fp)
+        if e: e[1].record()
+        hs.hs_unique_inverse(fp, tokens, lens, workspace=ws, out=outs)
+        if e: e[2].record()
+        hs.hs_scatter_results(payload, outs[2], dst=dst)
+        if e: e[3].record()
+
+    for _ in range(args.warmup):
+        step()
+    hs.hs_get_device_error()
+    torch.cuda.synchronize()
+    for i in range(K):
+        step(evs[i])
+    torch.cuda.synchronize()
+    hs.hs_get_device_error()
+    assert int(outs[0].item()) == n_u
+    t_fp = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
+    t_un = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
+    t_sc = statistics.mean(e[2].elapsed_time(e[3]) for e in evs)
+    t_all = statistics.mean(e[0].elapsed_time(e[3]) for e in evs)
+    L = w["lens"].astype(np.int64)
+    sizes = np.bincount(gi, minlength=n_u)
+    multi = sizes[gi] > 1
+    tok_bytes = 4 * int(L.sum())
+    fp_bytes = tok_bytes + 4 * n + 8 * n
+    un_bytes = 4 * int(L[multi].sum()) + 8 * n + 8 * n
+    sc_bytes = n_u * W + n * W + 4 * n
+    return {
+        "workload": "dedup_heavy: 400,000 rows x 512 int32 (lens U[64,512], Zipf(1.1) over "
+                    "100,000 distinct) -> %d unique; scatter %d B per row" % (n_u, W),
+        "metric": "dedup rows/s (fingerprint + unique/inverse + scatter)",
+        "value": n / (t_all / 1e3), "ms_per_step": t_all, "steps": K,
+        "kernels": {
+            "hs_fingerprint": _roof(fp_bytes, None, t_fp, peaks),
+            "hs_unique_inverse": _roof(un_bytes, None, t_un, peaks),
+            "hs_scatter_results": _roof(sc_bytes, None, t_sc, peaks)},
+        "bytes_note": "fingerprint: valid token bytes + lens + fp; unique: full-row verify "
+                      "re-read of every row in a group of size >= 2 + fp in + unique_idx/inverse "
+                      "out (sort scratch is L2-resident and not counted); scatter: unique rows "
+                      "once + every destination row + map",
+        "token_bytes_one_pass": tok_bytes}
+
+
+def row_batch_sweep(args, dev, peaks) -> dict:
+    """Adaptive-batch sweep: latency p50/p99 and q/s per batch size against a
+    2,097,152 x 768 corpus."""
+    import numpy as np
+    import torch
+
+    import paper_2607_22578_gb300 as hs
+    from synth import configs
+    cfg = configs.BATCH_SWEEP
+    C = configs.sweep_corpus(seed=args.seed)
+    corpus = _dev_array(C, dev)
+    N, d = C.shape
+    del C
+    stage = hs.EmbedRetrieveStage(corpus, cfg["k"], max_queries=max(cfg["batches"]))
+    out = {"workload": "batch_sweep: corpus 2,097,152 x 768 bf16, 20% in-batch duplicates, "
+                       "k=10", "metric": "per-batch latency and queries/s", "batches": {}}
+    for B in cfg["batches"]:
+        nb = 50 if B >= 4096 else 200
+        batches = [_dev_array(configs.build_sweep_batch(B, seed=1000 + i)["queries"], dev)
+                   for i in range(nb + 3)]
+        lat, ret, nus = [], [], []
+        for i, q in enumerate(batches):
+            e0, e1, r0, r1 = _ev(), _ev(), _ev(), _ev()
+            e0.record()
+            _, _, nu = stage.retrieve(q, (r0, r1))
+            e1.record()
+            torch.cuda.synchronize()
+            if i >= 3:
+                lat.append(e0.elapsed_time(e1))
+                ret.append(r0.elapsed_time(r1))
+                nus.append(nu)
+        hs.hs_get_device_error()
+        qu = float(np.mean(nus))
+        t_ret = float(np.mean(ret))
+        rb = 2.0 * N * d + 2.0 * qu * d + qu * cfg["k"] * 8
+        out["batches"][str(B)] = {
+            "merged_queries_mean": qu, "latency_ms_p50": float(np.percentile(lat, 50)),
+            "latency_ms_p99": float(np.percentile(lat, 99)),
+            "queries_per_s": B * len(lat) / (sum(lat) / 1e3),
+            "retrieval": _roof(rb, 2.0 * qu * N * d, t_ret, peaks)}
+        del batches
+    return out
+
+
+def row_large_corpus(args, dev, peaks) -> dict:
+    """Large corpus: 4096 merged queries x 8,388,608 x 1024, k = 100."""
+    import torch
+
+    import paper_2607_22578_gb300 as hs
+    from synth import configs
+    w = configs.build_large_corpus(seed=args.seed)
+    corpus, queries = _dev_array(w["corpus"], dev), _dev_array(w["queries"], dev)
+    N, d = w["corpus"].shape
+    Q, k = w["queries"].shape[0], w["k"]
+    del w
+    ws = torch.empty(hs.hs_retrieve_topk_workspace(Q, N, d, k), dtype=torch.uint8, device=dev)
+    outs = (torch.empty((Q, k), dtype=torch.float32, device=dev),
+            torch.empty((Q, k), dtype=torch.int32, device=dev))
+    for _ in range(2):
+        hs.hs_retrieve_topk(queries, corpus, k, workspace=ws, out=outs)
+    torch.cuda.synchronize()
+    K = max(1, min(args.steps, 10))
+    e0, e1 = _ev(), _ev()
+    e0.record()
+    for _ in range(K):
+        hs.hs_retrieve_topk(queries, corpus, k, workspace=ws, out=outs)
+    e1.record()
+    torch.cuda.synchronize()
+    hs.hs_get_device_error()
+    ms = e0.elapsed_time(e1) / K
+    return {"workload": "large_corpus: 4096 merged queries x 8,388,608 x 1024 bf16 "
+                        "(1024 planted clusters), k=100",
+            "metric": "merged queries/s", "value": Q / (ms / 1e3), "steps": K,
+            "retrieval": _roof(2.0 * N * d, 2.0 * Q * N * d, ms, peaks)}
+
+
+def rag_mix_breakdown(stage, tokens, queries, K: int) -> dict:
+    """Per-phase device time of the RAG-mix step (same calls as the step)."""
+    import torch
+
+    import paper_2607_22578_gb300 as hs
+    from paper_2607_22578_gb300 import _lib
+    names = ["chunk_fingerprint", "chunk_unique", "query_fingerprint", "query_unique",
+             "count_sync_and_gather", "retrieve_topk", "scatter_results"]
+    acc = {n: 0.0 for n in names}
+    for _ in range(K):
+        ev = [_ev() for _ in range(len(names) + 1)]
+        ev[0].record()
+        fp = _lib.hs_fingerprint(tokens)
+        ev[1].record()
+        _lib.hs_unique_inverse(fp, tokens, workspace=stage.ws_c, out=stage.c_out)
+        ev[2].record()
+        qi32 = queries.view(torch.int32)
+        qfp = _lib.hs_fingerprint(qi32)
+        ev[3].record()
+        nu, uidx, inv = _lib.hs_unique_inverse(qfp, qi32, workspace=stage.ws_q, out=stage.q_out)
+        ev[4].record()
+        n_unique = int(nu.item())
+        uq = _lib.hs_scatter_results(queries, uidx[:n_unique])
+        ev[5].record()
+        s_u, i_u = _lib.hs_retrieve_topk(uq, stage.corpus, stage.k, workspace=stage.ws_r)
+        ev[6].record()
+        _lib.hs_scatter_results(s_u, inv)
+        _lib.hs_scatter_results(i_u, inv)
+        ev[7].record()
+        torch.cuda.synchronize()
+        for i, n in enumerate(names):
+            acc[n] += ev[i].elapsed_time(ev[i + 1])
+    hs.hs_get_device_error()
+    return {n: v / K for n, v in acc.items()}
+
+
+def rows_arm(args) -> int:
+    import torch
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    peaks, kind = load_peaks()
+    fn = {"dedup_heavy": row_dedup_heavy, "batch_sweep": row_batch_sweep,
+          "large_corpus": row_large_corpus}[args.workload]
+    line = fn(args, dev, peaks)
+    line["peaks"] = {"hbm_gbs": peaks["hbm_gbs"], "bf16_tflops": peaks["bf16_tflops"],
+                     "source": kind}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def main() -> int:
     ap = argparse.ArgumentParser(description=__doc__.split("\n\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -394,6 +624,12 @@ def main() -> int:
     ap.add_argument("--cpu-budget", type=float, default=20.0,
                     help="seconds of host time for the oracle baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--workload", default="rag_mix",
+                    choices=["rag_mix", "dedup_heavy", "batch_sweep", "large_corpus"],
+                    help="rag_mix is the headline step; the others measure the other "
+                         "rows of the hot-path table (one GPU)")
+    ap.add_argument("--breakdown", action="store_true",
+                    help="add per-phase device times of the rag_mix step")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -413,6 +649,8 @@ def main() -> int:
     try:
         if args.impl == "reference":
             return reference_arm(args, rank, world)
+        if args.workload != "rag_mix":
+            return rows_arm(args) if rank == 0 else 0
         return gpu_arm(args, rank, local_rank, world)
     finally:
         if world > 1:

@@ -3,16 +3,20 @@
 // Reuse Mechanism" (I)) and the merge sets M(v*) of Appendix A.2.
 //
 // Pipeline (all on the caller's stream, no host synchronisation):
-//   1. histogram of all eight 8-bit digits of the fingerprints (one pass);
-//   2. eight stable LSD radix passes over (fingerprint, row index), each a
-//      single kernel with decoupled look-back across tiles (bounded spins);
-//      stability keeps equal fingerprints in ascending row order, so each
-//      run of equal fingerprints starts with its smallest row index;
-//   3. segment heads: inclusive max-scan of "fingerprint differs from the
-//      previous one" positions;
+//   1. histogram of the four 8-bit digits of each fingerprint's upper 32
+//      bits (one pass);
+//   2. four stable LSD radix passes over (upper 32 fingerprint bits, row
+//      index), each a single kernel with decoupled look-back across tiles
+//      (bounded spins); stability keeps equal keys in ascending row order, so
+//      each run of equal keys starts with its smallest row index;
+//   3. segment heads: inclusive max-scan of "key differs from the previous
+//      one" positions;
 //   4. verify: every non-head row is compared in full (length + tokens) with
 //      its segment head by one warp; equal rows take the head as their
-//      representative, a mismatch marks the segment as collided;
+//      representative, a mismatch marks the segment as collided.  A segment
+//      holds rows whose fingerprints agree in the upper 32 bits; rows that
+//      differ (in the lower bits, or in content under a true collision) are
+//      never merged, they only send the segment through step 5;
 //   5. collided segments only: exact regrouping by repeated peeling (the
 //      first unassigned row becomes a representative, all rows equal to it
 //      join it);
@@ -27,7 +31,8 @@ namespace {
 constexpr int kSortThreads = 256;
 constexpr int kSortItems = 16;
 constexpr int kSortTile = kSortThreads * kSortItems;  // 4096 keys per tile
-constexpr int kPasses = 8;
+constexpr int kPasses = 4;   // digits of bits 32..63 of the fingerprint
+constexpr int kLookBatch = 8;  // predecessor statuses read per round trip
 constexpr uint32_t kFlagA = 1u << 30;  // tile aggregate published
 constexpr uint32_t kFlagP = 2u << 30;  // inclusive prefix published
 constexpr uint32_t kValMask = (1u << 30) - 1u;
@@ -57,8 +62,8 @@ Layout layout(int64_t n) {
   L.scan_status0 = o;  o += align256(sizeof(uint64_t) * (size_t)scan_tiles);
   L.scan_status1 = o;  o += align256(sizeof(uint64_t) * (size_t)scan_tiles);
   L.zero_end = o;
-  L.keys0 = o;         o += align256(sizeof(uint64_t) * (size_t)n);
-  L.keys1 = o;         o += align256(sizeof(uint64_t) * (size_t)n);
+  L.keys0 = o;         o += align256(sizeof(uint32_t) * (size_t)n);
+  L.keys1 = o;         o += align256(sizeof(uint32_t) * (size_t)n);
   L.vals0 = o;         o += align256(sizeof(uint32_t) * (size_t)n);
   L.vals1 = o;         o += align256(sizeof(uint32_t) * (size_t)n);
   L.seg_head = o;      o += align256(sizeof(int32_t) * (size_t)n);
@@ -113,7 +118,7 @@ __global__ void __launch_bounds__(256) sort_hist_kernel(const uint64_t* __restri
   __syncthreads();
   for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n;
        e += (int64_t)gridDim.x * blockDim.x) {
-    const uint64_t k = __ldg(fp + e);
+    const uint32_t k = (uint32_t)(__ldg(fp + e) >> 32);
 #pragma unroll
     for (int p = 0; p < kPasses; ++p) atomicAdd(&h[p * 256 + ((k >> (8 * p)) & 0xff)], 1u);
   }
@@ -126,9 +131,12 @@ __global__ void __launch_bounds__(256) sort_hist_kernel(const uint64_t* __restri
 // Tile t holds keys [t*4096, (t+1)*4096); warp w of the tile owns the 512 keys
 // [w*512, (w+1)*512), read striped (item i of lane l is key w*512 + i*32 + l),
 // so processing items in order with lanes in order follows the input order.
+// Pass 0 reads the caller's 64-bit fingerprints (fp_in) and implicit row
+// indices; later passes read the previous pass's (key, value) arrays.
 __global__ void __launch_bounds__(kSortThreads) onesweep_kernel(
-    int pass, const uint64_t* __restrict__ keys_in, const uint32_t* __restrict__ vals_in,
-    uint64_t* __restrict__ keys_out, uint32_t* __restrict__ vals_out, int64_t n,
+    int pass, const uint64_t* __restrict__ fp_in, const uint32_t* __restrict__ keys_in,
+    const uint32_t* __restrict__ vals_in, uint32_t* __restrict__ keys_out,
+    uint32_t* __restrict__ vals_out, int64_t n,
     const uint32_t* __restrict__ hist, uint32_t* status, uint32_t* tile_ctr, unsigned* err) {
   __shared__ uint32_t s_tile;
   __shared__ uint32_t warp_cnt[kSortThreads / 32][256];
@@ -157,15 +165,15 @@ __global__ void __launch_bounds__(kSortThreads) onesweep_kernel(
   const int64_t base = (int64_t)tile * kSortTile + w * (kSortItems * 32);
   const int shift = 8 * pass;
 
-  uint64_t k[kSortItems];
+  uint32_t k[kSortItems];
   uint32_t v[kSortItems];
   uint32_t rank[kSortItems];
 #pragma unroll
   for (int i = 0; i < kSortItems; ++i) {
     const int64_t e = base + i * 32 + lane;
     if (e < n) {
-      k[i] = keys_in[e];
-      v[i] = vals_in ? vals_in[e] : (uint32_t)e;
+      k[i] = fp_in ? (uint32_t)(fp_in[e] >> 32) : keys_in[e];
+      v[i] = fp_in ? (uint32_t)e : vals_in[e];
     } else {
       k[i] = 0;
       v[i] = 0;
@@ -199,10 +207,21 @@ __global__ void __launch_bounds__(kSortThreads) onesweep_kernel(
     st[tid] = kFlagP | tile_count;
   } else {
     st[(size_t)tile * 256 + tid] = kFlagA | tile_count;
-    for (int64_t j = (int64_t)tile - 1; j >= 0; --j) {
-      const uint32_t s = wait_flag32(st + (size_t)j * 256 + tid, err);
-      prefix += s & kValMask;
-      if ((s & ~kValMask) == kFlagP) break;
+    // Walk back kLookBatch predecessors per round trip; stop at the first
+    // inclusive prefix.
+    bool done = false;
+    for (int64_t j0 = (int64_t)tile - 1; j0 >= 0 && !done; j0 -= kLookBatch) {
+      uint32_t sv[kLookBatch];
+#pragma unroll
+      for (int b = 0; b < kLookBatch; ++b) sv[b] = j0 - b >= 0 ? st[(size_t)(j0 - b) * 256 + tid] : (2u << 30);
+#pragma unroll
+      for (int b = 0; b < kLookBatch; ++b) {
+        if (done) break;
+        uint32_t sb = sv[b];
+        if ((sb & ~kValMask) == 0) sb = wait_flag32(st + (size_t)(j0 - b) * 256 + tid, err);
+        if (j0 - b >= 0) prefix += sb & kValMask;
+        if ((sb & ~kValMask) == kFlagP) done = true;
+      }
     }
     st[(size_t)tile * 256 + tid] = kFlagP | ((prefix + tile_count) & kValMask);
   }
@@ -221,8 +240,8 @@ __global__ void __launch_bounds__(kSortThreads) onesweep_kernel(
 }
 
 // ---- 3./6. single-pass scans with decoupled look-back ---------------------------------------
-struct HeadPos {  // value(p) = p if the sorted fingerprint changes at p, else 0
-  const uint64_t* keys;
+struct HeadPos {  // value(p) = p if the sorted key changes at p, else 0
+  const uint32_t* keys;
   __device__ int32_t operator()(int64_t p) const {
     return (p == 0 || keys[p] != keys[p - 1]) ? (int32_t)p : 0;
   }
@@ -286,10 +305,19 @@ __global__ void __launch_bounds__(kScanThreads) scan_kernel(Src src, int64_t n, 
       st[0] = (2ull << 32) | (uint32_t)tile_total;
     } else {
       st[tile] = (1ull << 32) | (uint32_t)tile_total;
-      for (int64_t j = (int64_t)tile - 1; j >= 0; --j) {
-        const unsigned long long s = wait_flag64(st + j, err);
-        prefix = op((int32_t)(uint32_t)s, prefix);
-        if ((s >> 32) == 2ull) break;
+      bool done = false;
+      for (int64_t j0 = (int64_t)tile - 1; j0 >= 0 && !done; j0 -= kLookBatch) {
+        unsigned long long sv[kLookBatch];
+#pragma unroll
+        for (int b = 0; b < kLookBatch; ++b) sv[b] = j0 - b >= 0 ? st[j0 - b] : (2ull << 32);
+#pragma unroll
+        for (int b = 0; b < kLookBatch; ++b) {
+          if (done) break;
+          unsigned long long sb = sv[b];
+          if ((sb >> 32) == 0) sb = wait_flag64(st + (j0 - b), err);
+          if (j0 - b >= 0) prefix = op((int32_t)(uint32_t)sb, prefix);
+          if ((sb >> 32) == 2ull) done = true;
+        }
       }
       st[tile] = (2ull << 32) | (uint32_t)op(prefix, tile_total);
     }
@@ -463,8 +491,8 @@ hs_status launch_unique_inverse(const uint64_t* fp, const int32_t* tokens, int64
   uint32_t* coll_count = reinterpret_cast<uint32_t*>(w + L.coll_count);
   auto* scan0 = reinterpret_cast<unsigned long long*>(w + L.scan_status0);
   auto* scan1 = reinterpret_cast<unsigned long long*>(w + L.scan_status1);
-  uint64_t* keys[2] = {reinterpret_cast<uint64_t*>(w + L.keys0),
-                       reinterpret_cast<uint64_t*>(w + L.keys1)};
+  uint32_t* keys[2] = {reinterpret_cast<uint32_t*>(w + L.keys0),
+                       reinterpret_cast<uint32_t*>(w + L.keys1)};
   uint32_t* vals[2] = {reinterpret_cast<uint32_t*>(w + L.vals0),
                        reinterpret_cast<uint32_t*>(w + L.vals1)};
   int32_t* seg_head = reinterpret_cast<int32_t*>(w + L.seg_head);
@@ -479,18 +507,18 @@ hs_status launch_unique_inverse(const uint64_t* fp, const int32_t* tokens, int64
   const int64_t scan_tiles = (n + kScanTile - 1) / kScanTile;
 
   sort_hist_kernel<<<grid_for(n, 256 * 8, sms * 4), 256, 0, stream>>>(fp, n, hist);
-  // Eight passes; pass 0 reads the caller's fingerprints and implicit indices.
-  const uint64_t* kin = fp;
+  // Four passes; pass 0 reads the caller's fingerprints and implicit indices.
+  const uint32_t* kin = nullptr;
   const uint32_t* vin = nullptr;
   int out = 0;
   for (int pass = 0; pass < kPasses; ++pass) {
     onesweep_kernel<<<(unsigned)sort_tiles, kSortThreads, 0, stream>>>(
-        pass, kin, vin, keys[out], vals[out], n, hist, status, ctr, err);
+        pass, pass == 0 ? fp : nullptr, kin, vin, keys[out], vals[out], n, hist, status, ctr, err);
     kin = keys[out];
     vin = vals[out];
     out ^= 1;
   }
-  const uint64_t* skeys = kin;
+  const uint32_t* skeys = kin;
   const uint32_t* svals = vin;
 
   scan_kernel<HeadPos, OpMax, false><<<(unsigned)scan_tiles, kScanThreads, 0, stream>>>(
@@ -515,7 +543,7 @@ hs_status launch_unique_inverse(const uint64_t* fp, const int32_t* tokens, int64
       IsRep{rep}, n, uid, scan1, ctr + 9, n_unique_dev, err);
   finalize_kernel<<<grid_for(n, 256, sms * 8), 256, 0, stream>>>(rep, uid, n, unique_idx,
                                                                  inverse);
-  count_launches(14);  // hist, 8 radix passes, 2 scans, verify, resolve, finalize
+  count_launches(10);  // hist, 4 radix passes, 2 scans, verify, resolve, finalize
   return cuda_fail(cudaGetLastError(), "unique_inverse launch");
 }
 
