@@ -2,12 +2,11 @@
 // part of the node semantic signature Sig(v) (Section 3.3, Eq. 2).
 //
 // FNV-1a is a serial chain over the octets of one row, so parallelism comes
-// from rows: each lane of a warp owns one row at a time and streams it in
-// 128-byte blocks of 16-byte loads, the next block in flight while the current
-// one is hashed.  Rows have
-// different lengths; a lane that finishes its row claims the next unclaimed
-// row of its warp's range (warp-synchronous ballot, no atomics), so the
-// lanes of a warp stay busy until the range is drained.
+// from rows: each lane of a warp owns one row at a time and streams it through
+// a private shared-memory ring filled by cp.async several blocks ahead.  Rows
+// have different lengths; a lane that has issued its whole row claims the next
+// unclaimed row of its warp's range (warp-synchronous ballot, no atomics), so
+// the lanes of a warp stay busy until the range is drained.
 //
 // Arithmetic: h = (hi:lo) as two 32-bit words; a multiply by the prime
 // 2^40 + 0x1b3 is one wide 32x32 multiply, one multiply-add and one
@@ -80,28 +79,143 @@ __device__ __forceinline__ void hash4(uint32_t& lo, uint32_t& hi, const int4 v) 
   }
 }
 
-__device__ __forceinline__ int4 ld_stream16(const int32_t* p) {
-  int4 v;
-  asm volatile("ld.global.nc.L1::no_allocate.v4.s32 {%0, %1, %2, %3}, [%4];"
-               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-               : "l"(p));
-  return v;
-}
-
 __device__ __forceinline__ void hash_partial(uint32_t& lo, uint32_t& hi, const int4 v, int w) {
   hash_word(lo, hi, (uint32_t)v.x);
   if (w > 1) hash_word(lo, hi, (uint32_t)v.y);
   if (w > 2) hash_word(lo, hi, (uint32_t)v.z);
 }
 
-constexpr int kBlockPieces = 8;  // 8 x 16 B = 32 tokens per block
+// ---- vector path: per-lane cp.async pipeline ----------------------------------------
+// A lane owns one row at a time.  Its row is cut into blocks of 16 tokens
+// (four 16-byte pieces); the lane keeps kDepth blocks in a private ring in
+// shared memory, filled by cp.async (16-byte, L2-only) kDepth-1 blocks ahead
+// of the block it hashes.  The issue side claims the next row as soon as the
+// current one is fully issued, so a row boundary costs no exposed latency.
+// In-flight data lives in shared memory, not registers, so occupancy stays
+// high.  The ring is padded by 16 bytes per lane so the eight lanes of a
+// quarter-warp read different banks.
+constexpr int kDepth = 6;
+constexpr int kBlockWords = 16;
+constexpr int kLaneBytes = kDepth * kBlockWords * 4 + 16;
+constexpr int kFpThreads = 64;
 
-// VEC: tokens 16-byte aligned and row_stride % 4 == 0, so every row starts
-// on a 16-byte boundary and its ceil(len/4) 16-byte pieces lie inside the
-// row.  A lane hashes one 128-byte block of its row while the next block is
-// already in flight.
-template <bool VEC>
-__global__ void __launch_bounds__(256) fingerprint_kernel(
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+__global__ void __launch_bounds__(kFpThreads) fingerprint_async_kernel(
+    const int32_t* __restrict__ tokens, int64_t n, int32_t stride,
+    const int32_t* __restrict__ lens, uint64_t seed, uint64_t* __restrict__ fp_out,
+    int64_t rows_per_warp, unsigned* err) {
+  extern __shared__ uint8_t ring_all[];
+  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t r_begin = warp * rows_per_warp;
+  if (r_begin >= n) return;
+  const int64_t r_end = min(n, r_begin + rows_per_warp);
+  const uint32_t ring = smem_u32(ring_all + threadIdx.x * kLaneBytes);
+  const uint8_t* ring_p = ring_all + threadIdx.x * kLaneBytes;
+  const uint32_t seed_lo = (uint32_t)seed, seed_hi = (uint32_t)(seed >> 32);
+
+  // Issue side.
+  int64_t irow = -1;
+  int32_t ipos = 0, ilen = 0;
+  const int32_t* isrc = tokens;
+  // Per-slot metadata: row (or -1), valid words, first/last block of the row.
+  int64_t m_row[kDepth];
+  int32_t m_words[kDepth];
+  bool m_first[kDepth], m_last[kDepth];
+#pragma unroll
+  for (int s = 0; s < kDepth; ++s) {
+    m_row[s] = -1;
+    m_words[s] = 0;
+    m_first[s] = m_last[s] = false;
+  }
+  // Hash side.
+  uint32_t lo = seed_lo, hi = seed_hi;
+  int64_t next = r_begin;
+
+  for (;;) {
+#pragma unroll
+    for (int si = 0; si < kDepth; ++si) {
+      // ---- claim rows for lanes whose issue side is free, in lane order
+      unsigned need = __ballot_sync(0xffffffffu, irow < 0);
+      while (need != 0u && next < r_end) {
+        const int64_t avail = r_end - next;
+        const int rank = __popc(need & lanemask_lt());
+        if (irow < 0 && rank < avail) {
+          const int64_t r = next + rank;
+          int32_t L = lens ? __ldg(lens + r) : stride;
+          if (L < 0 || L > stride) {
+            set_error(err, kErrInvalidArg);
+            fp_out[r] = 0ull;
+          } else if (L == 0) {
+            fp_out[r] = seed;
+          } else {
+            irow = r;
+            ipos = 0;
+            ilen = L;
+            isrc = tokens + r * (int64_t)stride;
+          }
+        }
+        next += min((int64_t)__popc(need), avail);
+        need = __ballot_sync(0xffffffffu, irow < 0);
+      }
+      // ---- issue one block into slot si
+      if (irow >= 0) {
+        const int32_t words = min(kBlockWords, ilen - ipos);
+        const uint32_t dst = ring + si * kBlockWords * 4;
+#pragma unroll
+        for (int pc = 0; pc < kBlockWords / 4; ++pc)
+          if (4 * pc < words) cp_async16(dst + 16 * pc, isrc + ipos + 4 * pc);
+        m_row[si] = irow;
+        m_words[si] = words;
+        m_first[si] = ipos == 0;
+        ipos += words;
+        m_last[si] = ipos >= ilen;
+        if (ipos >= ilen) irow = -1;
+      } else {
+        m_row[si] = -1;
+      }
+      cp_async_commit();
+      // ---- hash the oldest slot (issued kDepth-1 rounds ago)
+      const int sc = (si + 1) % kDepth;
+      cp_async_wait<kDepth - 1>();
+      if (m_row[sc] >= 0) {
+        if (m_first[sc]) {
+          lo = seed_lo;
+          hi = seed_hi;
+        }
+        const int4* blk = reinterpret_cast<const int4*>(ring_p + sc * kBlockWords * 4);
+        const int32_t w = m_words[sc];
+#pragma unroll
+        for (int pc = 0; pc < kBlockWords / 4; ++pc) {
+          if (4 * pc + 4 <= w) {
+            hash4(lo, hi, blk[pc]);
+          } else if (4 * pc < w) {
+            hash_partial(lo, hi, blk[pc], w - 4 * pc);
+          }
+        }
+        if (m_last[sc]) fp_out[m_row[sc]] = ((uint64_t)hi << 32) | lo;
+        m_row[sc] = -1;
+      }
+    }
+    bool pending = irow >= 0;
+#pragma unroll
+    for (int s = 0; s < kDepth; ++s) pending |= m_row[s] >= 0;
+    if (!__any_sync(0xffffffffu, pending) && next >= r_end) break;
+  }
+  cp_async_wait<0>();
+}
+
+// ---- word path (tokens not 16-byte aligned, or row_stride % 4 != 0) -------------------
+__global__ void __launch_bounds__(256) fingerprint_words_kernel(
     const int32_t* __restrict__ tokens, int64_t n, int32_t stride,
     const int32_t* __restrict__ lens, uint64_t seed, uint64_t* __restrict__ fp_out,
     int64_t rows_per_warp, unsigned* err) {
@@ -110,109 +224,52 @@ __global__ void __launch_bounds__(256) fingerprint_kernel(
   if (r_begin >= n) return;
   const int64_t r_end = min(n, r_begin + rows_per_warp);
   const uint32_t seed_lo = (uint32_t)seed, seed_hi = (uint32_t)(seed >> 32);
-
   bool busy = false;
   int64_t row = 0;
-  int32_t len = 0, pos = 0, pieces = 0, full = 0, blk = 0;
+  int32_t len = 0, pos = 0;
   uint32_t lo = seed_lo, hi = seed_hi;
   const int32_t* src = tokens;
-  int4 buf[kBlockPieces];
-
-  auto load_block = [&](int b, int4 (&dst)[kBlockPieces]) {
-    const int4* base = reinterpret_cast<const int4*>(src) + kBlockPieces * b;
-#pragma unroll
-    for (int i = 0; i < kBlockPieces; ++i)
-      if (kBlockPieces * b + i < pieces) dst[i] = ld_stream16(reinterpret_cast<const int32_t*>(base + i));
-  };
-
-  // Start row r on this lane.  Rows of length 0 are finished at once; rows
-  // with an invalid length are reported and written as 0.
-  auto begin_row = [&](int64_t r) {
-    row = r;
-    pos = 0;
-    blk = 0;
-    lo = seed_lo;
-    hi = seed_hi;
-    src = tokens + r * (int64_t)stride;
-    int32_t L = lens ? __ldg(lens + r) : stride;
-    if (L < 0 || L > stride) {
-      set_error(err, kErrInvalidArg);
-      fp_out[r] = 0ull;
-      busy = false;
-      return;
-    }
-    len = L;
-    if (L == 0) {
-      fp_out[r] = seed;
-      busy = false;
-      return;
-    }
-    pieces = (L + 3) >> 2;
-    full = L >> 2;
-    if (VEC) load_block(0, buf);
-    busy = true;
-  };
-
   int64_t next = r_begin;
   for (;;) {
-    // Hand unclaimed rows to idle lanes, in lane order.
     unsigned idle = __ballot_sync(0xffffffffu, !busy);
     while (idle != 0u && next < r_end) {
       const int64_t avail = r_end - next;
       const int rank = __popc(idle & lanemask_lt());
-      if (!busy && rank < avail) begin_row(next + rank);
+      if (!busy && rank < avail) {
+        const int64_t r = next + rank;
+        int32_t L = lens ? __ldg(lens + r) : stride;
+        if (L < 0 || L > stride) {
+          set_error(err, kErrInvalidArg);
+          fp_out[r] = 0ull;
+        } else if (L == 0) {
+          fp_out[r] = seed;
+        } else {
+          row = r;
+          pos = 0;
+          len = L;
+          lo = seed_lo;
+          hi = seed_hi;
+          src = tokens + r * (int64_t)stride;
+          busy = true;
+        }
+      }
       next += min((int64_t)__popc(idle), avail);
       idle = __ballot_sync(0xffffffffu, !busy);
     }
     if (!__any_sync(0xffffffffu, busy)) break;
     if (busy) {
-      if (VEC) {
-        int4 nxt[kBlockPieces];
-        const bool more = kBlockPieces * (blk + 1) < pieces;
-        if (more) load_block(blk + 1, nxt);
+      const int32_t rem = len - pos;
+      const int32_t m = rem < 16 ? rem : 16;
 #pragma unroll
-        for (int i = 0; i < kBlockPieces; ++i) {
-          const int pi = kBlockPieces * blk + i;
-          if (pi < full)
-            hash4(lo, hi, buf[i]);
-          else if (pi < pieces)
-            hash_partial(lo, hi, buf[i], len & 3);
-        }
-        if (more) {
-#pragma unroll
-          for (int i = 0; i < kBlockPieces; ++i) buf[i] = nxt[i];
-          ++blk;
-        } else {
-          fp_out[row] = ((uint64_t)hi << 32) | lo;
-          busy = false;
-        }
-      } else {
-        const int32_t rem = len - pos;
-        const int32_t m = rem < 16 ? rem : 16;
-#pragma unroll
-        for (int j = 0; j < 16; ++j)
-          if (j < m) hash_word(lo, hi, (uint32_t)__ldg(src + pos + j));
-        pos += m;
-        if (pos >= len) {
-          fp_out[row] = ((uint64_t)hi << 32) | lo;
-          busy = false;
-        }
+      for (int j = 0; j < 16; ++j)
+        if (j < m) hash_word(lo, hi, (uint32_t)__ldg(src + pos + j));
+      pos += m;
+      if (pos >= len) {
+        fp_out[row] = ((uint64_t)hi << 32) | lo;
+        busy = false;
       }
     }
   }
-}
-
-int resident_warps(const void* kernel) {
-  static int cached[2] = {0, 0};
-  const int slot = (kernel == (const void*)fingerprint_kernel<true>) ? 0 : 1;
-  if (cached[slot] == 0) {
-    int blocks = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&blocks, kernel, 256, 0) != cudaSuccess ||
-        blocks < 1)
-      blocks = 1;
-    cached[slot] = blocks * 8 * num_sms();
-  }
-  return cached[slot];
 }
 
 }  // namespace
@@ -221,22 +278,29 @@ hs_status launch_fingerprint(const int32_t* tokens, int64_t n, int32_t stride,
                              const int32_t* lens, uint64_t seed, uint64_t* fp_out,
                              cudaStream_t stream) {
   const bool vec = ((reinterpret_cast<uintptr_t>(tokens) & 15u) == 0) && (stride % 4 == 0);
-  const void* kfn = vec ? (const void*)fingerprint_kernel<true>
-                        : (const void*)fingerprint_kernel<false>;
-  const int64_t warps_target = resident_warps(kfn);
-  // At least one row per lane; more rows per warp once the grid is full.
-  int64_t rpw = (n + warps_target - 1) / warps_target;
-  if (rpw < 32) rpw = 32;
-  const int64_t warps = (n + rpw - 1) / rpw;
-  const int64_t blocks = (warps + 7) / 8;
   unsigned* err = device_error_word();
   if (!err) return fail(HS_ERR_CUDA, "could not resolve the device error word");
-  if (vec)
-    fingerprint_kernel<true><<<(unsigned)blocks, 256, 0, stream>>>(tokens, n, stride, lens, seed,
-                                                                    fp_out, rpw, err);
-  else
-    fingerprint_kernel<false><<<(unsigned)blocks, 256, 0, stream>>>(tokens, n, stride, lens,
-                                                                     seed, fp_out, rpw, err);
+  const int64_t sms = num_sms();
+  if (vec) {
+    // 64-thread blocks, up to 8 per SM (shared-memory rings of 25.6 KB): at
+    // least one row per lane, more once 16 warps per SM are busy.
+    const int64_t warps_target = sms * 16;
+    int64_t rpw = (n + warps_target - 1) / warps_target;
+    if (rpw < 32) rpw = 32;
+    const int64_t warps = (n + rpw - 1) / rpw;
+    const int64_t blocks = (warps + 1) / 2;
+    const size_t smem = (size_t)kFpThreads * kLaneBytes;
+    fingerprint_async_kernel<<<(unsigned)blocks, kFpThreads, smem, stream>>>(
+        tokens, n, stride, lens, seed, fp_out, rpw, err);
+  } else {
+    const int64_t warps_target = sms * 32;
+    int64_t rpw = (n + warps_target - 1) / warps_target;
+    if (rpw < 32) rpw = 32;
+    const int64_t warps = (n + rpw - 1) / rpw;
+    const int64_t blocks = (warps + 7) / 8;
+    fingerprint_words_kernel<<<(unsigned)blocks, 256, 0, stream>>>(tokens, n, stride, lens, seed,
+                                                                   fp_out, rpw, err);
+  }
   count_launches(1);
   return cuda_fail(cudaGetLastError(), "fingerprint launch");
 }

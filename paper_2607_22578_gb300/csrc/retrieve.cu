@@ -110,27 +110,68 @@ __device__ void flush_candidates(float* cs, int32_t* ci, int et, int& cnt, float
     ci[(b + 1) * kEpi + et] = i;
   }
   // Merge with the current list (all of whose entries have lower corpus
-  // indices: on equal scores the list entry wins).
+  // indices: on equal scores the list entry wins).  The list is consumed in
+  // order, so its addresses are known ahead of the comparisons: it is read in
+  // windows of 8 with the next window in flight, not one dependent load at a
+  // time.
+  constexpr int Wn = 8;
   const float* As = Ls + (size_t)cur * k;
   const int32_t* Ai = Li + (size_t)cur * k;
   float* Os = Ls + (size_t)(cur ^ 1) * k;
   int32_t* Oi = Li + (size_t)(cur ^ 1) * k;
-  int a = 0, b = 0;
-  for (int o = 0; o < k; ++o) {
-    const float sb = b < cnt ? cs[b * kEpi + et] : -FLT_MAX;
-    const float sa = As[a];
-    if (b < cnt && sb > sa) {
-      Os[o] = sb;
-      Oi[o] = ci[b * kEpi + et];
-      ++b;
-    } else {
-      Os[o] = sa;
-      Oi[o] = Ai[a];
-      ++a;
+  float wa[Wn];
+  int32_t wi[Wn];
+#pragma unroll
+  for (int e = 0; e < Wn; ++e) {
+    wa[e] = e < k ? As[e] : -FLT_MAX;
+    wi[e] = e < k ? Ai[e] : -1;
+  }
+  int b = 0, o = 0;
+  float sb = cs[et];
+  int32_t ib = ci[et];
+  float last = -FLT_MAX;
+  for (int a0 = 0; a0 < k && o < k; a0 += Wn) {
+    float na[Wn];
+    int32_t ni[Wn];
+    const bool more = a0 + Wn < k;
+    if (more) {
+#pragma unroll
+      for (int e = 0; e < Wn; ++e) {
+        const bool in = a0 + Wn + e < k;
+        na[e] = in ? As[a0 + Wn + e] : -FLT_MAX;
+        ni[e] = in ? Ai[a0 + Wn + e] : -1;
+      }
+    }
+#pragma unroll
+    for (int e = 0; e < Wn; ++e) {
+      while (b < cnt && o < k && sb > wa[e]) {
+        Os[o] = sb;
+        Oi[o] = ib;
+        last = sb;
+        ++o;
+        ++b;
+        if (b < cnt) {
+          sb = cs[b * kEpi + et];
+          ib = ci[b * kEpi + et];
+        }
+      }
+      if (o < k && a0 + e < k) {
+        Os[o] = wa[e];
+        Oi[o] = wi[e];
+        last = wa[e];
+        ++o;
+      }
+    }
+    if (more) {
+#pragma unroll
+      for (int e = 0; e < Wn; ++e) {
+        wa[e] = na[e];
+        wi[e] = ni[e];
+      }
     }
   }
   cur ^= 1;
-  theta = Os[k - 1];
+  theta = last;  // the k-th entry of the new list
   cnt = 0;
 }
 
@@ -326,9 +367,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
           } else {
 #pragma unroll
-            for (int j0 = 0; j0 < 32; j0 += 8) {
+            for (int j0 = 0; j0 < 32; j0 += 4) {
 #pragma unroll
-              for (int j = j0; j < j0 + 8; ++j) {
+              for (int j = j0; j < j0 + 4; ++j) {
                 const float s = __uint_as_float(r[j]);
                 if (s > theta) {
                   cand_s[cnt * kEpi + et] = s;
@@ -336,7 +377,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                   ++cnt;
                 }
               }
-              if (__any_sync(0xffffffffu, cnt > kCap - 8))
+              if (__any_sync(0xffffffffu, cnt > kCap - 4))
                 flush_candidates(cand_s, cand_i, et, cnt, Ls, Li, k, cur, theta);
             }
           }
