@@ -538,7 +538,12 @@ def row_large_corpus(args, dev, peaks) -> dict:
 
     import paper_2607_22578_gb300 as hs
     from synth import configs
-    w = configs.build_large_corpus(seed=args.seed)
+    cfg = dict(configs.LARGE_CORPUS)
+    if args.k:
+        cfg["k"] = args.k
+    if args.corpus_rows:
+        cfg["N"] = args.corpus_rows
+    w = configs.build_large_corpus(cfg, seed=args.seed)
     corpus, queries = _dev_array(w["corpus"], dev), _dev_array(w["queries"], dev)
     N, d = w["corpus"].shape
     Q, k = w["queries"].shape[0], w["k"]
@@ -558,8 +563,8 @@ def row_large_corpus(args, dev, peaks) -> dict:
     torch.cuda.synchronize()
     hs.hs_get_device_error()
     ms = e0.elapsed_time(e1) / K
-    return {"workload": "large_corpus: 4096 merged queries x 8,388,608 x 1024 bf16 "
-                        "(1024 planted clusters), k=100",
+    return {"workload": "large_corpus: %d merged queries x %d x %d bf16 "
+                        "(1024 planted clusters), k=%d" % (Q, N, d, k),
             "metric": "merged queries/s", "value": Q / (ms / 1e3), "steps": K,
             "retrieval": _roof(2.0 * N * d, 2.0 * Q * N * d, ms, peaks)}
 
@@ -628,6 +633,9 @@ def main() -> int:
                     choices=["rag_mix", "dedup_heavy", "batch_sweep", "large_corpus"],
                     help="rag_mix is the headline step; the others measure the other "
                          "rows of the hot-path table (one GPU)")
+    ap.add_argument("--k", type=int, default=0, help="override k (large_corpus only)")
+    ap.add_argument("--corpus-rows", type=int, default=0,
+                    help="override the corpus size (large_corpus only; for profiling)")
     ap.add_argument("--breakdown", action="store_true",
                     help="add per-phase device times of the rag_mix step")
     args = ap.parse_args()

@@ -140,6 +140,15 @@ __global__ void __launch_bounds__(kFpThreads) fingerprint_async_kernel(
   // Hash side.
   uint32_t lo = seed_lo, hi = seed_hi;
   int64_t next = r_begin;
+  // Row lengths of the next 64 rows of the warp's range, prefetched: lane j
+  // holds rows wbase+j (len_a) and wbase+32+j (len_b); claims read them by
+  // shuffle, so claiming a row never waits on memory.
+  const uint32_t lane = threadIdx.x & 31u;
+  int64_t wbase = r_begin;
+  auto len_of = [&](int64_t r) -> int32_t {
+    return r < r_end ? (lens ? __ldg(lens + r) : stride) : 0;
+  };
+  int32_t len_a = len_of(wbase + lane), len_b = len_of(wbase + 32 + lane);
 
   for (;;) {
 #pragma unroll
@@ -149,9 +158,12 @@ __global__ void __launch_bounds__(kFpThreads) fingerprint_async_kernel(
       while (need != 0u && next < r_end) {
         const int64_t avail = r_end - next;
         const int rank = __popc(need & lanemask_lt());
+        const int off = (int)(next - wbase) + (irow < 0 ? rank : 0);  // 0..62
+        const int32_t La = __shfl_sync(0xffffffffu, len_a, off & 31);
+        const int32_t Lb = __shfl_sync(0xffffffffu, len_b, off & 31);
         if (irow < 0 && rank < avail) {
           const int64_t r = next + rank;
-          int32_t L = lens ? __ldg(lens + r) : stride;
+          const int32_t L = off < 32 ? La : Lb;
           if (L < 0 || L > stride) {
             set_error(err, kErrInvalidArg);
             fp_out[r] = 0ull;
@@ -165,6 +177,11 @@ __global__ void __launch_bounds__(kFpThreads) fingerprint_async_kernel(
           }
         }
         next += min((int64_t)__popc(need), avail);
+        if (next - wbase >= 32) {        // slide the length window by 32 rows
+          wbase += 32;
+          len_a = len_b;
+          len_b = len_of(wbase + 32 + lane);
+        }
         need = __ballot_sync(0xffffffffu, irow < 0);
       }
       // ---- issue one block into slot si
@@ -230,14 +247,23 @@ __global__ void __launch_bounds__(256) fingerprint_words_kernel(
   uint32_t lo = seed_lo, hi = seed_hi;
   const int32_t* src = tokens;
   int64_t next = r_begin;
+  const uint32_t lane = threadIdx.x & 31u;
+  int64_t wbase = r_begin;
+  auto len_of = [&](int64_t r) -> int32_t {
+    return r < r_end ? (lens ? __ldg(lens + r) : stride) : 0;
+  };
+  int32_t len_a = len_of(wbase + lane), len_b = len_of(wbase + 32 + lane);
   for (;;) {
     unsigned idle = __ballot_sync(0xffffffffu, !busy);
     while (idle != 0u && next < r_end) {
       const int64_t avail = r_end - next;
       const int rank = __popc(idle & lanemask_lt());
+      const int off = (int)(next - wbase) + (!busy ? rank : 0);
+      const int32_t La = __shfl_sync(0xffffffffu, len_a, off & 31);
+      const int32_t Lb = __shfl_sync(0xffffffffu, len_b, off & 31);
       if (!busy && rank < avail) {
         const int64_t r = next + rank;
-        int32_t L = lens ? __ldg(lens + r) : stride;
+        const int32_t L = off < 32 ? La : Lb;
         if (L < 0 || L > stride) {
           set_error(err, kErrInvalidArg);
           fp_out[r] = 0ull;
@@ -254,6 +280,11 @@ __global__ void __launch_bounds__(256) fingerprint_words_kernel(
         }
       }
       next += min((int64_t)__popc(idle), avail);
+      if (next - wbase >= 32) {
+        wbase += 32;
+        len_a = len_b;
+        len_b = len_of(wbase + 32 + lane);
+      }
       idle = __ballot_sync(0xffffffffu, !busy);
     }
     if (!__any_sync(0xffffffffu, busy)) break;
