@@ -91,13 +91,14 @@ __device__ __forceinline__ void hash_partial(uint32_t& lo, uint32_t& hi, const i
 // shared memory, filled by cp.async (16-byte, L2-only) kDepth-1 blocks ahead
 // of the block it hashes.  The issue side claims the next row as soon as the
 // current one is fully issued, so a row boundary costs no exposed latency.
-// In-flight data lives in shared memory, not registers, so occupancy stays
-// high.  The ring is padded by 16 bytes per lane so the eight lanes of a
+// In-flight data lives in shared memory, not registers: with a 3-slot ring
+// and 128-thread blocks, eight blocks (32 warps) fit on an SM.  The ring is
+// padded by 16 bytes per lane (208 B = 13 x 16 B) so the eight lanes of a
 // quarter-warp read different banks.
-constexpr int kDepth = 6;
+constexpr int kDepth = 3;
 constexpr int kBlockWords = 16;
 constexpr int kLaneBytes = kDepth * kBlockWords * 4 + 16;
-constexpr int kFpThreads = 64;
+constexpr int kFpThreads = 128;
 
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
@@ -110,7 +111,31 @@ __device__ __forceinline__ void cp_async_wait() {
   asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
-__global__ void __launch_bounds__(kFpThreads) fingerprint_async_kernel(
+__device__ __forceinline__ uint32_t word_of(const int4& v, int j) {
+  return (uint32_t)(j == 0 ? v.x : (j == 1 ? v.y : (j == 2 ? v.z : v.w)));
+}
+
+// Hash the first w (1..16) tokens of a block held in shared memory.  One
+// compact body: the four-token fast path when all four tokens are below 65536,
+// else token by token.
+__device__ __forceinline__ void hash_block(uint32_t& lo, uint32_t& hi, const int4* blk, int w) {
+#pragma unroll 1
+  for (int pc = 0; 4 * pc < w; ++pc) {
+    const int4 v = blk[pc];
+    const int nw = min(4, w - 4 * pc);
+    if (nw == 4 && (((uint32_t)v.x | (uint32_t)v.y | (uint32_t)v.z | (uint32_t)v.w) >> 16) == 0u) {
+      hash_word_small(lo, hi, (uint32_t)v.x);
+      hash_word_small(lo, hi, (uint32_t)v.y);
+      hash_word_small(lo, hi, (uint32_t)v.z);
+      hash_word_small(lo, hi, (uint32_t)v.w);
+    } else {
+#pragma unroll 1
+      for (int j = 0; j < nw; ++j) hash_word(lo, hi, word_of(v, j));
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kFpThreads, 8) fingerprint_async_kernel(
     const int32_t* __restrict__ tokens, int64_t n, int32_t stride,
     const int32_t* __restrict__ lens, uint64_t seed, uint64_t* __restrict__ fp_out,
     int64_t rows_per_warp, unsigned* err) {
@@ -127,15 +152,13 @@ __global__ void __launch_bounds__(kFpThreads) fingerprint_async_kernel(
   int64_t irow = -1;
   int32_t ipos = 0, ilen = 0;
   const int32_t* isrc = tokens;
-  // Per-slot metadata: row (or -1), valid words, first/last block of the row.
+  // Per-slot metadata: row (or -1) and info = words | first << 8 | last << 9.
   int64_t m_row[kDepth];
-  int32_t m_words[kDepth];
-  bool m_first[kDepth], m_last[kDepth];
+  int32_t m_info[kDepth];
 #pragma unroll
   for (int s = 0; s < kDepth; ++s) {
     m_row[s] = -1;
-    m_words[s] = 0;
-    m_first[s] = m_last[s] = false;
+    m_info[s] = 0;
   }
   // Hash side.
   uint32_t lo = seed_lo, hi = seed_hi;
@@ -192,11 +215,11 @@ __global__ void __launch_bounds__(kFpThreads) fingerprint_async_kernel(
         for (int pc = 0; pc < kBlockWords / 4; ++pc)
           if (4 * pc < words) cp_async16(dst + 16 * pc, isrc + ipos + 4 * pc);
         m_row[si] = irow;
-        m_words[si] = words;
-        m_first[si] = ipos == 0;
+        const bool first = ipos == 0;
         ipos += words;
-        m_last[si] = ipos >= ilen;
-        if (ipos >= ilen) irow = -1;
+        const bool last = ipos >= ilen;
+        m_info[si] = words | (first ? 256 : 0) | (last ? 512 : 0);
+        if (last) irow = -1;
       } else {
         m_row[si] = -1;
       }
@@ -205,21 +228,14 @@ __global__ void __launch_bounds__(kFpThreads) fingerprint_async_kernel(
       const int sc = (si + 1) % kDepth;
       cp_async_wait<kDepth - 1>();
       if (m_row[sc] >= 0) {
-        if (m_first[sc]) {
+        const int32_t info = m_info[sc];
+        if (info & 256) {
           lo = seed_lo;
           hi = seed_hi;
         }
-        const int4* blk = reinterpret_cast<const int4*>(ring_p + sc * kBlockWords * 4);
-        const int32_t w = m_words[sc];
-#pragma unroll
-        for (int pc = 0; pc < kBlockWords / 4; ++pc) {
-          if (4 * pc + 4 <= w) {
-            hash4(lo, hi, blk[pc]);
-          } else if (4 * pc < w) {
-            hash_partial(lo, hi, blk[pc], w - 4 * pc);
-          }
-        }
-        if (m_last[sc]) fp_out[m_row[sc]] = ((uint64_t)hi << 32) | lo;
+        hash_block(lo, hi, reinterpret_cast<const int4*>(ring_p + sc * kBlockWords * 4),
+                   info & 255);
+        if (info & 512) fp_out[m_row[sc]] = ((uint64_t)hi << 32) | lo;
         m_row[sc] = -1;
       }
     }
@@ -313,13 +329,13 @@ hs_status launch_fingerprint(const int32_t* tokens, int64_t n, int32_t stride,
   if (!err) return fail(HS_ERR_CUDA, "could not resolve the device error word");
   const int64_t sms = num_sms();
   if (vec) {
-    // 64-thread blocks, up to 8 per SM (shared-memory rings of 25.6 KB): at
-    // least one row per lane, more once 16 warps per SM are busy.
-    const int64_t warps_target = sms * 16;
+    // 128-thread blocks, eight per SM (26.6 KB rings each): at least one row
+    // per lane, more once 32 warps per SM are busy.
+    const int64_t warps_target = sms * 32;
     int64_t rpw = (n + warps_target - 1) / warps_target;
     if (rpw < 32) rpw = 32;
     const int64_t warps = (n + rpw - 1) / rpw;
-    const int64_t blocks = (warps + 1) / 2;
+    const int64_t blocks = (warps + 3) / 4;
     const size_t smem = (size_t)kFpThreads * kLaneBytes;
     fingerprint_async_kernel<<<(unsigned)blocks, kFpThreads, smem, stream>>>(
         tokens, n, stride, lens, seed, fp_out, rpw, err);

@@ -365,11 +365,27 @@ __device__ bool rows_equal_warp(const int32_t* __restrict__ tokens, int32_t stri
   bool diff = false;
   int32_t done = 0;
   if (VEC) {
+    // Up to three 16-byte pieces of each row per lane in flight per round
+    // trip: a 384-token row is compared in one round trip.
     const int32_t pieces = la >> 2;
-    for (int32_t j = lane; j < pieces; j += 32) {
-      const int4 x = __ldg(reinterpret_cast<const int4*>(ra) + j);
-      const int4 y = __ldg(reinterpret_cast<const int4*>(rb) + j);
-      diff |= (x.x != y.x) | (x.y != y.y) | (x.z != y.z) | (x.w != y.w);
+    const int4* pa = reinterpret_cast<const int4*>(ra);
+    const int4* pb = reinterpret_cast<const int4*>(rb);
+    for (int32_t j0 = 0; j0 < pieces; j0 += 96) {
+      int4 x[3], y[3];
+#pragma unroll
+      for (int u = 0; u < 3; ++u) {
+        const int32_t j = j0 + u * 32 + lane;
+        if (j < pieces) {
+          x[u] = __ldg(pa + j);
+          y[u] = __ldg(pb + j);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 3; ++u) {
+        const int32_t j = j0 + u * 32 + lane;
+        if (j < pieces)
+          diff |= (x[u].x != y[u].x) | (x[u].y != y[u].y) | (x[u].z != y[u].z) | (x[u].w != y[u].w);
+      }
     }
     done = pieces << 2;
   }
