@@ -91,14 +91,15 @@ __device__ __forceinline__ void hash_partial(uint32_t& lo, uint32_t& hi, const i
 // shared memory, filled by cp.async (16-byte, L2-only) kDepth-1 blocks ahead
 // of the block it hashes.  The issue side claims the next row as soon as the
 // current one is fully issued, so a row boundary costs no exposed latency.
-// In-flight data lives in shared memory, not registers: with a 3-slot ring
-// and 128-thread blocks, eight blocks (32 warps) fit on an SM.  The ring is
-// padded by 16 bytes per lane (208 B = 13 x 16 B) so the eight lanes of a
-// quarter-warp read different banks.
-constexpr int kDepth = 3;
+// In-flight data lives in shared memory, not registers.  Many rows: a 3-slot
+// ring and 128-thread blocks, eight blocks (32 warps) per SM.  Few rows (too
+// few to fill the SMs that way): an 8-slot ring and one-warp blocks, so each
+// lane keeps seven blocks in flight and the warps spread over all SMs.  The
+// ring is padded to an odd multiple of 16 bytes per lane so the eight lanes
+// of a quarter-warp read different banks.
 constexpr int kBlockWords = 16;
-constexpr int kLaneBytes = kDepth * kBlockWords * 4 + 16;
-constexpr int kFpThreads = 128;
+template <int D>
+constexpr int lane_bytes() { return D * kBlockWords * 4 + 16; }  // odd multiple of 16 B
 
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
@@ -135,7 +136,8 @@ __device__ __forceinline__ void hash_block(uint32_t& lo, uint32_t& hi, const int
   }
 }
 
-__global__ void __launch_bounds__(kFpThreads, 8) fingerprint_async_kernel(
+template <int kDepth, int kFpThreads>
+__global__ void __launch_bounds__(kFpThreads) fingerprint_async_kernel(
     const int32_t* __restrict__ tokens, int64_t n, int32_t stride,
     const int32_t* __restrict__ lens, uint64_t seed, uint64_t* __restrict__ fp_out,
     int64_t rows_per_warp, unsigned* err) {
@@ -144,6 +146,7 @@ __global__ void __launch_bounds__(kFpThreads, 8) fingerprint_async_kernel(
   const int64_t r_begin = warp * rows_per_warp;
   if (r_begin >= n) return;
   const int64_t r_end = min(n, r_begin + rows_per_warp);
+  constexpr int kLaneBytes = lane_bytes<kDepth>();
   const uint32_t ring = smem_u32(ring_all + threadIdx.x * kLaneBytes);
   const uint8_t* ring_p = ring_all + threadIdx.x * kLaneBytes;
   const uint32_t seed_lo = (uint32_t)seed, seed_hi = (uint32_t)(seed >> 32);
@@ -329,16 +332,21 @@ hs_status launch_fingerprint(const int32_t* tokens, int64_t n, int32_t stride,
   if (!err) return fail(HS_ERR_CUDA, "could not resolve the device error word");
   const int64_t sms = num_sms();
   if (vec) {
-    // 128-thread blocks, eight per SM (26.6 KB rings each): at least one row
-    // per lane, more once 32 warps per SM are busy.
-    const int64_t warps_target = sms * 32;
-    int64_t rpw = (n + warps_target - 1) / warps_target;
-    if (rpw < 32) rpw = 32;
-    const int64_t warps = (n + rpw - 1) / rpw;
-    const int64_t blocks = (warps + 3) / 4;
-    const size_t smem = (size_t)kFpThreads * kLaneBytes;
-    fingerprint_async_kernel<<<(unsigned)blocks, kFpThreads, smem, stream>>>(
-        tokens, n, stride, lens, seed, fp_out, rpw, err);
+    const int64_t lanes_full = sms * 32 * 32;   // 32 warps per SM, one row per lane
+    if (n >= lanes_full) {
+      // 128-thread blocks, eight per SM (26.6 KB rings each).
+      const int64_t warps_target = sms * 32;
+      const int64_t rpw = (n + warps_target - 1) / warps_target;
+      const int64_t warps = (n + rpw - 1) / rpw;
+      const int64_t blocks = (warps + 3) / 4;
+      fingerprint_async_kernel<3, 128><<<(unsigned)blocks, 128, 128 * lane_bytes<3>(), stream>>>(
+          tokens, n, stride, lens, seed, fp_out, rpw, err);
+    } else {
+      // One row per lane, one-warp blocks with 8-slot rings (16.9 KB).
+      const int64_t warps = (n + 31) / 32;
+      fingerprint_async_kernel<8, 32><<<(unsigned)warps, 32, 32 * lane_bytes<8>(), stream>>>(
+          tokens, n, stride, lens, seed, fp_out, 32, err);
+    }
   } else {
     const int64_t warps_target = sms * 32;
     int64_t rpw = (n + warps_target - 1) / warps_target;

@@ -393,26 +393,92 @@ __device__ bool rows_equal_warp(const int32_t* __restrict__ tokens, int32_t stri
   return !__any_sync(0xffffffffu, diff);
 }
 
+// Verify: lane i of a warp loads the metadata of position p0+i (segment head,
+// row index, head row, both lengths) so the dependent lookups of 32 positions
+// share their round trips; then the two half-warps compare two pairs of rows
+// at a time, 16 lanes x up to 6 pieces of each row in flight.
+template <bool VEC>
+__device__ __forceinline__ bool half_rows_differ(const int32_t* __restrict__ tokens,
+                                                 int32_t stride, int64_t a, int64_t b, int32_t len,
+                                                 int hl) {
+  const int32_t* ra = tokens + a * (int64_t)stride;
+  const int32_t* rb = tokens + b * (int64_t)stride;
+  bool diff = false;
+  int32_t done = 0;
+  if (VEC) {
+    const int32_t pieces = len >> 2;
+    const int4* pa = reinterpret_cast<const int4*>(ra);
+    const int4* pb = reinterpret_cast<const int4*>(rb);
+    for (int32_t j0 = 0; j0 < pieces; j0 += 96) {
+      int4 x[6], y[6];
+#pragma unroll
+      for (int u = 0; u < 6; ++u) {
+        const int32_t j = j0 + u * 16 + hl;
+        if (j < pieces) {
+          x[u] = __ldg(pa + j);
+          y[u] = __ldg(pb + j);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 6; ++u) {
+        const int32_t j = j0 + u * 16 + hl;
+        if (j < pieces)
+          diff |= (x[u].x != y[u].x) | (x[u].y != y[u].y) | (x[u].z != y[u].z) | (x[u].w != y[u].w);
+      }
+    }
+    done = pieces << 2;
+  }
+  for (int32_t t = done + hl; t < len; t += 16) diff |= (__ldg(ra + t) != __ldg(rb + t));
+  return diff;
+}
+
 template <bool VEC>
 __global__ void __launch_bounds__(256) verify_kernel(
     const uint32_t* __restrict__ vals, const int32_t* __restrict__ seg_head, int64_t n,
     const int32_t* __restrict__ tokens, int32_t stride, const int32_t* __restrict__ lens,
     int32_t* __restrict__ rep, int32_t* coll_flag, int32_t* coll_list, uint32_t* coll_count,
     unsigned* err) {
-  const int lane = threadIdx.x & 31;
+  const int lane = threadIdx.x & 31, half = lane >> 4, hl = lane & 15;
   const int64_t warps = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  for (int64_t p = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; p < n; p += warps) {
-    const int32_t h = seg_head[p];
-    const int64_t a = vals[p];
-    if (h == (int32_t)p) {
-      if (lane == 0) rep[a] = (int32_t)a;
-      continue;
+  const int64_t w = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  for (int64_t p0 = w * 32; p0 < n; p0 += warps * 32) {
+    const int64_t p = p0 + lane;
+    const bool valid = p < n;
+    const int32_t h = valid ? seg_head[p] : 0;
+    const bool head = valid && h == (int32_t)p;
+    const int64_t a = valid ? (int64_t)vals[p] : 0;
+    const int64_t b = (valid && !head) ? (int64_t)vals[h] : a;
+    const int32_t la = valid ? clamp_len(lens, a, stride, err) : 0;
+    const int32_t lb = (valid && !head) ? clamp_len(lens, b, stride, err) : la;
+    bool need = valid && !head;
+    if (head) rep[a] = (int32_t)a;
+    if (need && la != lb) {               // different lengths: never equal
+      rep[a] = (int32_t)a;
+      if (atomicCAS(coll_flag + h, 0, 1) == 0) coll_list[atomicAdd(coll_count, 1u)] = h;
+      need = false;
     }
-    const int64_t b = vals[h];
-    const bool eq = rows_equal_warp<VEC>(tokens, stride, lens, a, b, err);
-    if (lane == 0) {
-      rep[a] = eq ? (int32_t)b : (int32_t)a;
-      if (!eq && atomicCAS(coll_flag + h, 0, 1) == 0) coll_list[atomicAdd(coll_count, 1u)] = h;
+    unsigned todo = __ballot_sync(0xffffffffu, need);
+    while (todo != 0u) {
+      const int j0 = __ffs(todo) - 1;
+      todo &= todo - 1;
+      int j1 = -1;
+      if (todo != 0u) {
+        j1 = __ffs(todo) - 1;
+        todo &= todo - 1;
+      }
+      const int j = half == 0 ? j0 : j1;
+      const int src = j < 0 ? 0 : j;
+      const int64_t aj = __shfl_sync(0xffffffffu, a, src);
+      const int64_t bj = __shfl_sync(0xffffffffu, b, src);
+      const int32_t lj = __shfl_sync(0xffffffffu, la, src);
+      const int32_t hj = __shfl_sync(0xffffffffu, h, src);
+      const bool diff = j >= 0 && half_rows_differ<VEC>(tokens, stride, aj, bj, lj, hl);
+      const unsigned dm = __ballot_sync(0xffffffffu, diff);
+      const bool eq = ((dm >> (half * 16)) & 0xffffu) == 0u;
+      if (j >= 0 && hl == 0) {
+        rep[aj] = eq ? (int32_t)bj : (int32_t)aj;
+        if (!eq && atomicCAS(coll_flag + hj, 0, 1) == 0) coll_list[atomicAdd(coll_count, 1u)] = hj;
+      }
     }
   }
 }
@@ -541,7 +607,7 @@ hs_status launch_unique_inverse(const uint64_t* fp, const int32_t* tokens, int64
       HeadPos{skeys}, n, seg_head, scan0, ctr + 8, nullptr, err);
 
   const bool vec = ((reinterpret_cast<uintptr_t>(tokens) & 15u) == 0) && (stride % 4 == 0);
-  const unsigned vgrid = grid_for(n * 32, 256, sms * 16);
+  const unsigned vgrid = grid_for(n, 256, sms * 8);   // one warp per 32 positions
   if (vec)
     verify_kernel<true><<<vgrid, 256, 0, stream>>>(svals, seg_head, n, tokens, stride, lens, rep,
                                                    coll_flag, coll_list, coll_count, err);
