@@ -268,8 +268,9 @@ def gpu_arm(args, rank: int, local_rank: int, world: int) -> int:
         return stage.retrieve(queries, ev)
 
     for _ in range(args.warmup):
-        _, _, n_u = step()
+        _, _, nu_dev = step()
     hs.hs_get_device_error()
+    n_u = int(nu_dev.item())
 
     K = args.steps
     rev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
@@ -282,7 +283,7 @@ def gpu_arm(args, rank: int, local_rank: int, world: int) -> int:
     l0 = hs.hs_launch_count()
     start.record()
     for i in range(K):
-        _, _, n_u = step(rev[i])
+        step(rev[i])
     end.record()
     torch.cuda.synchronize()
     barrier(world)
@@ -311,11 +312,11 @@ def gpu_arm(args, rank: int, local_rank: int, world: int) -> int:
         d_tok.copy_(h_tokens, non_blocking=True)
         d_q.view(torch.int16).copy_(h_queries, non_blocking=True)
         stage.dedup_chunks(d_tok)
-        s, i, nu = stage.retrieve(d_q)
+        s, i, _ = stage.retrieve(d_q)
         h_s.copy_(s, non_blocking=True)
         h_i.copy_(i, non_blocking=True)
         torch.cuda.current_stream().synchronize()   # the results are read on the host
-        return nu
+        return n_u
 
     for _ in range(3):
         e2e_step()
@@ -512,9 +513,10 @@ def row_batch_sweep(args, dev, peaks) -> dict:
         for i, q in enumerate(batches):
             e0, e1, r0, r1 = _ev(), _ev(), _ev(), _ev()
             e0.record()
-            _, _, nu = stage.retrieve(q, (r0, r1))
+            _, _, nu_dev = stage.retrieve(q, (r0, r1))
             e1.record()
             torch.cuda.synchronize()
+            nu = int(nu_dev.item())
             if i >= 3:
                 lat.append(e0.elapsed_time(e1))
                 ret.append(r0.elapsed_time(r1))
@@ -570,33 +572,35 @@ def row_large_corpus(args, dev, peaks) -> dict:
 
 
 def rag_mix_breakdown(stage, tokens, queries, K: int) -> dict:
-    """Per-phase device time of the RAG-mix step (same calls as the step)."""
+    """Per-phase device time of the RAG-mix step (the same calls as the
+    pipeline, with events between them)."""
     import torch
 
     import paper_2607_22578_gb300 as hs
     from paper_2607_22578_gb300 import _lib
     names = ["chunk_fingerprint", "chunk_unique", "query_fingerprint", "query_unique",
-             "count_sync_and_gather", "retrieve_topk", "scatter_results"]
+             "gather_unique_queries", "retrieve_topk", "scatter_results"]
     acc = {n: 0.0 for n in names}
+    Q = queries.shape[0]
     for _ in range(K):
         ev = [_ev() for _ in range(len(names) + 1)]
         ev[0].record()
-        fp = _lib.hs_fingerprint(tokens)
+        fp = _lib.hs_fingerprint(tokens, fp_out=stage.c_fp[:tokens.shape[0]])
         ev[1].record()
         _lib.hs_unique_inverse(fp, tokens, workspace=stage.ws_c, out=stage.c_out)
         ev[2].record()
         qi32 = queries.view(torch.int32)
-        qfp = _lib.hs_fingerprint(qi32)
+        qfp = _lib.hs_fingerprint(qi32, fp_out=stage.q_fp[:Q])
         ev[3].record()
         nu, uidx, inv = _lib.hs_unique_inverse(qfp, qi32, workspace=stage.ws_q, out=stage.q_out)
         ev[4].record()
-        n_unique = int(nu.item())
-        uq = _lib.hs_scatter_results(queries, uidx[:n_unique])
+        uq = _lib.hs_scatter_results(queries, uidx, dst=stage.uq[:Q])
         ev[5].record()
-        s_u, i_u = _lib.hs_retrieve_topk(uq, stage.corpus, stage.k, workspace=stage.ws_r)
+        s_u, i_u = _lib.hs_retrieve_topk_n(uq, nu, stage.corpus, stage.k, workspace=stage.ws_r,
+                                           out=(stage.s_u[:Q], stage.i_u[:Q]))
         ev[6].record()
-        _lib.hs_scatter_results(s_u, inv)
-        _lib.hs_scatter_results(i_u, inv)
+        _lib.hs_scatter_results(s_u, inv, dst=stage.scores[:Q])
+        _lib.hs_scatter_results(i_u, inv, dst=stage.ids[:Q])
         ev[7].record()
         torch.cuda.synchronize()
         for i, n in enumerate(names):

@@ -100,6 +100,8 @@ hs_status hs_fingerprint(const int32_t* tokens, int64_t n_rows, int32_t row_stri
  * tokens[j, 0:len] (words beyond len are ignored).  Outputs:
  *   *n_unique_dev      number of groups,
  *   unique_idx_out[u]  index of group u's first occurrence, ascending in u,
+ *                      for u < *n_unique_dev; 0 for u >= *n_unique_dev, so
+ *                      all n_rows entries form a valid row map,
  *   inverse_out[i]     group ordinal of row i (the redirected edge),
  * so rows[unique_idx[inverse[i]]] == rows[i].  fp must hold fingerprints of
  * these rows that are equal for equal rows (as hs_fingerprint produces with
@@ -114,7 +116,7 @@ hs_status hs_fingerprint(const int32_t* tokens, int64_t n_rows, int32_t row_stri
  * tokens, n_rows, row_stride, lens   as for hs_fingerprint;
  *                 1 <= ... n_rows <= 2^30 - 1 (0 writes *n_unique_dev = 0).
  * n_unique_dev    device int32 scalar.
- * unique_idx_out  device int32 [n_rows] (only the first *n_unique_dev used).
+ * unique_idx_out  device int32 [n_rows].
  * inverse_out     device int32 [n_rows].
  * workspace       device, >= hs_unique_inverse_workspace(n_rows) bytes,
  *                 256-byte aligned; contents on entry are ignored.
@@ -153,6 +155,24 @@ hs_status hs_retrieve_topk(const uint16_t* queries, int64_t n_queries, const uin
                            int64_t n_corpus, int32_t dim, int32_t k, float* scores_out,
                            int32_t* ids_out, void* workspace, size_t workspace_bytes,
                            hs_stream_t stream);
+
+/*
+ * hs_retrieve_topk_n — hs_retrieve_topk with the query count in device
+ * memory, so the merged queries of a batch can be retrieved without a host
+ * synchronisation (Section 3.3: merged nodes execute once).
+ *
+ * Processes the first min(*n_queries_dev, max_queries) rows of `queries`
+ * (rows up to max_queries must be addressable; the count is read on the
+ * device when the kernels run) and writes that many rows of scores_out and
+ * ids_out; later rows are left untouched.  Every other argument is as for
+ * hs_retrieve_topk with n_queries = max_queries, including the workspace
+ * size hs_retrieve_topk_workspace(max_queries, ...).
+ */
+hs_status hs_retrieve_topk_n(const uint16_t* queries, int64_t max_queries,
+                             const int32_t* n_queries_dev, const uint16_t* corpus,
+                             int64_t n_corpus, int32_t dim, int32_t k, float* scores_out,
+                             int32_t* ids_out, void* workspace, size_t workspace_bytes,
+                             hs_stream_t stream);
 
 /*
  * hs_scatter_results — row gather/scatter: dst[i, :] = src[map[i], :].

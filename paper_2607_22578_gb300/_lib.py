@@ -68,6 +68,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
             lib.hs_retrieve_topk_workspace.restype = sz
             lib.hs_retrieve_topk.argtypes = [P, i64, P, i64, i32, i32, P, P, P, sz, P]
             lib.hs_retrieve_topk.restype = st
+            lib.hs_retrieve_topk_n.argtypes = [P, i64, P, P, i64, i32, i32, P, P, P, sz, P]
+            lib.hs_retrieve_topk_n.restype = st
             lib.hs_scatter_results.argtypes = [P, i64, i64, P, i64, P, P]
             lib.hs_scatter_results.restype = st
             lib.hs_get_device_error.argtypes = [P]
@@ -181,6 +183,38 @@ def hs_retrieve_topk(queries: torch.Tensor, corpus: torch.Tensor, k: int,
                                 device=dev)
     _check(load().hs_retrieve_topk(_ptr(queries), Q, _ptr(corpus), N, d, k, _ptr(scores),
                                    _ptr(ids), _ptr(workspace), workspace.numel(), _stream(stream)))
+    return scores, ids
+
+
+def hs_retrieve_topk_n(queries: torch.Tensor, n_queries_dev: torch.Tensor, corpus: torch.Tensor,
+                       k: int, workspace: torch.Tensor | None = None, out: tuple | None = None,
+                       stream=None):
+    """hs_retrieve_topk over the first n_queries_dev[0] rows of `queries`
+    (a device int32 scalar, read when the kernels run).  Returns (scores,
+    ids) shaped like `queries` rows x k; rows past the count are left as
+    they were."""
+    _cuda(queries, "queries")
+    _cuda(corpus, "corpus")
+    _cuda(n_queries_dev, "n_queries_dev")
+    if n_queries_dev.dtype != torch.int32:
+        raise TypeError("n_queries_dev must be int32")
+    if queries.element_size() != 2 or corpus.element_size() != 2:
+        raise TypeError("queries and corpus must hold bf16 (2-byte) elements")
+    Q, d = queries.shape
+    N, d2 = corpus.shape
+    if d != d2:
+        raise ValueError("dimension mismatch")
+    dev = queries.device
+    if out is None:
+        out = (torch.empty((Q, k), dtype=torch.float32, device=dev),
+               torch.empty((Q, k), dtype=torch.int32, device=dev))
+    scores, ids = out
+    if workspace is None:
+        workspace = torch.empty(hs_retrieve_topk_workspace(Q, N, d, k), dtype=torch.uint8,
+                                device=dev)
+    _check(load().hs_retrieve_topk_n(_ptr(queries), Q, _ptr(n_queries_dev), _ptr(corpus), N, d,
+                                     k, _ptr(scores), _ptr(ids), _ptr(workspace),
+                                     workspace.numel(), _stream(stream)))
     return scores, ids
 
 

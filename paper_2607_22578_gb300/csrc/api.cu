@@ -17,8 +17,8 @@ hs_status launch_unique_inverse(const uint64_t*, const int32_t*, int64_t, int32_
                                 const int32_t*, int32_t*, int32_t*, int32_t*, void*,
                                 cudaStream_t);
 size_t retrieve_topk_workspace(int64_t, int64_t, int32_t, int32_t);
-hs_status launch_retrieve_topk(const uint16_t*, int64_t, const uint16_t*, int64_t, int32_t,
-                               int32_t, float*, int32_t*, void*, size_t, cudaStream_t);
+hs_status launch_retrieve_topk(const uint16_t*, int64_t, const int32_t*, const uint16_t*, int64_t,
+                               int32_t, int32_t, float*, int32_t*, void*, size_t, cudaStream_t);
 hs_status launch_scatter(const void*, int64_t, int64_t, const int32_t*, int64_t, void*,
                          cudaStream_t);
 
@@ -142,11 +142,11 @@ size_t hs_retrieve_topk_workspace(int64_t n_queries, int64_t n_corpus, int32_t d
   return retrieve_topk_workspace(n_queries, n_corpus, dim, k);
 }
 
-hs_status hs_retrieve_topk(const uint16_t* queries, int64_t n_queries, const uint16_t* corpus,
-                           int64_t n_corpus, int32_t dim, int32_t k, float* scores_out,
-                           int32_t* ids_out, void* workspace, size_t workspace_bytes,
-                           hs_stream_t stream) {
-  clear_msg();
+static hs_status retrieve_common(const uint16_t* queries, int64_t n_queries,
+                                 const int32_t* n_queries_dev, const uint16_t* corpus,
+                                 int64_t n_corpus, int32_t dim, int32_t k, float* scores_out,
+                                 int32_t* ids_out, void* workspace, size_t workspace_bytes,
+                                 hs_stream_t stream) {
   if (n_queries < 0) return fail(HS_ERR_INVALID_ARG, "n_queries < 0");
   if (n_corpus < 1 || n_corpus > 0x7fffffffLL)
     return fail(HS_ERR_INVALID_ARG, "n_corpus outside [1, 2^31 - 1]");
@@ -163,8 +163,31 @@ hs_status hs_retrieve_topk(const uint16_t* queries, int64_t n_queries, const uin
     return fail(HS_ERR_INVALID_ARG, "scores_out/ids_out misaligned");
   if (!workspace || !aligned(workspace, 256))
     return fail(HS_ERR_WORKSPACE, "workspace NULL or not 256-byte aligned");
-  return launch_retrieve_topk(queries, n_queries, corpus, n_corpus, dim, k, scores_out, ids_out,
-                              workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream));
+  if (n_queries_dev && !aligned(n_queries_dev, 4))
+    return fail(HS_ERR_INVALID_ARG, "n_queries_dev misaligned");
+  return launch_retrieve_topk(queries, n_queries, n_queries_dev, corpus, n_corpus, dim, k,
+                              scores_out, ids_out, workspace, workspace_bytes,
+                              reinterpret_cast<cudaStream_t>(stream));
+}
+
+hs_status hs_retrieve_topk(const uint16_t* queries, int64_t n_queries, const uint16_t* corpus,
+                           int64_t n_corpus, int32_t dim, int32_t k, float* scores_out,
+                           int32_t* ids_out, void* workspace, size_t workspace_bytes,
+                           hs_stream_t stream) {
+  clear_msg();
+  return retrieve_common(queries, n_queries, nullptr, corpus, n_corpus, dim, k, scores_out,
+                         ids_out, workspace, workspace_bytes, stream);
+}
+
+hs_status hs_retrieve_topk_n(const uint16_t* queries, int64_t max_queries,
+                             const int32_t* n_queries_dev, const uint16_t* corpus,
+                             int64_t n_corpus, int32_t dim, int32_t k, float* scores_out,
+                             int32_t* ids_out, void* workspace, size_t workspace_bytes,
+                             hs_stream_t stream) {
+  clear_msg();
+  if (!n_queries_dev) return fail(HS_ERR_INVALID_ARG, "n_queries_dev is NULL");
+  return retrieve_common(queries, max_queries, n_queries_dev, corpus, n_corpus, dim, k,
+                         scores_out, ids_out, workspace, workspace_bytes, stream);
 }
 
 hs_status hs_scatter_results(const void* src, int64_t n_src, int64_t row_bytes,

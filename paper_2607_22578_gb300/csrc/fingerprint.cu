@@ -37,15 +37,16 @@ __device__ __forceinline__ void mul_prime3(uint32_t& lo, uint32_t& hi) {
   lo = (uint32_t)t;
 }
 
-// Octet-wise rounds for one token, little-endian octet order.
+// Octet-wise rounds for one token, little-endian octet order; octets are
+// extracted with byte permutes, no branches.
 __device__ __forceinline__ void hash_word_full(uint32_t& lo, uint32_t& hi, uint32_t w) {
-  lo ^= (w & 0xffu);
+  lo ^= __byte_perm(w, 0u, 0x4440u);
   mul_prime(lo, hi);
-  lo ^= ((w >> 8) & 0xffu);
+  lo ^= __byte_perm(w, 0u, 0x4441u);
   mul_prime(lo, hi);
-  lo ^= ((w >> 16) & 0xffu);
+  lo ^= __byte_perm(w, 0u, 0x4442u);
   mul_prime(lo, hi);
-  lo ^= (w >> 24);
+  lo ^= w >> 24;
   mul_prime(lo, hi);
 }
 
@@ -64,26 +65,7 @@ __device__ __forceinline__ void hash_word(uint32_t& lo, uint32_t& hi, uint32_t w
     hash_word_full(lo, hi, w);
 }
 
-__device__ __forceinline__ void hash4(uint32_t& lo, uint32_t& hi, const int4 v) {
-  const uint32_t a = (uint32_t)v.x, b = (uint32_t)v.y, c = (uint32_t)v.z, d = (uint32_t)v.w;
-  if (((a | b | c | d) >> 16) == 0u) {
-    hash_word_small(lo, hi, a);
-    hash_word_small(lo, hi, b);
-    hash_word_small(lo, hi, c);
-    hash_word_small(lo, hi, d);
-  } else {
-    hash_word(lo, hi, a);
-    hash_word(lo, hi, b);
-    hash_word(lo, hi, c);
-    hash_word(lo, hi, d);
-  }
-}
 
-__device__ __forceinline__ void hash_partial(uint32_t& lo, uint32_t& hi, const int4 v, int w) {
-  hash_word(lo, hi, (uint32_t)v.x);
-  if (w > 1) hash_word(lo, hi, (uint32_t)v.y);
-  if (w > 2) hash_word(lo, hi, (uint32_t)v.z);
-}
 
 // ---- vector path: per-lane cp.async pipeline ----------------------------------------
 // A lane owns one row at a time.  Its row is cut into blocks of 16 tokens
@@ -124,11 +106,18 @@ __device__ __forceinline__ void hash_block(uint32_t& lo, uint32_t& hi, const int
   for (int pc = 0; 4 * pc < w; ++pc) {
     const int4 v = blk[pc];
     const int nw = min(4, w - 4 * pc);
-    if (nw == 4 && (((uint32_t)v.x | (uint32_t)v.y | (uint32_t)v.z | (uint32_t)v.w) >> 16) == 0u) {
-      hash_word_small(lo, hi, (uint32_t)v.x);
-      hash_word_small(lo, hi, (uint32_t)v.y);
-      hash_word_small(lo, hi, (uint32_t)v.z);
-      hash_word_small(lo, hi, (uint32_t)v.w);
+    if (nw == 4) {
+      if ((((uint32_t)v.x | (uint32_t)v.y | (uint32_t)v.z | (uint32_t)v.w) >> 16) == 0u) {
+        hash_word_small(lo, hi, (uint32_t)v.x);
+        hash_word_small(lo, hi, (uint32_t)v.y);
+        hash_word_small(lo, hi, (uint32_t)v.z);
+        hash_word_small(lo, hi, (uint32_t)v.w);
+      } else {
+        hash_word_full(lo, hi, (uint32_t)v.x);
+        hash_word_full(lo, hi, (uint32_t)v.y);
+        hash_word_full(lo, hi, (uint32_t)v.z);
+        hash_word_full(lo, hi, (uint32_t)v.w);
+      }
     } else {
 #pragma unroll 1
       for (int j = 0; j < nw; ++j) hash_word(lo, hi, word_of(v, j));

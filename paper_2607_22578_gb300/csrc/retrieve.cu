@@ -56,8 +56,9 @@ static_assert((size_t)kCap * kEpi * 8 == kEpiSmem, "candidate buffer size");
 constexpr size_t kSmem = 1024 + (size_t)kStages * kStageBytes + kBarBytes + kEpiSmem;
 
 struct Params {
-  int64_t Q, N, tiles;
-  int32_t k, kb_count, qblocks, nsplit;
+  int64_t Qmax, N, tiles;
+  const int32_t* count_dev;  // queries to process: min(*count_dev, Qmax); NULL: Qmax
+  int32_t k, kb_count, sms;
   float* part_s;     // [Q][2 * nsplit][k]: one list per (split, column half)
   int32_t* part_i;
   float* list_s;     // large-k: [grid][kEpi][2][k]
@@ -65,12 +66,53 @@ struct Params {
   unsigned* err;
 };
 
-__device__ __forceinline__ void unit_coords(const Params& p, int64_t u, int& qb, int& split,
-                                            int64_t& t0, int64_t& t1) {
-  qb = (int)(u % p.qblocks);
-  split = (int)(u / p.qblocks);
-  t0 = (int64_t)split * p.tiles / p.nsplit;
-  t1 = (int64_t)(split + 1) * p.tiles / p.nsplit;
+__host__ __device__ inline int64_t gcd64(int64_t a, int64_t b) {
+  while (b) {
+    const int64_t t = a % b;
+    a = b;
+    b = t;
+  }
+  return a;
+}
+
+// Largest split count a plan may use: every split needs a corpus tile, and
+// the merge sorts 2 * nsplit * k candidates per query.
+__host__ __device__ inline int64_t max_splits(int64_t sms, int64_t tiles, int32_t k) {
+  int64_t ns = sms;
+  if (ns > tiles) ns = tiles;
+  if (ns > kMergeMax / (2 * k)) ns = kMergeMax / (2 * k);
+  return ns < 1 ? 1 : ns;
+}
+
+// Work decomposition for Q queries: query blocks of 128 and corpus splits;
+// units = qblocks * nsplit is a multiple of the SM count when the caps allow.
+// Host and device evaluate the same function, so a launch can take its query
+// count from device memory.
+struct SplitPlan {
+  int32_t qblocks, nsplit;
+};
+__host__ __device__ inline SplitPlan split_plan(int64_t Q, int64_t tiles, int32_t k, int64_t sms) {
+  SplitPlan sp;
+  sp.qblocks = (int32_t)((Q + BM - 1) / BM);
+  int64_t ns = sms / gcd64(sms, sp.qblocks > 0 ? sp.qblocks : 1);
+  const int64_t cap = max_splits(sms, tiles, k);
+  if (ns > cap) ns = cap;
+  sp.nsplit = (int32_t)ns;
+  return sp;
+}
+
+__device__ __forceinline__ int64_t query_count(const Params& p) {
+  if (!p.count_dev) return p.Qmax;
+  const int64_t c = *p.count_dev;
+  return c < 0 ? 0 : (c > p.Qmax ? p.Qmax : c);
+}
+
+__device__ __forceinline__ void unit_coords(const SplitPlan& sp, int64_t tiles, int64_t u, int& qb,
+                                            int& split, int64_t& t0, int64_t& t1) {
+  qb = (int)(u % sp.qblocks);
+  split = (int)(u / sp.qblocks);
+  t0 = (int64_t)split * tiles / sp.nsplit;
+  t1 = (int64_t)(split + 1) * tiles / sp.nsplit;
 }
 
 // Insert (s, idx) into a list sorted by score descending.  idx is larger than
@@ -218,7 +260,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  const int64_t units = (int64_t)p.qblocks * p.nsplit;
+  const int64_t Q = query_count(p);
+  const SplitPlan sp = split_plan(Q, p.tiles, p.k, p.sms);
+  const int64_t units = Q > 0 ? (int64_t)sp.qblocks * sp.nsplit : 0;
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
@@ -229,7 +273,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int64_t u = blockIdx.x; u < units; u += gridDim.x) {
         int qb, split;
         int64_t t0, t1;
-        unit_coords(p, u, qb, split, t0, t1);
+        unit_coords(sp, p.tiles, u, qb, split, t0, t1);
         for (int64_t t = t0; t < t1; ++t) {
           for (int kb = 0; kb < p.kb_count; ++kb) {
             if (!mbar_wait(empty + stage, phase ^ 1u, abort_flag)) goto producer_done;
@@ -254,7 +298,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int64_t u = blockIdx.x; u < units; u += gridDim.x) {
         int qb, split;
         int64_t t0, t1;
-        unit_coords(p, u, qb, split, t0, t1);
+        unit_coords(sp, p.tiles, u, qb, split, t0, t1);
         for (int64_t t = t0; t < t1; ++t, ++tile_i) {
           const uint32_t acc = tile_i & 1u, aphase = (tile_i >> 1) & 1u;
           if (!mbar_wait(tempty + acc, aphase ^ 1u, abort_flag)) goto mma_done;
@@ -289,7 +333,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int et = ew * 32 + lane;            // epilogue thread index, 0..255
     const uint32_t lane_addr = (uint32_t)(quarter * 32) << 16;
     const int k = p.k;
-    const int lists = 2 * p.nsplit;
+    const int lists = 2 * sp.nsplit;
     uint32_t tile_i = 0;
     float* stage_f = reinterpret_cast<float*>(epi_smem);            // KREG: [8][kEpi][4]
     float* cand_s = reinterpret_cast<float*>(epi_smem);             // large k: [kCap][kEpi]
@@ -299,9 +343,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int64_t u = blockIdx.x; u < units; u += gridDim.x) {
       int qb, split;
       int64_t t0, t1;
-      unit_coords(p, u, qb, split, t0, t1);
+      unit_coords(sp, p.tiles, u, qb, split, t0, t1);
       const int64_t q = (int64_t)qb * BM + row;
-      const bool valid_q = q < p.Q;
+      const bool valid_q = q < Q;
       float theta = -FLT_MAX;
       float ls[KREG > 0 ? KREG : 1];
       int32_t li[KREG > 0 ? KREG : 1];
@@ -433,13 +477,18 @@ __device__ __forceinline__ void unpack_key(uint64_t key, float& s, int32_t& idx)
   idx = (int32_t)(0xffffffffu - (uint32_t)key);
 }
 
-__global__ void __launch_bounds__(256) merge_kernel(const float* __restrict__ part_s,
-                                                    const int32_t* __restrict__ part_i, int64_t Q,
-                                                    int32_t lists, int32_t k, int32_t p2,
-                                                    float* __restrict__ out_s,
+__global__ void __launch_bounds__(256) merge_kernel(const Params p, float* __restrict__ out_s,
                                                     int32_t* __restrict__ out_i) {
   extern __shared__ uint64_t keys[];
+  const int64_t Q = query_count(p);
+  const SplitPlan sp = split_plan(Q, p.tiles, p.k, p.sms);
+  const int k = p.k;
+  const int lists = 2 * sp.nsplit;
   const int m = lists * k;
+  int p2 = 1;
+  while (p2 < m) p2 <<= 1;
+  const float* __restrict__ part_s = p.part_s;
+  const int32_t* __restrict__ part_i = p.part_i;
   for (int64_t q = blockIdx.x; q < Q; q += gridDim.x) {
     const float* ps = part_s + (size_t)q * m;
     const int32_t* pi = part_i + (size_t)q * m;
@@ -504,51 +553,10 @@ bool make_map(CUtensorMap* map, const uint16_t* base, int64_t rows, int32_t d, u
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-int64_t gcd64(int64_t a, int64_t b) {
-  while (b) {
-    const int64_t t = a % b;
-    a = b;
-    b = t;
-  }
-  return a;
-}
-
-// Largest split count a plan may use: every split needs a corpus tile, and
-// the merge sorts 2 * nsplit * k candidates per query.
-int64_t max_splits(int64_t sms, int64_t tiles, int32_t k) {
-  int64_t ns = sms;
-  if (ns > tiles) ns = tiles;
-  if (ns > kMergeMax / (2 * k)) ns = kMergeMax / (2 * k);
-  return ns < 1 ? 1 : ns;
-}
-
-struct Plan {
-  int32_t qblocks, nsplit, kreg, p2;
-  int64_t tiles, grid;
-  size_t part_bytes, list_bytes, total;
-};
-
-Plan plan(int64_t Q, int64_t N, int32_t d, int32_t k) {
-  Plan pl{};
-  (void)d;
-  const int64_t sms = num_sms();
-  pl.qblocks = (int32_t)((Q + BM - 1) / BM);
-  pl.tiles = (N + BN - 1) / BN;
-  // Units = qblocks * nsplit is a multiple of the SM count when possible.
-  int64_t ns = sms / gcd64(sms, pl.qblocks > 0 ? pl.qblocks : 1);
-  const int64_t cap = max_splits(sms, pl.tiles, k);
-  if (ns > cap) ns = cap;
-  pl.nsplit = (int32_t)ns;
-  pl.kreg = k <= 16 ? 16 : (k <= 32 ? 32 : 0);
+int p2_for(int64_t nsplit, int32_t k) {
   int p2 = 1;
-  while (p2 < 2 * pl.nsplit * k) p2 <<= 1;
-  pl.p2 = p2;
-  const int64_t units = (int64_t)pl.qblocks * pl.nsplit;
-  pl.grid = units < sms ? units : sms;
-  pl.part_bytes = (((size_t)Q * 2 * pl.nsplit * k * 4) + 255) & ~(size_t)255;
-  pl.list_bytes = pl.kreg ? 0 : ((((size_t)pl.grid * kEpi * 2 * k * 4) + 255) & ~(size_t)255);
-  pl.total = 2 * pl.part_bytes + 2 * pl.list_bytes + 256;
-  return pl;
+  while (p2 < 2 * nsplit * k) p2 <<= 1;
+  return p2;
 }
 
 template <int KREG>
@@ -568,7 +576,7 @@ hs_status launch_kernel(const CUtensorMap& mq, const CUtensorMap& mc, const Para
 }  // namespace
 
 // Upper bound over every query count up to Q: a plan's split count is at most
-// max_splits() and its grid at most the SM count, so one workspace serves
+// max_splits() and the grid is at most the SM count, so one workspace serves
 // every batch of at most Q queries.
 size_t retrieve_topk_workspace(int64_t Q, int64_t N, int32_t d, int32_t k) {
   if (Q <= 0 || N <= 0 || k <= 0) return 256;
@@ -580,41 +588,57 @@ size_t retrieve_topk_workspace(int64_t Q, int64_t N, int32_t d, int32_t k) {
   return 2 * part + 2 * list + 256;
 }
 
-hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Q, const uint16_t* corpus,
-                               int64_t N, int32_t d, int32_t k, float* scores_out,
-                               int32_t* ids_out, void* ws, size_t ws_bytes,
+// Qmax rows of `queries` are addressable; the kernels process the first
+// count of them, count = *count_dev (clamped to [0, Qmax]) or Qmax if
+// count_dev is NULL.
+hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int32_t* count_dev,
+                               const uint16_t* corpus, int64_t N, int32_t d, int32_t k,
+                               float* scores_out, int32_t* ids_out, void* ws, size_t ws_bytes,
                                cudaStream_t stream) {
   unsigned* err = device_error_word();
   if (!err) return fail(HS_ERR_CUDA, "could not resolve the device error word");
-  const Plan pl = plan(Q, N, d, k);
-  if (ws_bytes < pl.total)
-    return fail(HS_ERR_WORKSPACE, "retrieve workspace too small: %zu < %zu", ws_bytes, pl.total);
+  const int64_t sms = num_sms();
+  const int64_t tiles = (N + BN - 1) / BN;
+  const size_t need = retrieve_topk_workspace(Qmax, N, d, k);
+  if (ws_bytes < need)
+    return fail(HS_ERR_WORKSPACE, "retrieve workspace too small: %zu < %zu", ws_bytes, need);
   CUtensorMap mq, mc;
-  if (!make_map(&mq, queries, Q, d, BM) || !make_map(&mc, corpus, N, d, BN))
+  if (!make_map(&mq, queries, Qmax, d, BM) || !make_map(&mc, corpus, N, d, BN))
     return fail(HS_ERR_CUDA, "cuTensorMapEncodeTiled failed (driver entry point or arguments)");
+  const int64_t ns_max = max_splits(sms, tiles, k);
+  const size_t part = (((size_t)Qmax * 2 * ns_max * k * 4) + 255) & ~(size_t)255;
+  const size_t list = k <= 32 ? 0 : ((((size_t)sms * kEpi * 2 * k * 4) + 255) & ~(size_t)255);
   char* w = static_cast<char*>(ws);
   Params prm{};
-  prm.Q = Q;
+  prm.Qmax = Qmax;
   prm.N = N;
-  prm.tiles = pl.tiles;
+  prm.tiles = tiles;
+  prm.count_dev = count_dev;
   prm.k = k;
   prm.kb_count = (d + BK - 1) / BK;
-  prm.qblocks = pl.qblocks;
-  prm.nsplit = pl.nsplit;
+  prm.sms = (int32_t)sms;
   prm.part_s = reinterpret_cast<float*>(w);
-  prm.part_i = reinterpret_cast<int32_t*>(w + pl.part_bytes);
-  prm.list_s = reinterpret_cast<float*>(w + 2 * pl.part_bytes);
-  prm.list_i = reinterpret_cast<int32_t*>(w + 2 * pl.part_bytes + pl.list_bytes);
+  prm.part_i = reinterpret_cast<int32_t*>(w + part);
+  prm.list_s = reinterpret_cast<float*>(w + 2 * part);
+  prm.list_i = reinterpret_cast<int32_t*>(w + 2 * part + list);
   prm.err = err;
+  // With a host-known count the grid is the plan's unit count (capped at the
+  // SM count); with a device count every SM gets a CTA and idle ones exit.
+  int64_t grid = sms;
+  if (!count_dev) {
+    const SplitPlan sp = split_plan(Qmax, tiles, k, sms);
+    const int64_t units = (int64_t)sp.qblocks * sp.nsplit;
+    if (units < grid) grid = units;
+  }
   hs_status st;
-  if (pl.kreg == 16)
-    st = launch_kernel<16>(mq, mc, prm, pl.grid, stream);
-  else if (pl.kreg == 32)
-    st = launch_kernel<32>(mq, mc, prm, pl.grid, stream);
+  if (k <= 16)
+    st = launch_kernel<16>(mq, mc, prm, grid, stream);
+  else if (k <= 32)
+    st = launch_kernel<32>(mq, mc, prm, grid, stream);
   else
-    st = launch_kernel<0>(mq, mc, prm, pl.grid, stream);
+    st = launch_kernel<0>(mq, mc, prm, grid, stream);
   if (st != HS_OK) return st;
-  const size_t msmem = (size_t)pl.p2 * 8;
+  const size_t msmem = (size_t)p2_for(ns_max, k) * 8;
   static size_t merge_configured = 0;
   if (msmem > 48 * 1024 && msmem > merge_configured) {
     cudaError_t e = cudaFuncSetAttribute(merge_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -622,9 +646,8 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Q, const uint16_
     if (e != cudaSuccess) return cuda_fail(e, "merge smem attribute");
     merge_configured = msmem;
   }
-  int64_t mgrid = Q < (int64_t)num_sms() * 8 ? Q : (int64_t)num_sms() * 8;
-  merge_kernel<<<(unsigned)mgrid, 256, msmem, stream>>>(prm.part_s, prm.part_i, Q, 2 * pl.nsplit,
-                                                        k, pl.p2, scores_out, ids_out);
+  const int64_t mgrid = Qmax < sms * 8 ? Qmax : sms * 8;
+  merge_kernel<<<(unsigned)mgrid, 256, msmem, stream>>>(prm, scores_out, ids_out);
   count_launches(2);  // retrieve_kernel + merge_kernel
   return cuda_fail(cudaGetLastError(), "merge launch");
 }

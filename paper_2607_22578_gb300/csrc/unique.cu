@@ -537,13 +537,16 @@ __global__ void __launch_bounds__(256) resolve_kernel(
 
 __global__ void __launch_bounds__(256) finalize_kernel(const int32_t* __restrict__ rep,
                                                        const int32_t* __restrict__ uid, int64_t n,
+                                                       const int32_t* __restrict__ n_unique,
                                                        int32_t* __restrict__ unique_idx,
                                                        int32_t* __restrict__ inverse) {
+  const int64_t nu = *n_unique;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
        i += (int64_t)gridDim.x * blockDim.x) {
     const int32_t r = rep[i];
     inverse[i] = uid[r];
     if (r == (int32_t)i) unique_idx[uid[i]] = (int32_t)i;
+    if (i >= nu) unique_idx[i] = 0;     // the tail is a valid row map too
   }
 }
 
@@ -623,8 +626,8 @@ hs_status launch_unique_inverse(const uint64_t* fp, const int32_t* tokens, int64
                                                              err);
   scan_kernel<IsRep, OpSum, true><<<(unsigned)scan_tiles, kScanThreads, 0, stream>>>(
       IsRep{rep}, n, uid, scan1, ctr + 9, n_unique_dev, err);
-  finalize_kernel<<<grid_for(n, 256, sms * 8), 256, 0, stream>>>(rep, uid, n, unique_idx,
-                                                                 inverse);
+  finalize_kernel<<<grid_for(n, 256, sms * 8), 256, 0, stream>>>(rep, uid, n, n_unique_dev,
+                                                                 unique_idx, inverse);
   count_launches(10);  // hist, 4 radix passes, 2 scans, verify, resolve, finalize
   return cuda_fail(cudaGetLastError(), "unique_inverse launch");
 }

@@ -4,10 +4,12 @@ Composition of the C-ABI calls only (no arithmetic here):
   chunks:  hs_fingerprint -> hs_unique_inverse      (merge duplicate chunk nodes)
   queries: hs_fingerprint -> hs_unique_inverse      (merge duplicate query nodes,
            -> hs_scatter_results (gather unique)     Section 3.3 (I))
-           -> hs_retrieve_topk                      (one retrieval per merged node)
+           -> hs_retrieve_topk_n                    (one retrieval per merged node)
            -> hs_scatter_results (fan results back to every originating query)
-The single host synchronisation is the read of the unique-query count, which
-sizes the retrieval launch.
+Nothing here synchronises with the host: the merged-query count stays in
+device memory (hs_retrieve_topk_n reads it when its kernels run), and the
+unique-index tail beyond that count is a valid row map, so the gather can
+always cover the whole batch.  Buffers are allocated once per stage.
 """
 from __future__ import annotations
 
@@ -17,7 +19,7 @@ from . import _lib
 
 
 class EmbedRetrieveStage:
-    """Holds the resident corpus and reusable workspaces for repeated batches."""
+    """Holds the resident corpus and reusable buffers for repeated batches."""
 
     def __init__(self, corpus: torch.Tensor, k: int, max_queries: int,
                  max_chunk_rows: int = 0):
@@ -29,46 +31,50 @@ class EmbedRetrieveStage:
         dev = corpus.device
         self.device = dev
         self.max_queries = int(max_queries)
-        self.ws_q = torch.empty(_lib.hs_unique_inverse_workspace(max_queries), dtype=torch.uint8,
-                                device=dev)
-        self.ws_r = torch.empty(_lib.hs_retrieve_topk_workspace(max_queries, self.N, self.d, k),
+        mq, mc = self.max_queries, max(int(max_chunk_rows), 1)
+        i32 = dict(dtype=torch.int32, device=dev)
+        self.ws_q = torch.empty(_lib.hs_unique_inverse_workspace(mq), dtype=torch.uint8, device=dev)
+        self.ws_r = torch.empty(_lib.hs_retrieve_topk_workspace(mq, self.N, self.d, k),
                                 dtype=torch.uint8, device=dev)
-        self.ws_c = torch.empty(_lib.hs_unique_inverse_workspace(max(max_chunk_rows, 1)),
-                                dtype=torch.uint8, device=dev)
-        self.q_out = (torch.empty(1, dtype=torch.int32, device=dev),
-                      torch.empty(max_queries, dtype=torch.int32, device=dev),
-                      torch.empty(max_queries, dtype=torch.int32, device=dev))
-        self.c_out = (torch.empty(1, dtype=torch.int32, device=dev),
-                      torch.empty(max(max_chunk_rows, 1), dtype=torch.int32, device=dev),
-                      torch.empty(max(max_chunk_rows, 1), dtype=torch.int32, device=dev))
-        self.launches = 0
+        self.ws_c = torch.empty(_lib.hs_unique_inverse_workspace(mc), dtype=torch.uint8, device=dev)
+        self.q_out = (torch.empty(1, **i32), torch.empty(mq, **i32), torch.empty(mq, **i32))
+        self.c_out = (torch.empty(1, **i32), torch.empty(mc, **i32), torch.empty(mc, **i32))
+        self.q_fp = torch.empty(mq, dtype=torch.int64, device=dev)
+        self.c_fp = torch.empty(mc, dtype=torch.int64, device=dev)
+        self.uq = torch.empty((mq, self.d), dtype=corpus.dtype, device=dev)
+        self.s_u = torch.empty((mq, self.k), dtype=torch.float32, device=dev)
+        self.i_u = torch.empty((mq, self.k), **i32)
+        self.scores = torch.empty((mq, self.k), dtype=torch.float32, device=dev)
+        self.ids = torch.empty((mq, self.k), **i32)
 
     def dedup_chunks(self, tokens: torch.Tensor, lens: torch.Tensor | None = None):
         """Fingerprint + exact unique of chunk rows.  Returns (n_unique_dev,
-        unique_idx, inverse, fp)."""
-        fp = _lib.hs_fingerprint(tokens, lens)
+        unique_idx, inverse, fp) as device tensors."""
+        n = tokens.shape[0]
+        fp = _lib.hs_fingerprint(tokens, lens, fp_out=self.c_fp[:n])
         nu, uidx, inv = _lib.hs_unique_inverse(fp, tokens, lens, workspace=self.ws_c,
                                                out=self.c_out)
         return nu, uidx, inv, fp
 
     def retrieve(self, queries: torch.Tensor, events: tuple | None = None):
         """Merged retrieval of a query batch.  Returns (scores [Q, k],
-        ids [Q, k], n_unique) for every original query.  If ``events`` is a
-        pair of CUDA events they are recorded on the current stream around
-        the hs_retrieve_topk launch (kernel timing for the roofline)."""
+        ids [Q, k], n_unique_dev) for every original query; n_unique_dev is
+        a one-element device tensor.  If ``events`` is a pair of CUDA events
+        they are recorded on the current stream around the retrieval launch
+        (kernel timing for the roofline)."""
         Q, d = queries.shape
         if Q > self.max_queries:
             raise ValueError("batch larger than max_queries")
         qi32 = queries.view(torch.int32)
-        fp = _lib.hs_fingerprint(qi32)
+        fp = _lib.hs_fingerprint(qi32, fp_out=self.q_fp[:Q])
         nu, uidx, inv = _lib.hs_unique_inverse(fp, qi32, workspace=self.ws_q, out=self.q_out)
-        n_unique = int(nu.item())                     # the one host synchronisation
-        uq = _lib.hs_scatter_results(queries, uidx[:n_unique])
+        uq = _lib.hs_scatter_results(queries, uidx, dst=self.uq[:Q])
         if events is not None:
             events[0].record()
-        s_u, i_u = _lib.hs_retrieve_topk(uq, self.corpus, self.k, workspace=self.ws_r)
+        s_u, i_u = _lib.hs_retrieve_topk_n(uq, nu, self.corpus, self.k, workspace=self.ws_r,
+                                           out=(self.s_u[:Q], self.i_u[:Q]))
         if events is not None:
             events[1].record()
-        scores = _lib.hs_scatter_results(s_u, inv)
-        ids = _lib.hs_scatter_results(i_u, inv)
-        return scores, ids, n_unique
+        scores = _lib.hs_scatter_results(s_u, inv, dst=self.scores[:Q])
+        ids = _lib.hs_scatter_results(i_u, inv, dst=self.ids[:Q])
+        return scores, ids, nu

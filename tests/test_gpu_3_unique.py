@@ -131,3 +131,16 @@ def test_workspace_too_small_is_rejected():
     with pytest.raises(hs.HsError) as e:
         hs.hs_unique_inverse(f, t, workspace=ws)
     assert e.value.status == hs.HS_ERR_WORKSPACE
+
+
+def test_unique_idx_tail_is_a_valid_map():
+    w = configs.build_retrieval_mix(configs.TINY, corpus=False)
+    t = to_dev(w["tokens"])
+    f = hs.hs_fingerprint(t)
+    uidx = torch.full((t.shape[0],), 12345, dtype=torch.int32, device="cuda")
+    nu = torch.empty(1, dtype=torch.int32, device="cuda")
+    inv = torch.empty(t.shape[0], dtype=torch.int32, device="cuda")
+    hs.hs_unique_inverse(f, t, out=(nu, uidx, inv))
+    hs.hs_get_device_error()
+    n = int(nu.item())
+    assert n == 128 and (uidx[n:] == 0).all()

@@ -189,3 +189,32 @@ def test_deterministic():
     b = hs.hs_retrieve_topk(Qd, Cd, 10)
     hs.hs_get_device_error()
     assert torch.equal(a[0], b[0]) and torch.equal(a[1], b[1])
+
+
+def test_device_count_matches_host_count():
+    Q, C = unit_pair(300, 5000, 256, 9)
+    Qd, Cd = to_dev(Q), to_dev(C)
+    for k in (10, 20, 40):
+        ref_s, ref_i = hs.hs_retrieve_topk(Qd[:177], Cd, k)
+        cnt = torch.tensor([177], dtype=torch.int32, device="cuda")
+        s = torch.full((300, k), -7.0, device="cuda")
+        i = torch.full((300, k), -7, dtype=torch.int32, device="cuda")
+        hs.hs_retrieve_topk_n(Qd, cnt, Cd, k, out=(s, i))
+        hs.hs_get_device_error()
+        assert torch.equal(s[:177], ref_s) and torch.equal(i[:177], ref_i)
+        assert (s[177:] == -7.0).all() and (i[177:] == -7).all()   # rows past the count untouched
+
+
+def test_device_count_zero_and_clamped():
+    Q, C = unit_pair(64, 3000, 128, 10)
+    Qd, Cd = to_dev(Q), to_dev(C)
+    s = torch.full((64, 5), 3.0, device="cuda")
+    i = torch.full((64, 5), 3, dtype=torch.int32, device="cuda")
+    hs.hs_retrieve_topk_n(Qd, torch.zeros(1, dtype=torch.int32, device="cuda"), Cd, 5, out=(s, i))
+    hs.hs_get_device_error()
+    assert (s == 3.0).all() and (i == 3).all()
+    big = torch.tensor([1 << 30], dtype=torch.int32, device="cuda")
+    s2, i2 = hs.hs_retrieve_topk_n(Qd, big, Cd, 5)
+    ref_s, ref_i = hs.hs_retrieve_topk(Qd, Cd, 5)
+    hs.hs_get_device_error()
+    assert torch.equal(s2, ref_s) and torch.equal(i2, ref_i)

@@ -26,8 +26,9 @@ def test_stage_matches_oracle(cfg):
     assert (fp.cpu().numpy().view(np.uint64) == oracle.fingerprint(w["tokens"])).all()
 
     Q = w["queries"]
-    scores, ids, n_unique = stage.retrieve(to_dev(Q))
+    scores, ids, nu_dev = stage.retrieve(to_dev(Q))
     hs.hs_get_device_error()
+    n_unique = int(nu_dev.item())
     quidx, qinv = oracle.unique_inverse(Q.view(np.int32))
     assert n_unique == len(quidx)
     s, i = scores.cpu().numpy(), ids.cpu().numpy()
