@@ -264,8 +264,7 @@ def gpu_arm(args, rank: int, local_rank: int, world: int) -> int:
     stage = hs.EmbedRetrieveStage(corpus, k, max_queries=n_q, max_chunk_rows=n_chunk)
 
     def step(ev=None):
-        stage.dedup_chunks(tokens)
-        return stage.retrieve(queries, ev)
+        return stage.step(tokens, queries, events=ev)[1]
 
     for _ in range(args.warmup):
         _, _, nu_dev = step()
@@ -311,8 +310,7 @@ def gpu_arm(args, rank: int, local_rank: int, world: int) -> int:
     def e2e_step():
         d_tok.copy_(h_tokens, non_blocking=True)
         d_q.view(torch.int16).copy_(h_queries, non_blocking=True)
-        stage.dedup_chunks(d_tok)
-        s, i, _ = stage.retrieve(d_q)
+        _, (s, i, _) = stage.step(d_tok, d_q)
         h_s.copy_(s, non_blocking=True)
         h_i.copy_(i, non_blocking=True)
         torch.cuda.current_stream().synchronize()   # the results are read on the host

@@ -30,6 +30,8 @@
 // lists of each query with a bitonic sort of packed (score, index) keys.
 #include <float.h>
 
+#include <algorithm>
+
 #include "hs_internal.cuh"
 
 namespace hs {
@@ -58,7 +60,9 @@ constexpr size_t kSmem = 1024 + (size_t)kStages * kStageBytes + kBarBytes + kEpi
 struct Params {
   int64_t Qmax, N, tiles;
   const int32_t* count_dev;  // queries to process: min(*count_dev, Qmax); NULL: Qmax
-  int32_t k, kb_count, sms;
+  int32_t k, kb_count;
+  int32_t slots;             // concurrent unit executors the plan targets (CTAs / cl)
+  int32_t cl;                // CTAs per cluster: 1, or 2 sharing corpus tiles by multicast
   float* part_s;     // [Q][2 * nsplit][k]: one list per (split, column half)
   int32_t* part_i;
   float* list_s;     // large-k: [grid][kEpi][2][k]
@@ -84,18 +88,21 @@ __host__ __device__ inline int64_t max_splits(int64_t sms, int64_t tiles, int32_
   return ns < 1 ? 1 : ns;
 }
 
-// Work decomposition for Q queries: query blocks of 128 and corpus splits;
-// units = qblocks * nsplit is a multiple of the SM count when the caps allow.
-// Host and device evaluate the same function, so a launch can take its query
-// count from device memory.
+// Work decomposition for Q queries: query blocks of 128, grouped by cl (the
+// CTAs of a cluster take adjacent query blocks over the same corpus tiles),
+// and corpus splits; units = groups * nsplit is a multiple of the number of
+// unit executors (slots) when the caps allow.  Host and device evaluate the
+// same function, so a launch can take its query count from device memory.
 struct SplitPlan {
-  int32_t qblocks, nsplit;
+  int32_t qblocks, groups, nsplit;
 };
-__host__ __device__ inline SplitPlan split_plan(int64_t Q, int64_t tiles, int32_t k, int64_t sms) {
+__host__ __device__ inline SplitPlan split_plan(int64_t Q, int64_t tiles, int32_t k,
+                                                int64_t slots, int32_t cl) {
   SplitPlan sp;
   sp.qblocks = (int32_t)((Q + BM - 1) / BM);
-  int64_t ns = sms / gcd64(sms, sp.qblocks > 0 ? sp.qblocks : 1);
-  const int64_t cap = max_splits(sms, tiles, k);
+  sp.groups = (sp.qblocks + cl - 1) / cl;
+  int64_t ns = slots / gcd64(slots, sp.groups > 0 ? sp.groups : 1);
+  const int64_t cap = max_splits(slots, tiles, k);
   if (ns > cap) ns = cap;
   sp.nsplit = (int32_t)ns;
   return sp;
@@ -107,10 +114,11 @@ __device__ __forceinline__ int64_t query_count(const Params& p) {
   return c < 0 ? 0 : (c > p.Qmax ? p.Qmax : c);
 }
 
-__device__ __forceinline__ void unit_coords(const SplitPlan& sp, int64_t tiles, int64_t u, int& qb,
-                                            int& split, int64_t& t0, int64_t& t1) {
-  qb = (int)(u % sp.qblocks);
-  split = (int)(u / sp.qblocks);
+__device__ __forceinline__ void unit_coords(const SplitPlan& sp, int64_t tiles, int64_t u,
+                                            int rank, int cl, int& qb, int& split, int64_t& t0,
+                                            int64_t& t1) {
+  qb = (int)(u % sp.groups) * cl + rank;
+  split = (int)(u / sp.groups);
   t0 = (int64_t)split * tiles / sp.nsplit;
   t1 = (int64_t)(split + 1) * tiles / sp.nsplit;
 }
@@ -217,7 +225,7 @@ __device__ void flush_candidates(float* cs, int32_t* ci, int et, int& cnt, float
   cnt = 0;
 }
 
-template <int KREG>
+template <int KREG, int CL>
 __global__ void __launch_bounds__(kThreads, 1)
     retrieve_kernel(const __grid_constant__ CUtensorMap tmap_q,
                     const __grid_constant__ CUtensorMap tmap_c, const Params p) {
@@ -239,7 +247,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(full + s, 1);
-      mbar_init(empty + s, 1);
+      mbar_init(empty + s, CL);          // one commit from each CTA that fills the stage
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(tfull + a, 1);
@@ -259,10 +267,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  if (CL > 1) cluster_sync();            // peers' barriers exist before any multicast
   const uint32_t tmem_base = *tmem_slot;
+  const int rank = CL > 1 ? (int)cluster_ctarank() : 0;
   const int64_t Q = query_count(p);
-  const SplitPlan sp = split_plan(Q, p.tiles, p.k, p.sms);
-  const int64_t units = Q > 0 ? (int64_t)sp.qblocks * sp.nsplit : 0;
+  const SplitPlan sp = split_plan(Q, p.tiles, p.k, p.slots, CL);
+  const int64_t units = Q > 0 ? (int64_t)sp.groups * sp.nsplit : 0;
+  const int64_t u0 = blockIdx.x / CL, ustep = gridDim.x / CL;
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
@@ -270,17 +281,30 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint64_t pol_c = policy_evict_first();
       const uint64_t pol_q = policy_evict_last();
       uint32_t stage = 0, phase = 0;
-      for (int64_t u = blockIdx.x; u < units; u += gridDim.x) {
+      for (int64_t u = u0; u < units; u += ustep) {
         int qb, split;
         int64_t t0, t1;
-        unit_coords(sp, p.tiles, u, qb, split, t0, t1);
+        unit_coords(sp, p.tiles, u, rank, CL, qb, split, t0, t1);
         for (int64_t t = t0; t < t1; ++t) {
           for (int kb = 0; kb < p.kb_count; ++kb) {
             if (!mbar_wait(empty + stage, phase ^ 1u, abort_flag)) goto producer_done;
             mbar_arrive_expect_tx(full + stage, kStageBytes);
-            tma_load_2d_hint(sA + stage * kABytes, &tmap_q, full + stage, kb * BK, qb * BM, pol_q);
-            tma_load_2d_hint(sB + stage * kBBytes, &tmap_c, full + stage, kb * BK,
-                             (int32_t)(t * BN), pol_c);
+            // A query block past the last addressable row is loaded from
+            // row 0 instead: its scores are masked, and no box lies wholly
+            // outside the tensor.
+            const int32_t qy = (int64_t)qb * BM < p.Qmax ? qb * BM : 0;
+            tma_load_2d_hint(sA + stage * kABytes, &tmap_q, full + stage, kb * BK, qy, pol_q);
+            if (CL == 1) {
+              tma_load_2d_hint(sB + stage * kBBytes, &tmap_c, full + stage, kb * BK,
+                               (int32_t)(t * BN), pol_c);
+            } else {
+              // This CTA loads its half of the corpus tile into both CTAs.
+              // A half past the last row re-reads the first half (masked).
+              const int64_t cy = t * BN + rank * (BN / CL);
+              tma_load_2d_mc_hint(sB + stage * kBBytes + rank * (kBBytes / CL), &tmap_c,
+                                  full + stage, kb * BK, (int32_t)(cy < p.N ? cy : t * BN),
+                                  (uint16_t)((1u << CL) - 1u), pol_c);
+            }
             if (++stage == kStages) {
               stage = 0;
               phase ^= 1u;
@@ -295,10 +319,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_bf16_f32(BM, BN);
       uint32_t stage = 0, phase = 0, tile_i = 0;
-      for (int64_t u = blockIdx.x; u < units; u += gridDim.x) {
+      for (int64_t u = u0; u < units; u += ustep) {
         int qb, split;
         int64_t t0, t1;
-        unit_coords(sp, p.tiles, u, qb, split, t0, t1);
+        unit_coords(sp, p.tiles, u, rank, CL, qb, split, t0, t1);
         for (int64_t t = t0; t < t1; ++t, ++tile_i) {
           const uint32_t acc = tile_i & 1u, aphase = (tile_i >> 1) & 1u;
           if (!mbar_wait(tempty + acc, aphase ^ 1u, abort_flag)) goto mma_done;
@@ -313,7 +337,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int kk = 0; kk < BK / UK; ++kk)
               umma_bf16(d_tmem, a0 + (uint64_t)(kk * UK * 2 / 16), b0 + (uint64_t)(kk * UK * 2 / 16),
                         idesc, (kb | kk) != 0 ? 1u : 0u);
-            umma_commit(empty + stage);
+            if (CL == 1)
+              umma_commit(empty + stage);
+            else
+              umma_commit_mc(empty + stage, (uint16_t)((1u << CL) - 1u));
             if (++stage == kStages) {
               stage = 0;
               phase ^= 1u;
@@ -340,10 +367,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     int32_t* cand_i = reinterpret_cast<int32_t*>(epi_smem + (size_t)kCap * kEpi * 4);
     float* Ls = p.list_s + ((size_t)blockIdx.x * kEpi + et) * 2 * (size_t)k;
     int32_t* Li = p.list_i + ((size_t)blockIdx.x * kEpi + et) * 2 * (size_t)k;
-    for (int64_t u = blockIdx.x; u < units; u += gridDim.x) {
+    for (int64_t u = u0; u < units; u += ustep) {
       int qb, split;
       int64_t t0, t1;
-      unit_coords(sp, p.tiles, u, qb, split, t0, t1);
+      unit_coords(sp, p.tiles, u, rank, CL, qb, split, t0, t1);
       const int64_t q = (int64_t)qb * BM + row;
       const bool valid_q = q < Q;
       float theta = -FLT_MAX;
@@ -460,6 +487,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     tmem_dealloc(tmem_base, kTmemCols);
   }
+  if (CL > 1) cluster_sync();            // no CTA leaves while its peer may still signal it
   if (threadIdx.x == 0 && *abort_flag) set_error(p.err, kErrTimeout);
 }
 
@@ -481,7 +509,7 @@ __global__ void __launch_bounds__(256) merge_kernel(const Params p, float* __res
                                                     int32_t* __restrict__ out_i) {
   extern __shared__ uint64_t keys[];
   const int64_t Q = query_count(p);
-  const SplitPlan sp = split_plan(Q, p.tiles, p.k, p.sms);
+  const SplitPlan sp = split_plan(Q, p.tiles, p.k, p.slots, p.cl);
   const int k = p.k;
   const int lists = 2 * sp.nsplit;
   const int m = lists * k;
@@ -559,18 +587,97 @@ int p2_for(int64_t nsplit, int32_t k) {
   return p2;
 }
 
-template <int KREG>
-hs_status launch_kernel(const CUtensorMap& mq, const CUtensorMap& mc, const Params& prm,
-                        int64_t grid, cudaStream_t stream) {
+template <int KREG, int CL>
+hs_status configure_kernel() {
   static bool configured = false;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(retrieve_kernel<KREG>,
+    cudaError_t e = cudaFuncSetAttribute(retrieve_kernel<KREG, CL>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmem);
     if (e != cudaSuccess) return cuda_fail(e, "retrieve smem attribute");
     configured = true;
   }
-  retrieve_kernel<KREG><<<(unsigned)grid, kThreads, kSmem, stream>>>(mq, mc, prm);
-  return cuda_fail(cudaGetLastError(), "retrieve launch");
+  return HS_OK;
+}
+
+// Clusters of two that can be resident at once (one CTA per SM; pairs must
+// share a GPC), cached per kernel variant.
+template <int KREG>
+int64_t max_pairs() {
+  static int64_t cached = -1;
+  if (cached < 0) {
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.gridDim = dim3((unsigned)(num_sms() & ~1), 1, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = kSmem;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, retrieve_kernel<KREG, 2>, &cfg) != cudaSuccess) n = 0;
+    cached = n;
+  }
+  return cached;
+}
+
+template <int KREG, int CL>
+hs_status launch_kernel(const CUtensorMap& mq, const CUtensorMap& mc, const Params& prm,
+                        int64_t grid, cudaStream_t stream) {
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = CL;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.gridDim = dim3((unsigned)grid, 1, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = kSmem;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = CL > 1 ? 1 : 0;
+  return cuda_fail(cudaLaunchKernelEx(&cfg, retrieve_kernel<KREG, CL>, mq, mc, prm),
+                   "retrieve launch");
+}
+
+// Plan and launch for one register-list size.  Clusters of two when there
+// are at least two query blocks (they share corpus tiles), else single CTAs.
+template <int KREG>
+hs_status launch_variant(const uint16_t* corpus, int64_t N, int32_t d, const CUtensorMap& mq,
+                         Params& prm, cudaStream_t stream) {
+  const int64_t sms = num_sms();
+  const int64_t qblocks_max = (prm.Qmax + BM - 1) / BM;
+  hs_status st = configure_kernel<KREG, 1>();
+  if (st != HS_OK) return st;
+  int cl = 1;
+  int64_t slots = sms;
+  if (qblocks_max >= 2) {
+    st = configure_kernel<KREG, 2>();
+    if (st != HS_OK) return st;
+    const int64_t pairs = std::min<int64_t>(max_pairs<KREG>(), sms / 2);
+    if (pairs >= 1) {
+      cl = 2;
+      slots = pairs;
+    }
+  }
+  CUtensorMap mc;
+  if (!make_map(&mc, corpus, N, d, BN / cl))
+    return fail(HS_ERR_CUDA, "cuTensorMapEncodeTiled failed (driver entry point or arguments)");
+  prm.slots = (int32_t)slots;
+  prm.cl = cl;
+  // With a host-known count the grid covers only the plan's units; with a
+  // device count every slot gets a CTA (or pair) and idle ones exit.
+  int64_t execs = slots;
+  if (!prm.count_dev) {
+    const SplitPlan sp = split_plan(prm.Qmax, prm.tiles, prm.k, slots, cl);
+    const int64_t units = (int64_t)sp.groups * sp.nsplit;
+    if (units < execs) execs = units;
+  }
+  if (execs < 1) execs = 1;
+  return cl == 2 ? launch_kernel<KREG, 2>(mq, mc, prm, execs * 2, stream)
+                 : launch_kernel<KREG, 1>(mq, mc, prm, execs, stream);
 }
 
 }  // namespace
@@ -602,8 +709,8 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
   const size_t need = retrieve_topk_workspace(Qmax, N, d, k);
   if (ws_bytes < need)
     return fail(HS_ERR_WORKSPACE, "retrieve workspace too small: %zu < %zu", ws_bytes, need);
-  CUtensorMap mq, mc;
-  if (!make_map(&mq, queries, Qmax, d, BM) || !make_map(&mc, corpus, N, d, BN))
+  CUtensorMap mq;
+  if (!make_map(&mq, queries, Qmax, d, BM))
     return fail(HS_ERR_CUDA, "cuTensorMapEncodeTiled failed (driver entry point or arguments)");
   const int64_t ns_max = max_splits(sms, tiles, k);
   const size_t part = (((size_t)Qmax * 2 * ns_max * k * 4) + 255) & ~(size_t)255;
@@ -616,27 +723,18 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
   prm.count_dev = count_dev;
   prm.k = k;
   prm.kb_count = (d + BK - 1) / BK;
-  prm.sms = (int32_t)sms;
   prm.part_s = reinterpret_cast<float*>(w);
   prm.part_i = reinterpret_cast<int32_t*>(w + part);
   prm.list_s = reinterpret_cast<float*>(w + 2 * part);
   prm.list_i = reinterpret_cast<int32_t*>(w + 2 * part + list);
   prm.err = err;
-  // With a host-known count the grid is the plan's unit count (capped at the
-  // SM count); with a device count every SM gets a CTA and idle ones exit.
-  int64_t grid = sms;
-  if (!count_dev) {
-    const SplitPlan sp = split_plan(Qmax, tiles, k, sms);
-    const int64_t units = (int64_t)sp.qblocks * sp.nsplit;
-    if (units < grid) grid = units;
-  }
   hs_status st;
   if (k <= 16)
-    st = launch_kernel<16>(mq, mc, prm, grid, stream);
+    st = launch_variant<16>(corpus, N, d, mq, prm, stream);
   else if (k <= 32)
-    st = launch_kernel<32>(mq, mc, prm, grid, stream);
+    st = launch_variant<32>(corpus, N, d, mq, prm, stream);
   else
-    st = launch_kernel<0>(mq, mc, prm, grid, stream);
+    st = launch_variant<0>(corpus, N, d, mq, prm, stream);
   if (st != HS_OK) return st;
   const size_t msmem = (size_t)p2_for(ns_max, k) * 8;
   static size_t merge_configured = 0;

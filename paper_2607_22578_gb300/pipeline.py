@@ -78,3 +78,36 @@ class EmbedRetrieveStage:
         scores = _lib.hs_scatter_results(s_u, inv, dst=self.scores[:Q])
         ids = _lib.hs_scatter_results(i_u, inv, dst=self.ids[:Q])
         return scores, ids, nu
+
+    def step(self, tokens: torch.Tensor, queries: torch.Tensor,
+             lens: torch.Tensor | None = None, events: tuple | None = None):
+        """One batch of the whole stage.  The chunk merge and the query path
+        are independent, so the chunk fingerprint + unique run on a side
+        stream concurrently with the query fingerprint + unique, joined by an
+        event before the retrieval.  Returns (chunk (n_unique_dev,
+        unique_idx, inverse, fp), query (scores, ids, n_unique_dev))."""
+        main = torch.cuda.current_stream(self.device)
+        if not hasattr(self, "_side"):
+            self._side = torch.cuda.Stream(device=self.device)
+            self._fork = torch.cuda.Event()
+            self._join = torch.cuda.Event()
+        self._fork.record(main)
+        self._side.wait_event(self._fork)
+        with torch.cuda.stream(self._side):
+            chunk = self.dedup_chunks(tokens, lens)
+        self._join.record(self._side)
+        Q = queries.shape[0]
+        qi32 = queries.view(torch.int32)
+        fp = _lib.hs_fingerprint(qi32, fp_out=self.q_fp[:Q])
+        nu, uidx, inv = _lib.hs_unique_inverse(fp, qi32, workspace=self.ws_q, out=self.q_out)
+        uq = _lib.hs_scatter_results(queries, uidx, dst=self.uq[:Q])
+        main.wait_event(self._join)      # retrieval occupies every SM: chunk work first
+        if events is not None:
+            events[0].record()
+        s_u, i_u = _lib.hs_retrieve_topk_n(uq, nu, self.corpus, self.k, workspace=self.ws_r,
+                                           out=(self.s_u[:Q], self.i_u[:Q]))
+        if events is not None:
+            events[1].record()
+        scores = _lib.hs_scatter_results(s_u, inv, dst=self.scores[:Q])
+        ids = _lib.hs_scatter_results(i_u, inv, dst=self.ids[:Q])
+        return chunk, (scores, ids, nu)

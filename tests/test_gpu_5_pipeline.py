@@ -42,3 +42,19 @@ def test_stage_matches_oracle(cfg):
                                i[sample].reshape(-1)).reshape(-1, k)
     for r, q in enumerate(sample):
         check_topk(s[q], i[q], os_[r], oi_[r], exact[r], w["corpus"].shape[0], k)
+
+
+def test_step_runs_both_paths_and_matches_separate_calls():
+    w = configs.build_retrieval_mix(configs.TINY)
+    stage = hs.EmbedRetrieveStage(to_dev(w["corpus"]), w["k"], max_queries=len(w["queries"]),
+                                  max_chunk_rows=w["tokens"].shape[0])
+    t, q = to_dev(w["tokens"]), to_dev(w["queries"])
+    (cnu, cuidx, cinv, cfp), (s, i, qnu) = stage.step(t, q)
+    hs.hs_get_device_error()
+    ou, oi = oracle.unique_inverse(w["tokens"])
+    n = int(cnu.item())
+    assert n == len(ou) and (cuidx[:n].cpu().numpy() == ou).all()
+    assert (cinv.cpu().numpy() == oi).all()
+    s2, i2, _ = stage.retrieve(q)
+    hs.hs_get_device_error()
+    assert (s.cpu() == s2.cpu()).all() and (i.cpu() == i2.cpu()).all()
