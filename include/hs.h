@@ -128,6 +128,36 @@ hs_status hs_unique_inverse(const uint64_t* fp, const int32_t* tokens, int64_t n
                             size_t workspace_bytes, hs_stream_t stream);
 
 /*
+ * hs_unique_inverse_noalloc — hs_unique_inverse for callers that cannot
+ * allocate device memory.  The paper has no counterpart: this is a
+ * convenience of this library.
+ *
+ * Some callers may not allocate at the point where they merge rows: code
+ * running while a CUDA graph is being captured, plugins or embedded runtimes
+ * that are given a fixed memory budget and no allocator, and latency-critical
+ * request paths where an allocator call is an unbounded stall.  This entry
+ * point takes no workspace: its scratch is a fixed array inside the
+ * library's device memory (about 2.5 MB, present on every GPU that loads the
+ * library until the process exits), so it calls no allocator at all.
+ *
+ * Same arguments, outputs and error behaviour as hs_unique_inverse, except:
+ *   - n_rows must not exceed 65536 (larger n_rows returns
+ *     HS_ERR_INVALID_ARG and enqueues nothing; use hs_unique_inverse);
+ *   - every call on a device shares the one scratch array, so calls whose
+ *     work overlaps on the GPU (different streams, or different host threads
+ *     without ordering) race and give wrong results; calls on one stream are
+ *     ordered and safe.  Each call clears whatever part of the scratch must
+ *     start at zero, so leftovers of an earlier call do not matter;
+ *   - the first call on each device looks up that device's copy of the
+ *     scratch array (a host-side set-up step, done with the device current);
+ *     make that first call before any stream capture begins.
+ */
+hs_status hs_unique_inverse_noalloc(const uint64_t* fp, const int32_t* tokens, int64_t n_rows,
+                                    int32_t row_stride, const int32_t* lens,
+                                    int32_t* n_unique_dev, int32_t* unique_idx_out,
+                                    int32_t* inverse_out, hs_stream_t stream);
+
+/*
  * hs_retrieve_topk — dense retrieval of the merged queries, fused top-k.
  *
  * Paper: Section 4.1, "Workloads": queries and documents are embedded and

@@ -64,6 +64,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
             lib.hs_unique_inverse_workspace.restype = sz
             lib.hs_unique_inverse.argtypes = [P, P, i64, i32, P, P, P, P, P, sz, P]
             lib.hs_unique_inverse.restype = st
+            lib.hs_unique_inverse_noalloc.argtypes = [P, P, i64, i32, P, P, P, P, P]
+            lib.hs_unique_inverse_noalloc.restype = st
             lib.hs_retrieve_topk_workspace.argtypes = [i64, i64, i32, i32]
             lib.hs_retrieve_topk_workspace.restype = sz
             lib.hs_retrieve_topk.argtypes = [P, i64, P, i64, i32, i32, P, P, P, sz, P]
@@ -153,6 +155,28 @@ def hs_unique_inverse(fp: torch.Tensor, tokens: torch.Tensor, lens: torch.Tensor
     _check(load().hs_unique_inverse(_ptr(fp), _ptr(tokens), n, stride, _ptr(lens), _ptr(nu),
                                     _ptr(uidx), _ptr(inv), _ptr(workspace), workspace.numel(),
                                     _stream(stream)))
+    return nu, uidx[:n], inv[:n]
+
+
+def hs_unique_inverse_noalloc(fp: torch.Tensor, tokens: torch.Tensor,
+                              lens: torch.Tensor | None = None, out: tuple | None = None,
+                              stream=None):
+    """hs_unique_inverse without a workspace, for callers that cannot
+    allocate device memory (at most 65536 rows; the scratch is a fixed array
+    inside the library).  Pass preallocated `out` = (n_unique_dev [1],
+    unique_idx [n], inverse [n]) int32 tensors to allocate nothing here
+    either."""
+    _cuda(fp, "fp")
+    _cuda(tokens, "tokens")
+    n, stride = tokens.shape
+    dev = tokens.device
+    if out is None:
+        out = (torch.empty(1, dtype=torch.int32, device=dev),
+               torch.empty(max(n, 1), dtype=torch.int32, device=dev),
+               torch.empty(max(n, 1), dtype=torch.int32, device=dev))
+    nu, uidx, inv = out
+    _check(load().hs_unique_inverse_noalloc(_ptr(fp), _ptr(tokens), n, stride, _ptr(lens),
+                                            _ptr(nu), _ptr(uidx), _ptr(inv), _stream(stream)))
     return nu, uidx[:n], inv[:n]
 
 

@@ -67,6 +67,8 @@ unsigned* device_error_word() {
   return g_err_addr[dev];
 }
 
+void clear_last_error() { clear_msg(); }
+
 void count_launches(unsigned n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
 
 int num_sms() {

@@ -271,5 +271,6 @@ hs_status fail(hs_status s, const char* fmt, ...);
 hs_status cuda_fail(cudaError_t e, const char* what);
 unsigned* device_error_word();  // device address of the current device's error word
 int num_sms();
+void clear_last_error();
 void count_launches(unsigned n);  // diagnostics: kernels launched by this library
 }  // namespace hs

@@ -23,6 +23,8 @@
 //   6. exclusive sum-scan of "row is its own representative" gives each
 //      group its ordinal in first-occurrence order; the final kernel writes
 //      unique_idx and inverse.
+#include <mutex>
+
 #include "hs_internal.cuh"
 
 namespace hs {
@@ -49,7 +51,7 @@ struct Layout {
   size_t keys0, keys1, vals0, vals1, seg_head, rep, uid, coll_list, total;
 };
 
-Layout layout(int64_t n) {
+constexpr Layout layout(int64_t n) {
   Layout L{};
   const int64_t sort_tiles = (n + kSortTile - 1) / kSortTile;
   const int64_t scan_tiles = (n + kScanTile - 1) / kScanTile;
@@ -633,3 +635,76 @@ hs_status launch_unique_inverse(const uint64_t* fp, const int32_t* tokens, int64
 }
 
 }  // namespace hs
+
+// ---- allocation-free entry point -------------------------------------------------------------
+// Some callers cannot allocate device memory at the moment they merge rows:
+// code that runs while a CUDA graph is being captured (an allocation there
+// would be recorded into, or break, the graph), plugins and embedded runtimes
+// that are handed a fixed memory budget and may not touch the allocator, and
+// latency-critical request paths where an allocator call (or a pool that has
+// to grow) is an unbounded stall.  hs_unique_inverse_noalloc serves them with
+// a scratch area that is part of the library's own module memory: a
+// file-scope device array sized for kNoAllocMaxRows rows (about 2.5 MB),
+// which every GPU that loads the library holds until the process exits.
+namespace hs {
+namespace {
+constexpr int64_t kNoAllocMaxRows = 65536;
+constexpr size_t kNoAllocBytes = layout(kNoAllocMaxRows).total;
+static __device__ __align__(256) unsigned char g_noalloc_ws[kNoAllocBytes];
+constexpr int kNoAllocDevices = 64;
+void* g_noalloc_addr[kNoAllocDevices] = {};
+std::mutex g_noalloc_mu;
+
+// Device address of this device's copy of the scratch array.  In host code
+// the array's name is only a host-side stand-in, so the address is looked up
+// once per device, with that device current, and cached.
+hs_status noalloc_scratch(void** out) {
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (dev < 0 || dev >= kNoAllocDevices) return fail(HS_ERR_UNSUPPORTED, "device index %d", dev);
+  std::lock_guard<std::mutex> lk(g_noalloc_mu);
+  if (!g_noalloc_addr[dev]) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_noalloc_ws);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(scratch)");
+    g_noalloc_addr[dev] = p;
+  }
+  *out = g_noalloc_addr[dev];
+  return HS_OK;
+}
+}  // namespace
+}  // namespace hs
+
+extern "C" hs_status hs_unique_inverse_noalloc(const uint64_t* fp, const int32_t* tokens,
+                                               int64_t n_rows, int32_t row_stride,
+                                               const int32_t* lens, int32_t* n_unique_dev,
+                                               int32_t* unique_idx_out, int32_t* inverse_out,
+                                               hs_stream_t stream) {
+  using namespace hs;
+  clear_last_error();
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (n_rows < 0 || n_rows > kNoAllocMaxRows)
+    return fail(HS_ERR_INVALID_ARG, "n_rows outside [0, %lld], the allocation-free limit",
+                (long long)kNoAllocMaxRows);
+  if (row_stride < 0) return fail(HS_ERR_INVALID_ARG, "row_stride < 0");
+  if (!n_unique_dev) return fail(HS_ERR_INVALID_ARG, "n_unique_dev is NULL");
+  if (reinterpret_cast<uintptr_t>(n_unique_dev) % 4)
+    return fail(HS_ERR_INVALID_ARG, "n_unique_dev misaligned");
+  if (n_rows == 0)
+    return cuda_fail(cudaMemsetAsync(n_unique_dev, 0, sizeof(int32_t), s), "n_unique clear");
+  if (!fp || !unique_idx_out || !inverse_out || (!tokens && row_stride > 0))
+    return fail(HS_ERR_INVALID_ARG, "NULL input or output pointer");
+  if (reinterpret_cast<uintptr_t>(fp) % 8 || reinterpret_cast<uintptr_t>(tokens) % 4 ||
+      (lens && reinterpret_cast<uintptr_t>(lens) % 4) ||
+      reinterpret_cast<uintptr_t>(unique_idx_out) % 4 ||
+      reinterpret_cast<uintptr_t>(inverse_out) % 4)
+    return fail(HS_ERR_INVALID_ARG, "misaligned pointer");
+  void* scratch = nullptr;
+  const hs_status st = noalloc_scratch(&scratch);
+  if (st != HS_OK) return st;
+  // launch_unique_inverse clears the parts of the scratch that must start at
+  // zero on every call, so what an earlier call left there does not matter.
+  return launch_unique_inverse(fp, tokens, n_rows, row_stride, lens, n_unique_dev,
+                               unique_idx_out, inverse_out, scratch, s);
+}
