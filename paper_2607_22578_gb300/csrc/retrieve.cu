@@ -68,6 +68,11 @@ struct Params {
   float* list_s;     // large-k: [grid][kEpi][2][k]
   int32_t* list_i;
   unsigned* err;
+  // Optional per-query score floor (large-k path): query q only keeps scores
+  // >= floor[q * floor_stride + floor_index].  A floor never exceeds the
+  // query's final k-th best score, so it prunes without changing the result.
+  const float* floor;
+  int32_t floor_stride, floor_index;
 };
 
 __host__ __device__ inline int64_t gcd64(int64_t a, int64_t b) {
@@ -143,7 +148,7 @@ __device__ __forceinline__ void list_insert(float (&ls)[KREG], int32_t (&li)[KRE
 
 // ---- large-k helpers (per thread, serial) ---------------------------------------------
 __device__ void flush_candidates(float* cs, int32_t* ci, int et, int& cnt, float* Ls, int32_t* Li,
-                                 int k, int& cur, float& theta) {
+                                 int k, int& cur, float& theta, float floor_theta) {
   if (cnt == 0) return;
   // Stable insertion sort of the buffer, score descending (buffer order is
   // ascending corpus index, so ties keep the lower index first).
@@ -221,7 +226,7 @@ __device__ void flush_candidates(float* cs, int32_t* ci, int et, int& cnt, float
     }
   }
   cur ^= 1;
-  theta = last;  // the k-th entry of the new list
+  theta = fmaxf(last, floor_theta);  // the k-th entry of the new list, not below the floor
   cnt = 0;
 }
 
@@ -373,7 +378,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       unit_coords(sp, p.tiles, u, rank, CL, qb, split, t0, t1);
       const int64_t q = (int64_t)qb * BM + row;
       const bool valid_q = q < Q;
-      float theta = -FLT_MAX;
+      // Large k: start from the query's floor (a lower bound on its final k-th
+      // best score), so only scores that can still make the top k are kept.
+      float floor_theta = -FLT_MAX;
+      if (KREG == 0 && p.floor && valid_q) {
+        const float f = p.floor[(size_t)q * p.floor_stride + p.floor_index];
+        if (f > -FLT_MAX) floor_theta = nextafterf(f, -INFINITY);  // keep s >= f
+      }
+      float theta = floor_theta;
       float ls[KREG > 0 ? KREG : 1];
       int32_t li[KREG > 0 ? KREG : 1];
       int cnt = 0, cur = 0;
@@ -449,7 +461,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
               }
               if (__any_sync(0xffffffffu, cnt > kCap - 4))
-                flush_candidates(cand_s, cand_i, et, cnt, Ls, Li, k, cur, theta);
+                flush_candidates(cand_s, cand_i, et, cnt, Ls, Li, k, cur, theta, floor_theta);
             }
           }
         }
@@ -469,7 +481,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               oi[i] = li[i];
             }
         } else {
-          flush_candidates(cand_s, cand_i, et, cnt, Ls, Li, k, cur, theta);
+          flush_candidates(cand_s, cand_i, et, cnt, Ls, Li, k, cur, theta, floor_theta);
           for (int i = 0; i < k; ++i) {
             os[i] = Ls[(size_t)cur * k + i];
             oi[i] = Li[(size_t)cur * k + i];
@@ -505,8 +517,9 @@ __device__ __forceinline__ void unpack_key(uint64_t key, float& s, int32_t& idx)
   idx = (int32_t)(0xffffffffu - (uint32_t)key);
 }
 
+// Lists of p.k entries per (query, split, half) -> the kout best per query.
 __global__ void __launch_bounds__(256) merge_kernel(const Params p, float* __restrict__ out_s,
-                                                    int32_t* __restrict__ out_i) {
+                                                    int32_t* __restrict__ out_i, int32_t kout) {
   extern __shared__ uint64_t keys[];
   const int64_t Q = query_count(p);
   const SplitPlan sp = split_plan(Q, p.tiles, p.k, p.slots, p.cl);
@@ -538,12 +551,12 @@ __global__ void __launch_bounds__(256) merge_kernel(const Params p, float* __res
         __syncthreads();
       }
     }
-    for (int j = threadIdx.x; j < k; j += blockDim.x) {
-      float s;
-      int32_t idx;
-      unpack_key(keys[j], s, idx);
-      out_s[(size_t)q * k + j] = s;
-      out_i[(size_t)q * k + j] = idx;
+    for (int j = threadIdx.x; j < kout; j += blockDim.x) {
+      float s = -FLT_MAX;
+      int32_t idx = -1;
+      if (j < m) unpack_key(keys[j], s, idx);
+      out_s[(size_t)q * kout + j] = s;
+      out_i[(size_t)q * kout + j] = idx;
     }
     __syncthreads();
   }
@@ -728,26 +741,55 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
   prm.list_s = reinterpret_cast<float*>(w + 2 * part);
   prm.list_i = reinterpret_cast<int32_t*>(w + 2 * part + list);
   prm.err = err;
-  hs_status st;
-  if (k <= 16)
-    st = launch_variant<16>(corpus, N, d, mq, prm, stream);
-  else if (k <= 32)
-    st = launch_variant<32>(corpus, N, d, mq, prm, stream);
-  else
-    st = launch_variant<0>(corpus, N, d, mq, prm, stream);
-  if (st != HS_OK) return st;
-  const size_t msmem = (size_t)p2_for(ns_max, k) * 8;
-  static size_t merge_configured = 0;
-  if (msmem > 48 * 1024 && msmem > merge_configured) {
-    cudaError_t e = cudaFuncSetAttribute(merge_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)msmem);
-    if (e != cudaSuccess) return cuda_fail(e, "merge smem attribute");
-    merge_configured = msmem;
-  }
   const int64_t mgrid = Qmax < sms * 8 ? Qmax : sms * 8;
-  merge_kernel<<<(unsigned)mgrid, 256, msmem, stream>>>(prm, scores_out, ids_out);
+  auto merge = [&](const Params& pm, int32_t kout) -> hs_status {
+    const size_t msmem = (size_t)p2_for(max_splits(sms, pm.tiles, pm.k), pm.k) * 8;
+    static size_t merge_configured = 0;
+    if (msmem > 48 * 1024 && msmem > merge_configured) {
+      cudaError_t e = cudaFuncSetAttribute(merge_kernel,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize, (int)msmem);
+      if (e != cudaSuccess) return cuda_fail(e, "merge smem attribute");
+      merge_configured = msmem;
+    }
+    merge_kernel<<<(unsigned)mgrid, 256, msmem, stream>>>(pm, scores_out, ids_out, kout);
+    return cuda_fail(cudaGetLastError(), "merge launch");
+  };
+  hs_status st;
+  if (k <= 16) {
+    st = launch_variant<16>(corpus, N, d, mq, prm, stream);
+  } else if (k <= 32) {
+    st = launch_variant<32>(corpus, N, d, mq, prm, stream);
+  } else {
+    // Large k, two passes.  Pass 1 runs the register-list kernel (32 per
+    // list) over the first eighth of the corpus; the k-th best of the union
+    // of its lists is a score that k distinct corpus rows reach, hence at
+    // most the query's final k-th best: a floor.  Pass 2 runs the large-k
+    // kernel over the whole corpus keeping only scores >= the floor, which
+    // leaves few candidates per list.  Both passes' lists go through the
+    // same workspace; the floor is staged in scores_out and overwritten by
+    // the final merge.
+    if (tiles >= 64) {
+      Params p1 = prm;
+      p1.tiles = tiles / 8;
+      p1.N = p1.tiles * BN;
+      p1.k = 32;
+      p1.floor = nullptr;
+      st = launch_variant<32>(corpus, N, d, mq, p1, stream);
+      if (st != HS_OK) return st;
+      st = merge(p1, k);
+      if (st != HS_OK) return st;
+      count_launches(2);
+      prm.floor = scores_out;
+      prm.floor_stride = k;
+      prm.floor_index = k - 1;
+    }
+    st = launch_variant<0>(corpus, N, d, mq, prm, stream);
+  }
+  if (st != HS_OK) return st;
+  st = merge(prm, k);
+  if (st != HS_OK) return st;
   count_launches(2);  // retrieve_kernel + merge_kernel
-  return cuda_fail(cudaGetLastError(), "merge launch");
+  return HS_OK;
 }
 
 }  // namespace hs

@@ -218,3 +218,30 @@ def test_device_count_zero_and_clamped():
     ref_s, ref_i = hs.hs_retrieve_topk(Qd, Cd, 5)
     hs.hs_get_device_error()
     assert torch.equal(s2, ref_s) and torch.equal(i2, ref_i)
+
+
+def test_large_k_floor_with_ties_beyond_k():
+    # 60 exact copies of each query, some inside the first eighth of the
+    # corpus (the floor sample): the floor equals the copies' score, every
+    # copy ties with it, and the top 40 must be the 40 lowest-index copies.
+    nq, N, d, k = 6, 40000, 128, 40
+    Q, C = unit_pair(nq, N, d, 21)
+    rng = np.random.default_rng(3)
+    for q in range(nq):
+        pos = rng.choice(N, size=60, replace=False)
+        C[pos] = Q[q]
+    gs, gi = gpu_topk(to_dev(Q), to_dev(C), k)
+    parity(Q, C, k, gs, gi, range(nq))
+    os_, oi = oracle.topk(Q, C, k)
+    assert (gi == oi).all()
+
+
+def test_large_k_best_rows_outside_the_sample():
+    # The best rows of every query sit in the last part of the corpus, so the
+    # floor from the first eighth is far below the final k-th score.
+    nq, N, d, k = 5, 40000, 128, 64
+    Q, C = unit_pair(nq, N, d, 22)
+    for q in range(nq):
+        C[N - 200 - 30 * q: N - 30 * q] = Q[q]
+    gs, gi = gpu_topk(to_dev(Q), to_dev(C), k)
+    parity(Q, C, k, gs, gi, range(nq))
