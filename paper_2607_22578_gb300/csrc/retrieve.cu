@@ -449,19 +449,26 @@ __global__ void __launch_bounds__(kThreads, 1)
               __syncwarp();
             }
           } else {
+            // Same first test as above: a chunk whose maximum beats no
+            // lane's threshold costs one max-reduction and a vote.
+            float mx = __uint_as_float(r[0]);
 #pragma unroll
-            for (int j0 = 0; j0 < 32; j0 += 4) {
+            for (int j = 1; j < 32; ++j) mx = fmaxf(mx, __uint_as_float(r[j]));
+            if (__any_sync(0xffffffffu, mx > theta)) {
 #pragma unroll
-              for (int j = j0; j < j0 + 4; ++j) {
-                const float s = __uint_as_float(r[j]);
-                if (s > theta) {
-                  cand_s[cnt * kEpi + et] = s;
-                  cand_i[cnt * kEpi + et] = cbase + j;
-                  ++cnt;
+              for (int j0 = 0; j0 < 32; j0 += 4) {
+#pragma unroll
+                for (int j = j0; j < j0 + 4; ++j) {
+                  const float s = __uint_as_float(r[j]);
+                  if (s > theta) {
+                    cand_s[cnt * kEpi + et] = s;
+                    cand_i[cnt * kEpi + et] = cbase + j;
+                    ++cnt;
+                  }
                 }
+                if (__any_sync(0xffffffffu, cnt > kCap - 4))
+                  flush_candidates(cand_s, cand_i, et, cnt, Ls, Li, k, cur, theta, floor_theta);
               }
-              if (__any_sync(0xffffffffu, cnt > kCap - 4))
-                flush_candidates(cand_s, cand_i, et, cnt, Ls, Li, k, cur, theta, floor_theta);
             }
           }
         }
