@@ -239,6 +239,140 @@ __global__ void __launch_bounds__(kFpThreads) fingerprint_async_kernel(
   cp_async_wait<0>();
 }
 
+// ---- vector path, coalesced staging -----------------------------------------------
+// A warp owns 32 rows at a time, one per lane.  In each round it stages the
+// next chunk of up to 64 tokens of all 32 rows in shared memory: every copy
+// instruction moves two rows' contiguous 256-byte chunks (16 lanes per row),
+// so an instruction touches a handful of cache lines instead of 32 rows'
+// worth.  Each lane then hashes its own row's chunk from shared memory while
+// the next round's chunks are in flight (two buffers per warp).  A lane whose
+// row is exhausted claims the warp's next row for the following round.  Row
+// slots are 272 bytes (17 x 16 B) so the eight lanes of a quarter-warp read
+// different banks.
+constexpr int kChunk = 64;                       // tokens per row per round
+constexpr int kSlotBytes = kChunk * 4 + 16;      // 272 B
+constexpr int kRoundBytes = 32 * kSlotBytes;     // one buffer of one warp
+
+template <int WARPS>
+__global__ void __launch_bounds__(WARPS * 32) fingerprint_coal_kernel(
+    const int32_t* __restrict__ tokens, int64_t n, int32_t stride,
+    const int32_t* __restrict__ lens, uint64_t seed, uint64_t* __restrict__ fp_out,
+    int64_t rows_per_warp, unsigned* err) {
+  extern __shared__ uint8_t coal_smem[];
+  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t r_begin = warp * rows_per_warp;
+  if (r_begin >= n) return;
+  const int64_t r_end = min(n, r_begin + rows_per_warp);
+  const uint32_t lane = threadIdx.x & 31u;
+  uint8_t* wbuf = coal_smem + (threadIdx.x >> 5) * 2 * kRoundBytes;
+  const uint32_t wbuf_u32 = smem_u32(wbuf);
+  const uint32_t seed_lo = (uint32_t)seed, seed_hi = (uint32_t)(seed >> 32);
+
+  // Issue side: the next chunk of this lane's row to stage.
+  int64_t irow = -1;
+  int32_t ipos = 0, ilen = 0;
+  // Staged chunks per buffer: row (or -1), start position, tokens, row length.
+  int64_t prow[2] = {-1, -1};
+  int32_t ppos[2] = {0, 0}, pw[2] = {0, 0}, plen[2] = {0, 0};
+  uint32_t lo = seed_lo, hi = seed_hi;
+
+  int64_t next = r_begin;
+  int64_t wbase = r_begin;
+  auto len_of = [&](int64_t r) -> int32_t {
+    return r < r_end ? (lens ? __ldg(lens + r) : stride) : 0;
+  };
+  int32_t len_a = len_of(wbase + lane), len_b = len_of(wbase + 32 + lane);
+
+  // Claim rows for lanes whose issue side is free (lengths prefetched).
+  auto claim = [&]() {
+    unsigned need = __ballot_sync(0xffffffffu, irow < 0);
+    while (need != 0u && next < r_end) {
+      const int64_t avail = r_end - next;
+      const int rank = __popc(need & lanemask_lt());
+      const int off = (int)(next - wbase) + (irow < 0 ? rank : 0);
+      const int32_t La = __shfl_sync(0xffffffffu, len_a, off & 31);
+      const int32_t Lb = __shfl_sync(0xffffffffu, len_b, off & 31);
+      if (irow < 0 && rank < avail) {
+        const int64_t r = next + rank;
+        const int32_t L = off < 32 ? La : Lb;
+        if (L < 0 || L > stride) {
+          set_error(err, kErrInvalidArg);
+          fp_out[r] = 0ull;
+        } else if (L == 0) {
+          fp_out[r] = seed;
+        } else {
+          irow = r;
+          ipos = 0;
+          ilen = L;
+        }
+      }
+      next += min((int64_t)__popc(need), avail);
+      if (next - wbase >= 32) {
+        wbase += 32;
+        len_a = len_b;
+        len_b = len_of(wbase + 32 + lane);
+      }
+      need = __ballot_sync(0xffffffffu, irow < 0);
+    }
+  };
+
+  // Stage every lane's next chunk into buffer b, cooperatively.
+  auto issue = [&](int b) {
+    const int32_t w = irow >= 0 ? min(kChunk, ilen - ipos) : 0;
+    const int32_t pieces = (w + 3) >> 2;
+    const int32_t* src = tokens + (irow >= 0 ? irow * (int64_t)stride + ipos : 0);
+    prow[b] = irow;
+    ppos[b] = ipos;
+    pw[b] = w;
+    plen[b] = ilen;
+    if (irow >= 0) {
+      ipos += w;
+      if (ipos >= ilen) irow = -1;
+    }
+    const uint32_t dst0 = wbuf_u32 + b * kRoundBytes;
+    const uint32_t pc = lane & 15u;
+#pragma unroll 4
+    for (int i = 0; i < 16; ++i) {
+      const int j = 2 * i + (int)(lane >> 4);
+      const int32_t* sj = reinterpret_cast<const int32_t*>(
+          __shfl_sync(0xffffffffu, reinterpret_cast<uintptr_t>(src), j));
+      const int32_t pj = __shfl_sync(0xffffffffu, pieces, j);
+      if ((int32_t)pc < pj) cp_async16(dst0 + j * kSlotBytes + 16 * pc, sj + 4 * pc);
+    }
+    cp_async_commit();
+  };
+
+  // Hash this lane's staged chunk in buffer b.
+  auto hash = [&](int b) {
+    if (prow[b] < 0) return;
+    if (ppos[b] == 0) {
+      lo = seed_lo;
+      hi = seed_hi;
+    }
+    hash_block(lo, hi, reinterpret_cast<const int4*>(wbuf + b * kRoundBytes + lane * kSlotBytes),
+               pw[b]);
+    if (ppos[b] + pw[b] >= plen[b]) fp_out[prow[b]] = ((uint64_t)hi << 32) | lo;
+    prow[b] = -1;
+  };
+
+  claim();
+  issue(0);
+  for (;;) {
+#pragma unroll
+    for (int b = 0; b < 2; ++b) {
+      claim();
+      issue(b ^ 1);
+      cp_async_wait<1>();
+      __syncwarp();
+      hash(b);
+      __syncwarp();   // buffer b is reused by the next round's copies
+    }
+    const bool pending = irow >= 0 || prow[0] >= 0 || prow[1] >= 0;
+    if (!__any_sync(0xffffffffu, pending) && next >= r_end) break;
+  }
+  cp_async_wait<0>();
+}
+
 // ---- word path (tokens not 16-byte aligned, or row_stride % 4 != 0) -------------------
 __global__ void __launch_bounds__(256) fingerprint_words_kernel(
     const int32_t* __restrict__ tokens, int64_t n, int32_t stride,
@@ -321,19 +455,28 @@ hs_status launch_fingerprint(const int32_t* tokens, int64_t n, int32_t stride,
   if (!err) return fail(HS_ERR_CUDA, "could not resolve the device error word");
   const int64_t sms = num_sms();
   if (vec) {
-    const int64_t lanes_full = sms * 32 * 32;   // 32 warps per SM, one row per lane
+    // Coalesced staging: 4-warp blocks (68 KB of round buffers, three
+    // blocks per SM) once there are rows for 12 warps per SM, else one-warp
+    // blocks so the warps spread over all SMs.
+    const int64_t lanes_full = sms * 12 * 32;
     if (n >= lanes_full) {
-      // 128-thread blocks, eight per SM (26.6 KB rings each).
-      const int64_t warps_target = sms * 32;
+      const int64_t warps_target = sms * 12;
       const int64_t rpw = (n + warps_target - 1) / warps_target;
       const int64_t warps = (n + rpw - 1) / rpw;
       const int64_t blocks = (warps + 3) / 4;
-      fingerprint_async_kernel<3, 128><<<(unsigned)blocks, 128, 128 * lane_bytes<3>(), stream>>>(
+      const size_t smem = 4 * 2 * kRoundBytes;
+      static bool configured = false;
+      if (!configured) {
+        const cudaError_t e = cudaFuncSetAttribute(
+            fingerprint_coal_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return cuda_fail(e, "fingerprint smem attribute");
+        configured = true;
+      }
+      fingerprint_coal_kernel<4><<<(unsigned)blocks, 128, smem, stream>>>(
           tokens, n, stride, lens, seed, fp_out, rpw, err);
     } else {
-      // One row per lane, one-warp blocks with 8-slot rings (16.9 KB).
       const int64_t warps = (n + 31) / 32;
-      fingerprint_async_kernel<8, 32><<<(unsigned)warps, 32, 32 * lane_bytes<8>(), stream>>>(
+      fingerprint_coal_kernel<1><<<(unsigned)warps, 32, 2 * kRoundBytes, stream>>>(
           tokens, n, stride, lens, seed, fp_out, 32, err);
     }
   } else {
