@@ -25,16 +25,15 @@ constexpr uint32_t kP3Lo = (uint32_t)(kPrime3 & 0xffffffffull);
 constexpr uint32_t kP3Hi = (uint32_t)(kPrime3 >> 32);
 
 __device__ __forceinline__ void mul_prime(uint32_t& lo, uint32_t& hi) {
-  // (hi * 2^32 + lo) * (2^40 + 0x1b3) mod 2^64
-  const uint64_t t = (uint64_t)lo * 0x1b3u;
-  hi = (uint32_t)(t >> 32) + hi * 0x1b3u + (lo << 8);
-  lo = (uint32_t)t;
+  // (hi * 2^32 + lo) * (2^40 + 0x1b3) mod 2^64: the low word needs only lo,
+  // the high word adds hi * 0x1b3, the carry-out of lo * 0x1b3 and lo << 8.
+  hi = __umulhi(lo, 0x1b3u) + hi * 0x1b3u + (lo << 8);
+  lo = lo * 0x1b3u;
 }
 
 __device__ __forceinline__ void mul_prime3(uint32_t& lo, uint32_t& hi) {
-  const uint64_t t = (uint64_t)lo * kP3Lo;
-  hi = (uint32_t)(t >> 32) + lo * kP3Hi + hi * kP3Lo;
-  lo = (uint32_t)t;
+  hi = __umulhi(lo, kP3Lo) + lo * kP3Hi + hi * kP3Lo;
+  lo = lo * kP3Lo;
 }
 
 // Octet-wise rounds for one token, little-endian octet order; octets are
@@ -98,9 +97,9 @@ __device__ __forceinline__ uint32_t word_of(const int4& v, int j) {
   return (uint32_t)(j == 0 ? v.x : (j == 1 ? v.y : (j == 2 ? v.z : v.w)));
 }
 
-// Hash the first w (1..16) tokens of a block held in shared memory.  One
-// compact body: the four-token fast path when all four tokens are below 65536,
-// else token by token.
+// Hash the first w tokens of a block held in shared memory.  One compact
+// body: the four-token fast path when all four tokens are below 65536, else
+// token by token.
 __device__ __forceinline__ void hash_block(uint32_t& lo, uint32_t& hi, const int4* blk, int w) {
 #pragma unroll 1
   for (int pc = 0; 4 * pc < w; ++pc) {
@@ -349,8 +348,30 @@ __global__ void __launch_bounds__(WARPS * 32) fingerprint_coal_kernel(
       lo = seed_lo;
       hi = seed_hi;
     }
-    hash_block(lo, hi, reinterpret_cast<const int4*>(wbuf + b * kRoundBytes + lane * kSlotBytes),
-               pw[b]);
+    const int4* blk = reinterpret_cast<const int4*>(wbuf + b * kRoundBytes + lane * kSlotBytes);
+    bool done = false;
+    if (pw[b] == kChunk) {
+      // Whole chunk: check once that every token is below 65536, then run
+      // the two-round form straight through.
+      uint32_t any_big = 0;
+#pragma unroll 4
+      for (int pc = 0; pc < kChunk / 4; ++pc) {
+        const int4 v = blk[pc];
+        any_big |= (uint32_t)v.x | (uint32_t)v.y | (uint32_t)v.z | (uint32_t)v.w;
+      }
+      if ((any_big >> 16) == 0u) {
+#pragma unroll 4
+        for (int pc = 0; pc < kChunk / 4; ++pc) {
+          const int4 v = blk[pc];
+          hash_word_small(lo, hi, (uint32_t)v.x);
+          hash_word_small(lo, hi, (uint32_t)v.y);
+          hash_word_small(lo, hi, (uint32_t)v.z);
+          hash_word_small(lo, hi, (uint32_t)v.w);
+        }
+        done = true;
+      }
+    }
+    if (!done) hash_block(lo, hi, blk, pw[b]);
     if (ppos[b] + pw[b] >= plen[b]) fp_out[prow[b]] = ((uint64_t)hi << 32) | lo;
     prow[b] = -1;
   };
