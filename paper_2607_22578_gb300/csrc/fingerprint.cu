@@ -82,10 +82,15 @@ __device__ __forceinline__ void hash_word(uint32_t& lo, uint32_t& hi, uint32_t w
 // at the end of its row does not send the warp down a second path.  Slots
 // are 144 bytes (9 x 16 B) so the eight lanes of a quarter-warp hit
 // different banks.
-constexpr int kChunk = 32;                       // tokens per row per round
-constexpr int kSlotBytes = kChunk * 4 + 16;      // 144 B
-constexpr int kRoundBytes = 32 * kSlotBytes;     // one buffer of one warp
-constexpr int kWarpBytes = 2 * kRoundBytes + 64; // two buffers + two mbarriers + abort word
+// Per-warp shared memory for chunks of C tokens: two buffers of 32 slots
+// (C*4 + 16 bytes each, an odd multiple of 16 for C = 32 or 128), then two
+// mbarriers and an abort word.
+template <int C>
+constexpr int slot_bytes() { return C * 4 + 16; }
+template <int C>
+constexpr int round_bytes() { return 32 * slot_bytes<C>(); }
+template <int C>
+constexpr int warp_bytes() { return 2 * round_bytes<C>() + 64; }
 
 __device__ __forceinline__ void bulk_copy_g2s(uint32_t dst, const void* src, uint32_t bytes,
                                               uint32_t bar) {
@@ -96,16 +101,17 @@ __device__ __forceinline__ void bulk_copy_g2s(uint32_t dst, const void* src, uin
       : "memory");
 }
 
-// Hash tokens [0, w) of a chunk in shared memory (w <= kChunk).  Every lane
+// Hash tokens [0, w) of a chunk in shared memory (w <= C).  Every lane
 // walks the same pieces; words at or past w are masked out of the fast-path
 // test and skipped.
+template <int C>
 __device__ __forceinline__ void hash_chunk(uint32_t& lo, uint32_t& hi, const int4* blk, int w) {
 #pragma unroll 2
-  for (int pc = 0; pc < kChunk / 4; ++pc) {
+  for (int pc = 0; pc < C / 4; ++pc) {
     const int n = w - 4 * pc;                     // valid words in this piece (may be <= 0)
     if (__all_sync(0xffffffffu, n <= 0)) break;
     const int4 v = blk[pc];
-    const uint32_t x = (uint32_t)v.x;
+    const uint32_t x = n > 0 ? (uint32_t)v.x : 0u;
     const uint32_t y = n > 1 ? (uint32_t)v.y : 0u;
     const uint32_t z = n > 2 ? (uint32_t)v.z : 0u;
     const uint32_t q = n > 3 ? (uint32_t)v.w : 0u;
@@ -123,12 +129,15 @@ __device__ __forceinline__ void hash_chunk(uint32_t& lo, uint32_t& hi, const int
   }
 }
 
-template <int WARPS>
+template <int WARPS, int kChunk>
 __global__ void __launch_bounds__(WARPS * 32) fingerprint_tma_kernel(
     const int32_t* __restrict__ tokens, int64_t n, int32_t stride,
     const int32_t* __restrict__ lens, uint64_t seed, uint64_t* __restrict__ fp_out,
     int64_t rows_per_warp, unsigned* err) {
   extern __shared__ __align__(16) uint8_t tma_smem[];
+  constexpr int kSlotBytes = slot_bytes<kChunk>();
+  constexpr int kRoundBytes = round_bytes<kChunk>();
+  constexpr int kWarpBytes = warp_bytes<kChunk>();
   const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int64_t r_begin = warp * rows_per_warp;
   if (r_begin >= n) return;
@@ -219,8 +228,9 @@ __global__ void __launch_bounds__(WARPS * 32) fingerprint_tma_kernel(
       lo = seed_lo;
       hi = seed_hi;
     }
-    hash_chunk(lo, hi, reinterpret_cast<const int4*>(wbuf + b * kRoundBytes + lane * kSlotBytes),
-               prow[b] >= 0 ? pw[b] : 0);
+    hash_chunk<kChunk>(lo, hi,
+                       reinterpret_cast<const int4*>(wbuf + b * kRoundBytes + lane * kSlotBytes),
+                       prow[b] >= 0 ? pw[b] : 0);
     if (prow[b] >= 0 && ppos[b] + pw[b] >= plen[b]) fp_out[prow[b]] = ((uint64_t)hi << 32) | lo;
     prow[b] = -1;
     return true;
@@ -329,28 +339,29 @@ hs_status launch_fingerprint(const int32_t* tokens, int64_t n, int32_t stride,
   if (!err) return fail(HS_ERR_CUDA, "could not resolve the device error word");
   const int64_t sms = num_sms();
   if (vec) {
-    // Per-lane bulk copies: 8-warp blocks (73.7 KB of round buffers, three
-    // blocks = 24 warps per SM) once there are rows for all of them, else
-    // one-warp blocks so the warps spread over all SMs.
+    // Per-lane bulk copies: 8-warp blocks with 32-token chunks (74 KB of
+    // round buffers, three blocks = 24 warps per SM) once there are rows for
+    // all of them; else one-warp blocks with 128-token chunks, so the warps
+    // spread over all SMs and each lane has few, large rounds.
     const int64_t lanes_full = sms * 24 * 32;
     if (n >= lanes_full) {
       const int64_t warps_target = sms * 24;
       const int64_t rpw = (n + warps_target - 1) / warps_target;
       const int64_t warps = (n + rpw - 1) / rpw;
       const int64_t blocks = (warps + 7) / 8;
-      const size_t smem = 8 * (size_t)kWarpBytes;
+      const size_t smem = 8 * (size_t)warp_bytes<32>();
       static bool configured = false;
       if (!configured) {
         const cudaError_t e = cudaFuncSetAttribute(
-            fingerprint_tma_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+            fingerprint_tma_kernel<8, 32>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return cuda_fail(e, "fingerprint smem attribute");
         configured = true;
       }
-      fingerprint_tma_kernel<8><<<(unsigned)blocks, 256, smem, stream>>>(
+      fingerprint_tma_kernel<8, 32><<<(unsigned)blocks, 256, smem, stream>>>(
           tokens, n, stride, lens, seed, fp_out, rpw, err);
     } else {
       const int64_t warps = (n + 31) / 32;
-      fingerprint_tma_kernel<1><<<(unsigned)warps, 32, kWarpBytes, stream>>>(
+      fingerprint_tma_kernel<1, 128><<<(unsigned)warps, 32, warp_bytes<128>(), stream>>>(
           tokens, n, stride, lens, seed, fp_out, 32, err);
     }
   } else {
