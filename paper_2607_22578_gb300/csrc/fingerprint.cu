@@ -82,15 +82,15 @@ __device__ __forceinline__ void hash_word(uint32_t& lo, uint32_t& hi, uint32_t w
 // at the end of its row does not send the warp down a second path.  Slots
 // are 144 bytes (9 x 16 B) so the eight lanes of a quarter-warp hit
 // different banks.
-// Per-warp shared memory for chunks of C tokens: two buffers of 32 slots
-// (C*4 + 16 bytes each, an odd multiple of 16 for C = 32 or 128), then two
-// mbarriers and an abort word.
+// Per-warp shared memory for chunks of C tokens: NB round buffers of 32
+// slots (C*4 + 16 bytes each, an odd multiple of 16 for C = 32, 64 or 128),
+// then NB mbarriers and an abort word.
 template <int C>
 constexpr int slot_bytes() { return C * 4 + 16; }
 template <int C>
 constexpr int round_bytes() { return 32 * slot_bytes<C>(); }
-template <int C>
-constexpr int warp_bytes() { return 2 * round_bytes<C>() + 64; }
+template <int C, int NB>
+constexpr int warp_bytes() { return NB * round_bytes<C>() + 8 * NB + 16; }
 
 __device__ __forceinline__ void bulk_copy_g2s(uint32_t dst, const void* src, uint32_t bytes,
                                               uint32_t bar) {
@@ -129,7 +129,7 @@ __device__ __forceinline__ void hash_chunk(uint32_t& lo, uint32_t& hi, const int
   }
 }
 
-template <int WARPS, int kChunk>
+template <int WARPS, int kChunk, int NB>
 __global__ void __launch_bounds__(WARPS * 32) fingerprint_tma_kernel(
     const int32_t* __restrict__ tokens, int64_t n, int32_t stride,
     const int32_t* __restrict__ lens, uint64_t seed, uint64_t* __restrict__ fp_out,
@@ -137,20 +137,19 @@ __global__ void __launch_bounds__(WARPS * 32) fingerprint_tma_kernel(
   extern __shared__ __align__(16) uint8_t tma_smem[];
   constexpr int kSlotBytes = slot_bytes<kChunk>();
   constexpr int kRoundBytes = round_bytes<kChunk>();
-  constexpr int kWarpBytes = warp_bytes<kChunk>();
+  constexpr int kWarpBytes = warp_bytes<kChunk, NB>();
   const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int64_t r_begin = warp * rows_per_warp;
   if (r_begin >= n) return;
   const int64_t r_end = min(n, r_begin + rows_per_warp);
   const uint32_t lane = threadIdx.x & 31u;
   uint8_t* wbuf = tma_smem + (threadIdx.x >> 5) * kWarpBytes;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(wbuf + 2 * kRoundBytes);
-  volatile int* abort_word = reinterpret_cast<volatile int*>(bars + 2);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(wbuf + NB * kRoundBytes);
+  volatile int* abort_word = reinterpret_cast<volatile int*>(bars + NB);
   const uint32_t wbuf_u32 = smem_u32(wbuf);
   const uint32_t seed_lo = (uint32_t)seed, seed_hi = (uint32_t)(seed >> 32);
   if (lane == 0) {
-    mbar_init(bars + 0, 32);
-    mbar_init(bars + 1, 32);
+    for (int b = 0; b < NB; ++b) mbar_init(bars + b, 32);
     *abort_word = 0;
     fence_mbar_init();
   }
@@ -160,9 +159,15 @@ __global__ void __launch_bounds__(WARPS * 32) fingerprint_tma_kernel(
   int64_t irow = -1;
   int32_t ipos = 0, ilen = 0;
   // Staged chunk per buffer: row (or -1), start position, tokens, row length.
-  int64_t prow[2] = {-1, -1};
-  int32_t ppos[2] = {0, 0}, pw[2] = {0, 0}, plen[2] = {0, 0};
-  uint32_t phase[2] = {0u, 0u};
+  int64_t prow[NB];
+  int32_t ppos[NB], pw[NB], plen[NB];
+  uint32_t phase[NB];
+#pragma unroll
+  for (int b = 0; b < NB; ++b) {
+    prow[b] = -1;
+    ppos[b] = pw[b] = plen[b] = 0;
+    phase[b] = 0u;
+  }
   uint32_t lo = seed_lo, hi = seed_hi;
 
   int64_t next = r_begin;
@@ -236,25 +241,34 @@ __global__ void __launch_bounds__(WARPS * 32) fingerprint_tma_kernel(
     return true;
   };
 
-  claim();
-  issue(0);
+  // Rounds 0 .. NB-2 in flight before the first hash; then each step stages
+  // round r + NB - 1 and hashes round r.
+#pragma unroll
+  for (int b = 0; b < NB - 1; ++b) {
+    claim();
+    issue(b);
+  }
   for (;;) {
 #pragma unroll
-    for (int b = 0; b < 2; ++b) {
+    for (int b = 0; b < NB; ++b) {
       claim();
-      issue(b ^ 1);
+      issue((b + NB - 1) % NB);
       if (!hash(b)) {
         set_error(err, kErrTimeout);
         return;
       }
     }
-    const bool pending = irow >= 0 || prow[0] >= 0 || prow[1] >= 0;
+    bool pending = irow >= 0;
+#pragma unroll
+    for (int b = 0; b < NB; ++b) pending |= prow[b] >= 0;
     if (!__any_sync(0xffffffffu, pending) && next >= r_end) break;
   }
-  // The loop's last issue() went to buffer 0 and staged nothing (every lane
-  // was idle); its barrier phase completes on the 32 arrivals alone.  Wait
-  // for it so the warp leaves no barrier phase open.
-  if (!mbar_wait(bars + 0, phase[0], abort_word)) set_error(err, kErrTimeout);
+  // The last NB-1 issue() calls (buffers 0 .. NB-2) staged nothing: every
+  // lane was idle.  Their barrier phases complete on the 32 arrivals alone;
+  // wait for them so the warp leaves no phase open.
+#pragma unroll
+  for (int b = 0; b < NB - 1; ++b)
+    if (!mbar_wait(bars + b, phase[b], abort_word)) set_error(err, kErrTimeout);
 }
 
 // ---- word path (tokens not 16-byte aligned, or row_stride % 4 != 0) -------------------
@@ -343,25 +357,29 @@ hs_status launch_fingerprint(const int32_t* tokens, int64_t n, int32_t stride,
     // round buffers, three blocks = 24 warps per SM) once there are rows for
     // all of them; else one-warp blocks with 128-token chunks, so the warps
     // spread over all SMs and each lane has few, large rounds.
-    const int64_t lanes_full = sms * 24 * 32;
+    const int64_t lanes_full = sms * 12 * 32;
     if (n >= lanes_full) {
-      const int64_t warps_target = sms * 24;
+      // 32-token chunks, four buffers (three rounds in flight), 4-warp
+      // blocks of 73.9 KB: three blocks = 12 warps per SM.
+      const int64_t warps_target = sms * 12;
       const int64_t rpw = (n + warps_target - 1) / warps_target;
       const int64_t warps = (n + rpw - 1) / rpw;
-      const int64_t blocks = (warps + 7) / 8;
-      const size_t smem = 8 * (size_t)warp_bytes<32>();
+      const int64_t blocks = (warps + 3) / 4;
+      const size_t smem = 4 * (size_t)warp_bytes<32, 4>();
       static bool configured = false;
       if (!configured) {
-        const cudaError_t e = cudaFuncSetAttribute(
-            fingerprint_tma_kernel<8, 32>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        const cudaError_t e = cudaFuncSetAttribute(fingerprint_tma_kernel<4, 32, 4>,
+                                                   cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                   (int)smem);
         if (e != cudaSuccess) return cuda_fail(e, "fingerprint smem attribute");
         configured = true;
       }
-      fingerprint_tma_kernel<8, 32><<<(unsigned)blocks, 256, smem, stream>>>(
+      fingerprint_tma_kernel<4, 32, 4><<<(unsigned)blocks, 128, smem, stream>>>(
           tokens, n, stride, lens, seed, fp_out, rpw, err);
     } else {
+      // Few rows: one-warp blocks, 64-token chunks, four buffers (34 KB).
       const int64_t warps = (n + 31) / 32;
-      fingerprint_tma_kernel<1, 128><<<(unsigned)warps, 32, warp_bytes<128>(), stream>>>(
+      fingerprint_tma_kernel<1, 64, 4><<<(unsigned)warps, 32, warp_bytes<64, 4>(), stream>>>(
           tokens, n, stride, lens, seed, fp_out, 32, err);
     }
   } else {
