@@ -2,11 +2,10 @@
 // part of the node semantic signature Sig(v) (Section 3.3, Eq. 2).
 //
 // FNV-1a is a serial chain over the octets of one row, so parallelism comes
-// from rows: each lane of a warp owns one row at a time and streams it through
-// a private shared-memory ring filled by cp.async several blocks ahead.  Rows
-// have different lengths; a lane that has issued its whole row claims the next
-// unclaimed row of its warp's range (warp-synchronous ballot, no atomics), so
-// the lanes of a warp stay busy until the range is drained.
+// from rows: each lane of a warp owns one row at a time.  Rows are split into
+// full chunks of 32 tokens, hashed in registers by the chunk kernel with a
+// straight-line, predicate-free loop, and a tail of L mod 32 tokens, finished
+// by a one-thread-per-row tail kernel from the partial state.
 //
 // Arithmetic: h = (hi:lo) as two 32-bit words; a multiply by the prime
 // 2^40 + 0x1b3 is one wide 32x32 multiply, one multiply-add and one
@@ -66,107 +65,68 @@ __device__ __forceinline__ void hash_word(uint32_t& lo, uint32_t& hi, uint32_t w
 
 
 
-// ---- vector path: per-lane bulk copies (TMA) --------------------------------------
-// A warp owns 32 rows at a time, one per lane.  In each round every lane
-// stages the next chunk of up to kChunk tokens of its own row with one bulk
-// copy (cp.async.bulk: a contiguous, 16-byte aligned range of the row) into
-// its own slot of the warp's round buffer; the 32 copies of a round complete
-// on one mbarrier.  While a round's copies are in flight the lanes hash the
-// previous round's chunks (two buffers).  Each lane reads only its own slot,
-// so lanes never wait for each other except through the mbarrier.  A lane
-// whose row is exhausted claims the warp's next row for the next round
-// (lengths prefetched 64 rows ahead, handed out by shuffle).
+// ---- vector path: full chunks in registers, tails in a second kernel -------------
+// A warp owns 32 rows at a time, one per lane.  The chunk kernel hashes only
+// FULL chunks of T = 32 tokens: tokens [0, floor(L/T)*T) of every row with
+// L >= T.  Each lane loads its next chunk with 16- or 32-byte vector loads
+// straight into registers one chunk ahead of the chunk it hashes (NB register
+// buffers), so every lane runs the same straight-line hash over T tokens: no
+// per-token predicates and no masking.  After its last full chunk a row's
+// state goes to fp_out: the final fingerprint when T divides L, otherwise the
+// partial state, which the tail kernel finishes with the last L mod T tokens
+// (one thread per row, so the few short tails run with the whole GPU's
+// parallelism instead of serially at the end of each warp).  Rows shorter
+// than T and rows with an invalid length are left entirely to the tail
+// kernel.  A lane that has issued its row's last chunk claims the next
+// unclaimed row of its warp's range (lengths prefetched 64 rows ahead and
+// handed out by shuffle).
 //
-// The hash loop is uniform across lanes: a fixed walk over the chunk's
-// 16-byte pieces with tokens past the chunk's end masked per word, so a lane
-// at the end of its row does not send the warp down a second path.  Slots
-// are 144 bytes (9 x 16 B) so the eight lanes of a quarter-warp hit
-// different banks.
-// Per-warp shared memory for chunks of C tokens: NB round buffers of 32
-// slots (C*4 + 16 bytes each, an odd multiple of 16 for C = 32, 64 or 128),
-// then NB mbarriers and an abort word.
-template <int C>
-constexpr int slot_bytes() { return C * 4 + 16; }
-template <int C>
-constexpr int round_bytes() { return 32 * slot_bytes<C>(); }
-template <int C, int NB>
-constexpr int warp_bytes() { return NB * round_bytes<C>() + 8 * NB + 16; }
+// A chunk whose tokens are all below 65536 (in every live lane) takes the
+// two-round small-token hash; otherwise the whole chunk takes the octet-wise
+// rounds, which are exact for every token.
 
-__device__ __forceinline__ void bulk_copy_g2s(uint32_t dst, const void* src, uint32_t bytes,
-                                              uint32_t bar) {
-  asm volatile(
-      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::
-          "r"(dst),
-      "l"(src), "r"(bytes), "r"(bar)
-      : "memory");
-}
-
-// Hash tokens [0, w) of a chunk in shared memory (w <= C).  Every lane
-// walks the same pieces; words at or past w are masked out of the fast-path
-// test and skipped.
-template <int C>
-__device__ __forceinline__ void hash_chunk(uint32_t& lo, uint32_t& hi, const int4* blk, int w) {
-#pragma unroll 2
-  for (int pc = 0; pc < C / 4; ++pc) {
-    const int n = w - 4 * pc;                     // valid words in this piece (may be <= 0)
-    if (__all_sync(0xffffffffu, n <= 0)) break;
-    const int4 v = blk[pc];
-    const uint32_t x = n > 0 ? (uint32_t)v.x : 0u;
-    const uint32_t y = n > 1 ? (uint32_t)v.y : 0u;
-    const uint32_t z = n > 2 ? (uint32_t)v.z : 0u;
-    const uint32_t q = n > 3 ? (uint32_t)v.w : 0u;
-    if (((x | y | z | q) >> 16) == 0u) {
-      if (n > 0) hash_word_small(lo, hi, x);
-      if (n > 1) hash_word_small(lo, hi, y);
-      if (n > 2) hash_word_small(lo, hi, z);
-      if (n > 3) hash_word_small(lo, hi, q);
-    } else {
-      if (n > 0) hash_word(lo, hi, x);
-      if (n > 1) hash_word(lo, hi, y);
-      if (n > 2) hash_word(lo, hi, z);
-      if (n > 3) hash_word(lo, hi, q);
-    }
+template <int VB>
+__device__ __forceinline__ void load_vec(const int32_t* p, uint32_t* x) {
+  if constexpr (VB == 32) {
+    asm volatile("ld.global.nc.L1::no_allocate.v8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+                 : "=r"(x[0]), "=r"(x[1]), "=r"(x[2]), "=r"(x[3]), "=r"(x[4]), "=r"(x[5]),
+                   "=r"(x[6]), "=r"(x[7])
+                 : "l"(p));
+  } else {
+    asm volatile("ld.global.nc.L1::no_allocate.v4.b32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(x[0]), "=r"(x[1]), "=r"(x[2]), "=r"(x[3])
+                 : "l"(p));
   }
 }
 
-template <int WARPS, int kChunk, int NB>
-__global__ void __launch_bounds__(WARPS * 32) fingerprint_tma_kernel(
+constexpr int kTailChunk = 32;  // T: tokens per full chunk
+
+template <int VB, int K, int NB>
+__global__ void __launch_bounds__(256) fingerprint_chunks_kernel(
     const int32_t* __restrict__ tokens, int64_t n, int32_t stride,
     const int32_t* __restrict__ lens, uint64_t seed, uint64_t* __restrict__ fp_out,
-    int64_t rows_per_warp, unsigned* err) {
-  extern __shared__ __align__(16) uint8_t tma_smem[];
-  constexpr int kSlotBytes = slot_bytes<kChunk>();
-  constexpr int kRoundBytes = round_bytes<kChunk>();
-  constexpr int kWarpBytes = warp_bytes<kChunk, NB>();
+    int64_t rows_per_warp) {
+  constexpr int W = VB / 4;  // tokens per vector load
+  constexpr int T = W * K;   // tokens per chunk
+  static_assert(T == kTailChunk, "chunk size shared with the tail kernel");
   const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int64_t r_begin = warp * rows_per_warp;
   if (r_begin >= n) return;
   const int64_t r_end = min(n, r_begin + rows_per_warp);
   const uint32_t lane = threadIdx.x & 31u;
-  uint8_t* wbuf = tma_smem + (threadIdx.x >> 5) * kWarpBytes;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(wbuf + NB * kRoundBytes);
-  volatile int* abort_word = reinterpret_cast<volatile int*>(bars + NB);
-  const uint32_t wbuf_u32 = smem_u32(wbuf);
   const uint32_t seed_lo = (uint32_t)seed, seed_hi = (uint32_t)(seed >> 32);
-  if (lane == 0) {
-    for (int b = 0; b < NB; ++b) mbar_init(bars + b, 32);
-    *abort_word = 0;
-    fence_mbar_init();
-  }
-  __syncwarp();
 
-  // Issue side: the next chunk of this lane's row to stage.
+  // Issue side: the row being loaded, the next chunk's start, the end of its
+  // full chunks.
   int64_t irow = -1;
-  int32_t ipos = 0, ilen = 0;
-  // Staged chunk per buffer: row (or -1), start position, tokens, row length.
-  int64_t prow[NB];
-  int32_t ppos[NB], pw[NB], plen[NB];
-  uint32_t phase[NB];
+  int32_t ipos = 0, iend = 0;
+  uint32_t buf[NB][T];
+  int64_t brow[NB];
+  bool bfirst[NB], blast[NB];
 #pragma unroll
   for (int b = 0; b < NB; ++b) {
-    prow[b] = -1;
-    ppos[b] = pw[b] = plen[b] = 0;
-    phase[b] = 0u;
+    brow[b] = -1;
+    bfirst[b] = blast[b] = false;
   }
   uint32_t lo = seed_lo, hi = seed_hi;
 
@@ -186,17 +146,11 @@ __global__ void __launch_bounds__(WARPS * 32) fingerprint_tma_kernel(
       const int32_t La = __shfl_sync(0xffffffffu, len_a, off & 31);
       const int32_t Lb = __shfl_sync(0xffffffffu, len_b, off & 31);
       if (irow < 0 && rank < avail) {
-        const int64_t r = next + rank;
         const int32_t L = off < 32 ? La : Lb;
-        if (L < 0 || L > stride) {
-          set_error(err, kErrInvalidArg);
-          fp_out[r] = 0ull;
-        } else if (L == 0) {
-          fp_out[r] = seed;
-        } else {
-          irow = r;
+        if (L >= T && L <= stride) {
+          irow = next + rank;
           ipos = 0;
-          ilen = L;
+          iend = (L / T) * T;
         }
       }
       next += min((int64_t)__popc(need), avail);
@@ -209,40 +163,41 @@ __global__ void __launch_bounds__(WARPS * 32) fingerprint_tma_kernel(
     }
   };
 
-  // Stage this lane's next chunk into its slot of buffer b (one bulk copy).
+  // Load this lane's next full chunk into buffer b.
   auto issue = [&](int b) {
-    const int32_t w = irow >= 0 ? min(kChunk, ilen - ipos) : 0;
-    const uint32_t bytes = (uint32_t)((w + 3) >> 2) * 16u;
-    prow[b] = irow;
-    ppos[b] = ipos;
-    pw[b] = w;
-    plen[b] = ilen;
-    mbar_arrive_expect_tx(bars + b, bytes);
-    if (bytes) {
-      bulk_copy_g2s(wbuf_u32 + b * kRoundBytes + lane * kSlotBytes,
-                    tokens + irow * (int64_t)stride + ipos, bytes, smem_u32(bars + b));
-      ipos += w;
-      if (ipos >= ilen) irow = -1;
+    brow[b] = irow;
+    if (irow >= 0) {
+      const int32_t* src = tokens + irow * (int64_t)stride + ipos;
+#pragma unroll
+      for (int j = 0; j < K; ++j) load_vec<VB>(src + j * W, &buf[b][j * W]);
+      bfirst[b] = ipos == 0;
+      ipos += T;
+      blast[b] = ipos == iend;
+      if (blast[b]) irow = -1;
     }
   };
 
-  auto hash = [&](int b) -> bool {
-    if (!mbar_wait(bars + b, phase[b], abort_word)) return false;
-    phase[b] ^= 1u;
-    if (prow[b] >= 0 && ppos[b] == 0) {
-      lo = seed_lo;
-      hi = seed_hi;
+  // Hash buffer b (every lane, live or not: an idle lane's result is dropped).
+  auto consume = [&](int b) {
+    const bool live = brow[b] >= 0;
+    lo = (live && bfirst[b]) ? seed_lo : lo;
+    hi = (live && bfirst[b]) ? seed_hi : hi;
+    uint32_t any = 0;
+#pragma unroll
+    for (int t = 0; t < T; ++t) any |= buf[b][t];
+    if (__all_sync(0xffffffffu, !live || (any >> 16) == 0u)) {
+#pragma unroll
+      for (int t = 0; t < T; ++t) hash_word_small(lo, hi, buf[b][t]);
+    } else {
+#pragma unroll
+      for (int t = 0; t < T; ++t) hash_word_full(lo, hi, buf[b][t]);
     }
-    hash_chunk<kChunk>(lo, hi,
-                       reinterpret_cast<const int4*>(wbuf + b * kRoundBytes + lane * kSlotBytes),
-                       prow[b] >= 0 ? pw[b] : 0);
-    if (prow[b] >= 0 && ppos[b] + pw[b] >= plen[b]) fp_out[prow[b]] = ((uint64_t)hi << 32) | lo;
-    prow[b] = -1;
-    return true;
+    if (live && blast[b]) fp_out[brow[b]] = ((uint64_t)hi << 32) | lo;
+    brow[b] = -1;
   };
 
-  // Rounds 0 .. NB-2 in flight before the first hash; then each step stages
-  // round r + NB - 1 and hashes round r.
+  // Chunks 0 .. NB-2 in flight before the first hash; then each step loads
+  // chunk c + NB - 1 and hashes chunk c.
 #pragma unroll
   for (int b = 0; b < NB - 1; ++b) {
     claim();
@@ -253,22 +208,54 @@ __global__ void __launch_bounds__(WARPS * 32) fingerprint_tma_kernel(
     for (int b = 0; b < NB; ++b) {
       claim();
       issue((b + NB - 1) % NB);
-      if (!hash(b)) {
-        set_error(err, kErrTimeout);
-        return;
-      }
+      consume(b);
     }
     bool pending = irow >= 0;
 #pragma unroll
-    for (int b = 0; b < NB; ++b) pending |= prow[b] >= 0;
+    for (int b = 0; b < NB; ++b) pending |= brow[b] >= 0;
     if (!__any_sync(0xffffffffu, pending) && next >= r_end) break;
   }
-  // The last NB-1 issue() calls (buffers 0 .. NB-2) staged nothing: every
-  // lane was idle.  Their barrier phases complete on the 32 arrivals alone;
-  // wait for them so the warp leaves no phase open.
+}
+
+// The last L mod T tokens of every row (the whole row when L < T), one thread
+// per row, continuing from the partial state the chunk kernel left in fp_out.
+// Also the row-length checks: an invalid length sets the error flag and a
+// zero fingerprint; an empty row gets the seed.  Needs 16-byte aligned rows.
+__global__ void __launch_bounds__(256) fingerprint_tails_kernel(
+    const int32_t* __restrict__ tokens, int64_t n, int32_t stride,
+    const int32_t* __restrict__ lens, uint64_t seed, uint64_t* __restrict__ fp_out,
+    unsigned* err) {
+  constexpr int T = kTailChunk;
+  for (int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; r < n;
+       r += (int64_t)gridDim.x * blockDim.x) {
+    const int32_t L = lens ? __ldg(lens + r) : stride;
+    if (L < 0 || L > stride) {
+      set_error(err, kErrInvalidArg);
+      fp_out[r] = 0ull;
+      continue;
+    }
+    const int32_t m = L % T;
+    if (m == 0 && L > 0) continue;  // the chunk kernel wrote the final value
+    uint32_t lo = (uint32_t)seed, hi = (uint32_t)(seed >> 32);
+    if (L >= T) {
+      const uint64_t st = fp_out[r];
+      lo = (uint32_t)st;
+      hi = (uint32_t)(st >> 32);
+    }
+    const int32_t* src = tokens + r * (int64_t)stride + (L - m);
+    uint4 v[T / 4];
 #pragma unroll
-  for (int b = 0; b < NB - 1; ++b)
-    if (!mbar_wait(bars + b, phase[b], abort_word)) set_error(err, kErrTimeout);
+    for (int q = 0; q < T / 4; ++q)
+      if (4 * q < m) v[q] = __ldg(reinterpret_cast<const uint4*>(src + 4 * q));
+#pragma unroll
+    for (int q = 0; q < T / 4; ++q) {
+      if (4 * q < m) hash_word(lo, hi, v[q].x);
+      if (4 * q + 1 < m) hash_word(lo, hi, v[q].y);
+      if (4 * q + 2 < m) hash_word(lo, hi, v[q].z);
+      if (4 * q + 3 < m) hash_word(lo, hi, v[q].w);
+    }
+    fp_out[r] = ((uint64_t)hi << 32) | lo;
+  }
 }
 
 // ---- word path (tokens not 16-byte aligned, or row_stride % 4 != 0) -------------------
@@ -343,44 +330,57 @@ __global__ void __launch_bounds__(256) fingerprint_words_kernel(
   }
 }
 
+
+template <int VB, int K, int NB>
+hs_status launch_chunks(const int32_t* tokens, int64_t n, int32_t stride, const int32_t* lens,
+                        uint64_t seed, uint64_t* fp_out, int64_t sms, cudaStream_t stream) {
+  // Resident warps per SM at this kernel's register count (one query per
+  // process; the kernel uses no shared memory).
+  static int warps_per_sm = 0;
+  if (warps_per_sm == 0) {
+    int blocks = 0;
+    const cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
+        &blocks, fingerprint_chunks_kernel<VB, K, NB>, 256, 0);
+    if (e != cudaSuccess) return cuda_fail(e, "fingerprint occupancy");
+    warps_per_sm = blocks > 0 ? blocks * 8 : 8;
+  }
+  const int64_t warps_target = sms * warps_per_sm;
+  int64_t rpw = (n + warps_target - 1) / warps_target;
+  if (rpw < 32) rpw = 32;
+  const int64_t warps = (n + rpw - 1) / rpw;
+  // Few warps: one-warp blocks, so they spread over all SMs.
+  const int threads = warps >= sms * 8 ? 256 : 32;
+  const int64_t blocks = (warps * 32 + threads - 1) / threads;
+  fingerprint_chunks_kernel<VB, K, NB><<<(unsigned)blocks, threads, 0, stream>>>(
+      tokens, n, stride, lens, seed, fp_out, rpw);
+  count_launches(1);
+  return HS_OK;
+}
+
 }  // namespace
 
 hs_status launch_fingerprint(const int32_t* tokens, int64_t n, int32_t stride,
                              const int32_t* lens, uint64_t seed, uint64_t* fp_out,
                              cudaStream_t stream) {
-  const bool vec = ((reinterpret_cast<uintptr_t>(tokens) & 15u) == 0) && (stride % 4 == 0);
+  const uintptr_t base = reinterpret_cast<uintptr_t>(tokens);
+  const bool vec32 = (base & 31u) == 0 && stride % 8 == 0;
+  const bool vec16 = (base & 15u) == 0 && stride % 4 == 0;
   unsigned* err = device_error_word();
   if (!err) return fail(HS_ERR_CUDA, "could not resolve the device error word");
   const int64_t sms = num_sms();
-  if (vec) {
-    // Per-lane bulk copies: 8-warp blocks with 32-token chunks (74 KB of
-    // round buffers, three blocks = 24 warps per SM) once there are rows for
-    // all of them; else one-warp blocks with 128-token chunks, so the warps
-    // spread over all SMs and each lane has few, large rounds.
-    const int64_t lanes_full = sms * 12 * 32;
-    if (n >= lanes_full) {
-      // 32-token chunks, four buffers (three rounds in flight), 4-warp
-      // blocks of 73.9 KB: three blocks = 12 warps per SM.
-      const int64_t warps_target = sms * 12;
-      const int64_t rpw = (n + warps_target - 1) / warps_target;
-      const int64_t warps = (n + rpw - 1) / rpw;
-      const int64_t blocks = (warps + 3) / 4;
-      const size_t smem = 4 * (size_t)warp_bytes<32, 4>();
-      static bool configured = false;
-      if (!configured) {
-        const cudaError_t e = cudaFuncSetAttribute(fingerprint_tma_kernel<4, 32, 4>,
-                                                   cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                   (int)smem);
-        if (e != cudaSuccess) return cuda_fail(e, "fingerprint smem attribute");
-        configured = true;
-      }
-      fingerprint_tma_kernel<4, 32, 4><<<(unsigned)blocks, 128, smem, stream>>>(
-          tokens, n, stride, lens, seed, fp_out, rpw, err);
-    } else {
-      // Few rows: one-warp blocks, 64-token chunks, four buffers (34 KB).
-      const int64_t warps = (n + 31) / 32;
-      fingerprint_tma_kernel<1, 64, 4><<<(unsigned)warps, 32, warp_bytes<64, 4>(), stream>>>(
-          tokens, n, stride, lens, seed, fp_out, 32, err);
+  if (vec16) {
+    if (stride >= kTailChunk) {
+      const hs_status st =
+          vec32 ? launch_chunks<32, 4, 2>(tokens, n, stride, lens, seed, fp_out, sms, stream)
+                : launch_chunks<16, 8, 2>(tokens, n, stride, lens, seed, fp_out, sms, stream);
+      if (st != HS_OK) return st;
+    }
+    if (lens || stride % kTailChunk != 0 || stride == 0) {
+      int64_t blocks = (n + 255) / 256;
+      if (blocks > sms * 64) blocks = sms * 64;
+      fingerprint_tails_kernel<<<(unsigned)blocks, 256, 0, stream>>>(tokens, n, stride, lens,
+                                                                     seed, fp_out, err);
+      count_launches(1);
     }
   } else {
     const int64_t warps_target = sms * 32;
@@ -390,8 +390,8 @@ hs_status launch_fingerprint(const int32_t* tokens, int64_t n, int32_t stride,
     const int64_t blocks = (warps + 7) / 8;
     fingerprint_words_kernel<<<(unsigned)blocks, 256, 0, stream>>>(tokens, n, stride, lens, seed,
                                                                    fp_out, rpw, err);
+    count_launches(1);
   }
-  count_launches(1);
   return cuda_fail(cudaGetLastError(), "fingerprint launch");
 }
 

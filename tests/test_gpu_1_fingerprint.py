@@ -116,3 +116,25 @@ def test_deterministic():
     a = gpu_fp(w["tokens"], w["lens"])
     b = gpu_fp(w["tokens"], w["lens"])
     assert (a == b).all()
+
+
+@pytest.mark.parametrize("stride,offset", [(200, 0), (200, 4), (100, 0)])
+def test_chunk_paths_mixed_tokens(stride, offset):
+    # Rows of several 32-token chunks plus a ragged tail.  offset 4 leaves the
+    # base 16-byte (not 32-byte) aligned and stride 100 is not a multiple of
+    # 8 tokens: both take 16-byte loads.  One large token in every third row
+    # sends its chunk (and every other lane's chunk in that warp step) down
+    # the octet-wise rounds.
+    rng = np.random.default_rng(stride + offset)
+    n = 2 * (stride + 1)
+    tok = rng.integers(0, 32000, size=(n, stride)).astype(np.int32)
+    rows = np.arange(0, n, 3)
+    tok[rows, rng.integers(0, stride, size=len(rows))] = rng.integers(65536, 2**31 - 1,
+                                                                      size=len(rows))
+    lens = (np.arange(n) % (stride + 1)).astype(np.int32)
+    flat = np.zeros(offset + n * stride, np.int32)
+    flat[offset:] = tok.reshape(-1)
+    t = to_dev(flat)[offset:].view(n, stride)
+    out = hs.hs_fingerprint(t, to_dev(lens))
+    hs.hs_get_device_error()
+    assert (fp_host(out) == oracle.fingerprint(tok, lens)).all()
