@@ -7,17 +7,27 @@
 //
 // K6 (retrieve_kernel) is a persistent, warp-specialised tcgen05 kernel:
 //   warp 0      TMA producer: 128x64 query tile + 256x64 corpus tile per
-//               stage, 128-byte swizzle, 4-stage mbarrier ring;
-//   warp 1      MMA issuer: 4 x tcgen05.mma (M=128, N=256, K=16) per stage
-//               into a double-buffered fp32 accumulator in tensor memory
-//               (2 x 256 columns), tcgen05.commit releases smem stages;
+//               stage (CTA pair: + the 128x64 half of it), 128-byte swizzle,
+//               4-stage (pair: 6-stage) mbarrier ring;
+//   warp 1      MMA issuer: 4 x tcgen05.mma (M=128 or pair M=256, N=256,
+//               K=16) per stage into a double-buffered fp32 accumulator in
+//               tensor memory (2 x 256 columns), tcgen05.commit releases
+//               smem stages;
 //   warps 2-9   epilogue: two warps per TMEM lane quarter, each reading half
 //               of the 128 x 256 score tile with tcgen05.ld; thread = (query,
 //               column half); threshold filter + per-query top-k.
+// With two or more query blocks the CTAs run as pairs (clusters of two,
+// cta_group::2): the even CTA issues M = 256 MMAs that take the two CTAs'
+// query blocks as the two halves of A and the two 128-row halves of the
+// corpus tile, one staged in each CTA, as B.  Each CTA's tensor memory holds
+// the scores of its own query block against the whole tile, so each SM
+// stages half of every corpus tile and reads half as much shared memory per
+// MMA as a single CTA would.  The producer of each CTA loads its own query
+// tile and corpus half; both complete on the even CTA's barrier.
 // The Q x N score matrix never leaves the SM.  Work is split into units
-// (query block, corpus split); units that share a corpus split run at the
-// same time on different SMs, so each corpus tile is read from HBM about once
-// and served to the other query blocks from L2.
+// (query block pair, corpus split); units that share a corpus split run at
+// the same time on different SMs, so each corpus tile is read from HBM about
+// once and served to the other query blocks from L2.
 //
 // Top-k state per (query, half): for k <= 32 a sorted list in registers
 // (KREG = 16 or 32 slots).  A 32-column chunk whose maximum beats no lane's
@@ -41,28 +51,38 @@ constexpr int BM = 128;               // queries per tile: UMMA M = TMEM lanes
 constexpr int BN = 256;               // corpus rows per tile: UMMA N
 constexpr int BK = 64;                // K per stage: one 128-byte swizzle row
 constexpr int UK = 16;                // K per tcgen05.mma, kind::f16
-constexpr int kStages = 4;
 constexpr int kEpiWarps = 8;
 constexpr int kEpi = kEpiWarps * 32;  // epilogue threads
 constexpr int kThreads = 64 + kEpi;
 constexpr int kHalfCols = BN / 2;     // columns per epilogue thread per tile
 constexpr uint32_t kABytes = BM * BK * 2;
 constexpr uint32_t kBBytes = BN * BK * 2;
-constexpr uint32_t kStageBytes = kABytes + kBBytes;
 constexpr uint32_t kTmemCols = 2 * BN;
 constexpr int kCap = 16;              // candidate buffer per thread (large-k path)
 constexpr int kMergeMax = 16384;      // lists * k bound for K7
 constexpr size_t kBarBytes = 256;
 constexpr size_t kEpiSmem = (size_t)kEpi * 32 * 4;  // 32 KB: staging or candidate buffer
 static_assert((size_t)kCap * kEpi * 8 == kEpiSmem, "candidate buffer size");
-constexpr size_t kSmem = 1024 + (size_t)kStages * kStageBytes + kBarBytes + kEpiSmem;
+// Shared-memory ring per CTA.  Single CTA: a 128-row query tile and the
+// whole 256-row corpus tile per stage, 4 stages.  CTA pair (cta_group::2):
+// each CTA stages its own query tile and its 128-row half of the corpus
+// tile, so a stage is 32 KB and 6 fit.
+template <int CL>
+struct Ring {
+  static constexpr int stages = CL == 2 ? 6 : 4;
+  static constexpr uint32_t b_bytes = kBBytes / CL;
+  static constexpr uint32_t stage_bytes = kABytes + b_bytes;
+  static constexpr size_t smem = 1024 + (size_t)stages * stage_bytes + kBarBytes + kEpiSmem;
+};
+static_assert(Ring<1>::smem <= 232448 && Ring<2>::smem <= 232448, "shared memory per CTA");
+static_assert(8 * (2 * Ring<2>::stages + 4) + 8 <= kBarBytes, "barrier area");
 
 struct Params {
   int64_t Qmax, N, tiles;
   const int32_t* count_dev;  // queries to process: min(*count_dev, Qmax); NULL: Qmax
   int32_t k, kb_count;
   int32_t slots;             // concurrent unit executors the plan targets (CTAs / cl)
-  int32_t cl;                // CTAs per cluster: 1, or 2 sharing corpus tiles by multicast
+  int32_t cl;                // CTAs per cluster: 1, or 2 forming a CTA pair (M = 256 MMA)
   float* part_s;     // [Q][2 * nsplit][k]: one list per (split, column half)
   int32_t* part_i;
   float* list_s;     // large-k: [grid][kEpi][2][k]
@@ -234,6 +254,9 @@ template <int KREG, int CL>
 __global__ void __launch_bounds__(kThreads, 1)
     retrieve_kernel(const __grid_constant__ CUtensorMap tmap_q,
                     const __grid_constant__ CUtensorMap tmap_c, const Params p) {
+  constexpr int kStages = Ring<CL>::stages;
+  constexpr uint32_t kBLocal = Ring<CL>::b_bytes;
+  constexpr uint32_t kStageBytes = Ring<CL>::stage_bytes;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
@@ -248,15 +271,17 @@ __global__ void __launch_bounds__(kThreads, 1)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   uint8_t* epi_smem = smem + kStages * kStageBytes + kBarBytes;
 
+  // CTA pair: the even CTA (rank 0) owns the full and tempty barriers that
+  // both CTAs' loads and epilogues signal, and issues every MMA.
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(full + s, 1);
-      mbar_init(empty + s, CL);          // one commit from each CTA that fills the stage
+      mbar_init(empty + s, 1);
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(tfull + a, 1);
-      mbar_init(tempty + a, kEpiWarps);
+      mbar_init(tempty + a, kEpiWarps * CL);
     }
     *abort_flag = 0;
     fence_mbar_init();
@@ -266,13 +291,18 @@ __global__ void __launch_bounds__(kThreads, 1)
     prefetch_tmap(&tmap_c);
   }
   if (warp == 1) {
-    tmem_alloc(tmem_slot, kTmemCols);
-    tmem_relinquish();
+    if (CL == 2) {
+      tmem_alloc_pair(tmem_slot, kTmemCols);
+      tmem_relinquish_pair();
+    } else {
+      tmem_alloc(tmem_slot, kTmemCols);
+      tmem_relinquish();
+    }
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  if (CL > 1) cluster_sync();            // peers' barriers exist before any multicast
+  if (CL > 1) cluster_sync();            // the pair's barriers exist before any remote signal
   const uint32_t tmem_base = *tmem_slot;
   const int rank = CL > 1 ? (int)cluster_ctarank() : 0;
   const int64_t Q = query_count(p);
@@ -293,22 +323,25 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int64_t t = t0; t < t1; ++t) {
           for (int kb = 0; kb < p.kb_count; ++kb) {
             if (!mbar_wait(empty + stage, phase ^ 1u, abort_flag)) goto producer_done;
-            mbar_arrive_expect_tx(full + stage, kStageBytes);
             // A query block past the last addressable row is loaded from
             // row 0 instead: its scores are masked, and no box lies wholly
             // outside the tensor.
             const int32_t qy = (int64_t)qb * BM < p.Qmax ? qb * BM : 0;
-            tma_load_2d_hint(sA + stage * kABytes, &tmap_q, full + stage, kb * BK, qy, pol_q);
             if (CL == 1) {
-              tma_load_2d_hint(sB + stage * kBBytes, &tmap_c, full + stage, kb * BK,
+              mbar_arrive_expect_tx(full + stage, kStageBytes);
+              tma_load_2d_hint(sA + stage * kABytes, &tmap_q, full + stage, kb * BK, qy, pol_q);
+              tma_load_2d_hint(sB + stage * kBLocal, &tmap_c, full + stage, kb * BK,
                                (int32_t)(t * BN), pol_c);
             } else {
-              // This CTA loads its half of the corpus tile into both CTAs.
-              // A half past the last row re-reads the first half (masked).
+              // Both CTAs' bytes complete on the even CTA's full barrier,
+              // armed there for the pair.  A corpus half past the last row
+              // re-reads the tile's first half (masked).
+              if (rank == 0) mbar_arrive_expect_tx(full + stage, 2 * kStageBytes);
+              const uint32_t bar = cluster_smem_addr(full + stage, 0);
               const int64_t cy = t * BN + rank * (BN / CL);
-              tma_load_2d_mc_hint(sB + stage * kBBytes + rank * (kBBytes / CL), &tmap_c,
-                                  full + stage, kb * BK, (int32_t)(cy < p.N ? cy : t * BN),
-                                  (uint16_t)((1u << CL) - 1u), pol_c);
+              tma_load_2d_pair_hint(sA + stage * kABytes, &tmap_q, bar, kb * BK, qy, pol_q);
+              tma_load_2d_pair_hint(sB + stage * kBLocal, &tmap_c, bar, kb * BK,
+                                    (int32_t)(cy < p.N ? cy : t * BN), pol_c);
             }
             if (++stage == kStages) {
               stage = 0;
@@ -321,8 +354,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16_f32(BM, BN);
+    if (lane == 0 && rank == 0) {
+      constexpr uint32_t idesc = idesc_bf16_f32(BM * CL, BN);
       uint32_t stage = 0, phase = 0, tile_i = 0;
       for (int64_t u = u0; u < units; u += ustep) {
         int qb, split;
@@ -337,21 +370,28 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!mbar_wait(full + stage, phase, abort_flag)) goto mma_done;
             tc_fence_after();
             const uint64_t a0 = smem_desc_k_sw128(smem_u32(sA + stage * kABytes));
-            const uint64_t b0 = smem_desc_k_sw128(smem_u32(sB + stage * kBBytes));
+            const uint64_t b0 = smem_desc_k_sw128(smem_u32(sB + stage * kBLocal));
 #pragma unroll
-            for (int kk = 0; kk < BK / UK; ++kk)
-              umma_bf16(d_tmem, a0 + (uint64_t)(kk * UK * 2 / 16), b0 + (uint64_t)(kk * UK * 2 / 16),
-                        idesc, (kb | kk) != 0 ? 1u : 0u);
+            for (int kk = 0; kk < BK / UK; ++kk) {
+              const uint64_t koff = (uint64_t)(kk * UK * 2 / 16);
+              if (CL == 1)
+                umma_bf16(d_tmem, a0 + koff, b0 + koff, idesc, (kb | kk) != 0 ? 1u : 0u);
+              else
+                umma_bf16_pair(d_tmem, a0 + koff, b0 + koff, idesc, (kb | kk) != 0 ? 1u : 0u);
+            }
             if (CL == 1)
               umma_commit(empty + stage);
             else
-              umma_commit_mc(empty + stage, (uint16_t)((1u << CL) - 1u));
+              umma_commit_pair_mc(empty + stage, 0x3);
             if (++stage == kStages) {
               stage = 0;
               phase ^= 1u;
             }
           }
-          umma_commit(tfull + acc);
+          if (CL == 1)
+            umma_commit(tfull + acc);
+          else
+            umma_commit_pair_mc(tfull + acc, 0x3);
         }
       }
     mma_done:;
@@ -474,7 +514,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(tempty + acc);
+        if (lane == 0) {
+          if (CL == 1)
+            mbar_arrive(tempty + acc);
+          else
+            mbar_arrive_cluster(cluster_smem_addr(tempty + acc, 0));
+        }
       }
       if (valid_q) {
         const size_t o = ((size_t)q * lists + 2 * split + half) * k;
@@ -501,10 +546,14 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   tc_fence_before();
   __syncthreads();
+  if (CL > 1) cluster_sync();            // the pair's MMAs and remote signals are done
   if (warp == 1) {
     __syncwarp();
     tc_fence_after();
-    tmem_dealloc(tmem_base, kTmemCols);
+    if (CL == 2)
+      tmem_dealloc_pair(tmem_base, kTmemCols);
+    else
+      tmem_dealloc(tmem_base, kTmemCols);
   }
   if (CL > 1) cluster_sync();            // no CTA leaves while its peer may still signal it
   if (threadIdx.x == 0 && *abort_flag) set_error(p.err, kErrTimeout);
@@ -612,7 +661,8 @@ hs_status configure_kernel() {
   static bool configured = false;
   if (!configured) {
     cudaError_t e = cudaFuncSetAttribute(retrieve_kernel<KREG, CL>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmem);
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)Ring<CL>::smem);
     if (e != cudaSuccess) return cuda_fail(e, "retrieve smem attribute");
     configured = true;
   }
@@ -633,7 +683,7 @@ int64_t max_pairs() {
     attr[0].val.clusterDim.z = 1;
     cfg.gridDim = dim3((unsigned)(num_sms() & ~1), 1, 1);
     cfg.blockDim = dim3(kThreads, 1, 1);
-    cfg.dynamicSmemBytes = kSmem;
+    cfg.dynamicSmemBytes = Ring<2>::smem;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     int n = 0;
@@ -654,7 +704,7 @@ hs_status launch_kernel(const CUtensorMap& mq, const CUtensorMap& mc, const Para
   attr[0].val.clusterDim.z = 1;
   cfg.gridDim = dim3((unsigned)grid, 1, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
-  cfg.dynamicSmemBytes = kSmem;
+  cfg.dynamicSmemBytes = Ring<CL>::smem;
   cfg.stream = stream;
   cfg.attrs = attr;
   cfg.numAttrs = CL > 1 ? 1 : 0;
