@@ -107,10 +107,10 @@ hs_status hs_fingerprint(const int32_t* tokens, int64_t n_rows, int32_t row_stri
  * these rows that are equal for equal rows (as hs_fingerprint produces with
  * one seed); different rows may share a fingerprint (a collision): they are
  * told apart by a full row comparison, never merged.  Cost is linear in the
- * row bytes plus a radix sort of the upper 32 bits of the fingerprints; a
- * group of rows whose fingerprints agree in those bits but whose contents
- * differ is resolved by an extra pass that is quadratic in the number of
- * distinct rows in that group.
+ * row bytes of rows that have an equal-fingerprint predecessor, plus one hash
+ * table insert and lookup per row; rows whose fingerprint equals an earlier
+ * row's but whose contents differ (a collision) are regrouped by an extra
+ * pass that is quadratic in the number of such rows.
  *
  * fp              device uint64 [n_rows], 8-byte aligned.
  * tokens, n_rows, row_stride, lens   as for hs_fingerprint;

@@ -2,27 +2,26 @@
 // topological fusion within a time window (Section 3.3, "Dynamic Fusion and
 // Reuse Mechanism" (I)) and the merge sets M(v*) of Appendix A.2.
 //
-// Pipeline (all on the caller's stream, no host synchronisation):
-//   1. histogram of the four 8-bit digits of each fingerprint's upper 32
-//      bits (one pass);
-//   2. four stable LSD radix passes over (upper 32 fingerprint bits, row
-//      index), each a single kernel with decoupled look-back across tiles
-//      (bounded spins); stability keeps equal keys in ascending row order, so
-//      each run of equal keys starts with its smallest row index;
-//   3. segment heads: inclusive max-scan of "key differs from the previous
-//      one" positions;
-//   4. verify: every non-head row is compared in full (length + tokens) with
-//      its segment head by one warp; equal rows take the head as their
-//      representative, a mismatch marks the segment as collided.  A segment
-//      holds rows whose fingerprints agree in the upper 32 bits; rows that
-//      differ (in the lower bits, or in content under a true collision) are
-//      never merged, they only send the segment through step 5;
-//   5. collided segments only: exact regrouping by repeated peeling (the
-//      first unassigned row becomes a representative, all rows equal to it
-//      join it);
-//   6. exclusive sum-scan of "row is its own representative" gives each
-//      group its ordinal in first-occurrence order; the final kernel writes
-//      unique_idx and inverse.
+// The window's matching of a new node against the nodes already seen is a
+// lookup by signature; here it is a device hash table keyed by the 64-bit
+// fingerprint, whose value is the smallest row index carrying that key:
+//   1. insert: every row offers (fp, i); equal fingerprints within a warp are
+//      combined first, the slot keeps the minimum index (atomicMin);
+//   2. lookup + verify: rep[i] = the slot's index; a row with rep[i] != i is
+//      compared in full (length + tokens) with row rep[i] (two rows per warp
+//      round, 16 lanes each).  A mismatch — rows with equal fingerprints but
+//      different contents — sends the row to a collision list;
+//   3. collision list (empty unless fingerprints collide): exact regrouping
+//      by peeling — the smallest unassigned row becomes a representative and
+//      every listed row equal to it joins it;
+//   4. exclusive sum-scan of "row is its own representative" gives each
+//      group its ordinal in first-occurrence order (single pass, decoupled
+//      look-back with bounded spins); the final kernel writes unique_idx and
+//      inverse.
+// Up to kSmallRows rows, one launch does it all: every CTA builds the table
+// for all rows in its own shared memory (the same table in each), verifies
+// its share of the rows, and the last CTA to finish resolves the collision
+// list, scans and writes the outputs.
 #include <mutex>
 
 #include "hs_internal.cuh"
@@ -30,319 +29,105 @@
 namespace hs {
 namespace {
 
-constexpr int kSortThreads = 256;
-constexpr int kSortItems = 16;
-constexpr int kSortTile = kSortThreads * kSortItems;  // 4096 keys per tile
-constexpr int kPasses = 4;   // digits of bits 32..63 of the fingerprint
-constexpr int kLookBatch = 8;  // predecessor statuses read per round trip
-constexpr uint32_t kFlagA = 1u << 30;  // tile aggregate published
-constexpr uint32_t kFlagP = 2u << 30;  // inclusive prefix published
-constexpr uint32_t kValMask = (1u << 30) - 1u;
-
-constexpr int kScanThreads = 256;
+constexpr uint64_t kEmpty = ~0ull;      // free slot; fingerprint kEmpty has its own slot
+constexpr uint32_t kNoRow = 0xffffffffu;
+constexpr int kScanThreads = 1024;
 constexpr int kScanItems = 16;
 constexpr int kScanTile = kScanThreads * kScanItems;
+constexpr int kLookBatch = 8;           // predecessor statuses read per round trip
+constexpr int64_t kSmallRows = 4096;    // single-launch path
+constexpr int kSmallThreads = 512;
 
 constexpr size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
+constexpr int table_log2(int64_t n) {
+  int l = 6;
+  while ((int64_t(1) << l) < 2 * n) ++l;
+  return l;
+}
+
 struct Layout {
-  // zero-initialised region first
-  size_t hist, status, ctr, coll_flag, coll_count, scan_status0, scan_status1, zero_end;
-  size_t keys0, keys1, vals0, vals1, seg_head, rep, uid, coll_list, total;
+  int log2T;
+  // zero-initialised region first, then the region set to all-ones bytes
+  size_t ctr, scan_status, zero_end;
+  size_t keys, idx, ones_end;
+  size_t rep, uid, coll_list, total;
 };
+
+// Counters (uint32 each) in the zeroed region.
+constexpr int kCtrColl = 0;   // collision list length
+constexpr int kCtrScan = 1;   // scan tile ticket
+constexpr int kCtrDone = 2;   // CTAs finished (single-launch path)
 
 constexpr Layout layout(int64_t n) {
   Layout L{};
-  const int64_t sort_tiles = (n + kSortTile - 1) / kSortTile;
-  const int64_t scan_tiles = (n + kScanTile - 1) / kScanTile;
+  L.log2T = table_log2(n);
+  const size_t T1 = (size_t(1) << L.log2T) + 1;   // + the slot of fingerprint kEmpty
+  const int64_t tiles = (n + kScanTile - 1) / kScanTile;
   size_t o = 0;
-  L.hist = o;          o += align256(sizeof(uint32_t) * kPasses * 256);
-  L.status = o;        o += align256(sizeof(uint32_t) * kPasses * 256 * (size_t)sort_tiles);
-  L.ctr = o;           o += align256(sizeof(uint32_t) * 16);
-  L.coll_flag = o;     o += align256(sizeof(int32_t) * (size_t)n);
-  L.coll_count = o;    o += align256(sizeof(uint32_t));
-  L.scan_status0 = o;  o += align256(sizeof(uint64_t) * (size_t)scan_tiles);
-  L.scan_status1 = o;  o += align256(sizeof(uint64_t) * (size_t)scan_tiles);
+  L.ctr = o;          o += align256(sizeof(uint32_t) * 16);
+  L.scan_status = o;  o += align256(sizeof(uint64_t) * (size_t)tiles);
   L.zero_end = o;
-  L.keys0 = o;         o += align256(sizeof(uint32_t) * (size_t)n);
-  L.keys1 = o;         o += align256(sizeof(uint32_t) * (size_t)n);
-  L.vals0 = o;         o += align256(sizeof(uint32_t) * (size_t)n);
-  L.vals1 = o;         o += align256(sizeof(uint32_t) * (size_t)n);
-  L.seg_head = o;      o += align256(sizeof(int32_t) * (size_t)n);
-  L.rep = o;           o += align256(sizeof(int32_t) * (size_t)n);
-  L.uid = o;           o += align256(sizeof(int32_t) * (size_t)n);
-  L.coll_list = o;     o += align256(sizeof(int32_t) * (size_t)n);
+  L.keys = o;         o += align256(sizeof(uint64_t) * T1);
+  L.idx = o;          o += align256(sizeof(uint32_t) * T1);
+  L.ones_end = o;
+  L.rep = o;          o += align256(sizeof(int32_t) * (size_t)n);
+  L.uid = o;          o += align256(sizeof(int32_t) * (size_t)n);
+  L.coll_list = o;    o += align256(sizeof(int32_t) * (size_t)n);
   L.total = o;
   return L;
 }
 
-// Bounded spin on a 32-bit status word until its flag bits are non-zero.
-__device__ __forceinline__ uint32_t wait_flag32(const volatile uint32_t* p, unsigned* err) {
-  uint32_t s = *p;
-  if (s & ~kValMask) return s;
-  const uint64_t t0 = globaltimer_ns();
-  for (uint32_t it = 1;; ++it) {
-    s = *p;
-    if (s & ~kValMask) return s;
-    if ((it & 31u) == 0) {
-      __nanosleep(64);
-      if (globaltimer_ns() - t0 > kWaitLimitNs) {
-        set_error(err, kErrTimeout);
-        return kFlagP;  // give up: treat as a zero prefix
-      }
-    }
-  }
+// ---- hash table --------------------------------------------------------------------------
+// Open addressing with linear probing over 2^log2T slots (at least twice the
+// row count, so probes are short and a free slot always exists); the key
+// kEmpty marks a free slot, so the fingerprint kEmpty itself uses slot 2^log2T.
+__device__ __forceinline__ uint32_t home_slot(uint64_t f, int log2T) {
+  return (uint32_t)((f * 0x9E3779B97F4A7C15ull) >> (64 - log2T));
 }
 
-__device__ __forceinline__ uint64_t wait_flag64(const volatile unsigned long long* p,
-                                                unsigned* err) {
-  unsigned long long s = *p;
-  if (s >> 32) return s;
-  const uint64_t t0 = globaltimer_ns();
-  for (uint32_t it = 1;; ++it) {
-    s = *p;
-    if (s >> 32) return s;
-    if ((it & 31u) == 0) {
-      __nanosleep(64);
-      if (globaltimer_ns() - t0 > kWaitLimitNs) {
-        set_error(err, kErrTimeout);
-        return 2ull << 32;
-      }
+__device__ __forceinline__ uint32_t insert_key(uint64_t* keys, uint64_t f, int log2T) {
+  const uint32_t mask = (1u << log2T) - 1u;
+  if (f == kEmpty) return mask + 1u;
+  uint32_t s = home_slot(f, log2T);
+  for (uint32_t it = 0; it <= mask; ++it) {
+    uint64_t k = *reinterpret_cast<volatile uint64_t*>(keys + s);
+    if (k == kEmpty) {
+      k = atomicCAS(reinterpret_cast<unsigned long long*>(keys + s), (unsigned long long)kEmpty,
+                    (unsigned long long)f);
+      if (k == kEmpty) return s;
     }
+    if (k == f) return s;
+    s = (s + 1u) & mask;
   }
+  return mask + 1u;  // not reached: the table has more slots than rows
 }
 
-// ---- 1. digit histograms ---------------------------------------------------------------
-__global__ void __launch_bounds__(256) sort_hist_kernel(const uint64_t* __restrict__ fp, int64_t n,
-                                                        uint32_t* __restrict__ hist) {
-  __shared__ uint32_t h[kPasses * 256];
-  for (int i = threadIdx.x; i < kPasses * 256; i += blockDim.x) h[i] = 0;
-  __syncthreads();
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n;
-       e += (int64_t)gridDim.x * blockDim.x) {
-    const uint32_t k = (uint32_t)(__ldg(fp + e) >> 32);
-#pragma unroll
-    for (int p = 0; p < kPasses; ++p) atomicAdd(&h[p * 256 + ((k >> (8 * p)) & 0xff)], 1u);
+__device__ __forceinline__ uint32_t find_key(const uint64_t* keys, uint64_t f, int log2T) {
+  const uint32_t mask = (1u << log2T) - 1u;
+  if (f == kEmpty) return mask + 1u;
+  uint32_t s = home_slot(f, log2T);
+  for (uint32_t it = 0; it <= mask; ++it) {
+    const uint64_t k = keys[s];
+    if (k == f || k == kEmpty) return k == f ? s : mask + 1u;
+    s = (s + 1u) & mask;
   }
-  __syncthreads();
-  for (int i = threadIdx.x; i < kPasses * 256; i += blockDim.x)
-    if (h[i]) atomicAdd(&hist[i], h[i]);
+  return mask + 1u;
 }
 
-// ---- 2. one stable radix pass ----------------------------------------------------------------
-// Tile t holds keys [t*4096, (t+1)*4096); warp w of the tile owns the 512 keys
-// [w*512, (w+1)*512), read striped (item i of lane l is key w*512 + i*32 + l),
-// so processing items in order with lanes in order follows the input order.
-// Pass 0 reads the caller's 64-bit fingerprints (fp_in) and implicit row
-// indices; later passes read the previous pass's (key, value) arrays.
-__global__ void __launch_bounds__(kSortThreads) onesweep_kernel(
-    int pass, const uint64_t* __restrict__ fp_in, const uint32_t* __restrict__ keys_in,
-    const uint32_t* __restrict__ vals_in, uint32_t* __restrict__ keys_out,
-    uint32_t* __restrict__ vals_out, int64_t n,
-    const uint32_t* __restrict__ hist, uint32_t* status, uint32_t* tile_ctr, unsigned* err) {
-  __shared__ uint32_t s_tile;
-  __shared__ uint32_t warp_cnt[kSortThreads / 32][256];
-  __shared__ uint32_t digit_base[256];
-  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
-  if (tid == 0) s_tile = atomicAdd(tile_ctr + pass, 1u);
-  for (int i = tid; i < (kSortThreads / 32) * 256; i += kSortThreads) (&warp_cnt[0][0])[i] = 0;
-  // Exclusive scan of this pass's global digit counts (thread = digit).
-  {
-    const uint32_t c = hist[pass * 256 + tid];
-    uint32_t x = c;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const uint32_t y = __shfl_up_sync(0xffffffffu, x, o);
-      if (lane >= o) x += y;
-    }
-    __shared__ uint32_t wsum[8];
-    if (lane == 31) wsum[w] = x;
-    __syncthreads();
-    uint32_t add = 0;
-    for (int i = 0; i < w; ++i) add += wsum[i];
-    digit_base[tid] = add + x - c;
-  }
-  __syncthreads();
-  const uint32_t tile = s_tile;
-  const int64_t base = (int64_t)tile * kSortTile + w * (kSortItems * 32);
-  const int shift = 8 * pass;
-
-  uint32_t k[kSortItems];
-  uint32_t v[kSortItems];
-  uint32_t rank[kSortItems];
-#pragma unroll
-  for (int i = 0; i < kSortItems; ++i) {
-    const int64_t e = base + i * 32 + lane;
-    if (e < n) {
-      k[i] = fp_in ? (uint32_t)(fp_in[e] >> 32) : keys_in[e];
-      v[i] = fp_in ? (uint32_t)e : vals_in[e];
-    } else {
-      k[i] = 0;
-      v[i] = 0;
-    }
-  }
-#pragma unroll
-  for (int i = 0; i < kSortItems; ++i) {
-    const int64_t e = base + i * 32 + lane;
-    const bool valid = e < n;
-    const uint32_t d = valid ? (uint32_t)((k[i] >> shift) & 0xff) : 256u + lane;
-    const uint32_t peers = __match_any_sync(0xffffffffu, d);
-    const uint32_t before = valid ? warp_cnt[w][d] : 0u;
-    rank[i] = before + __popc(peers & lanemask_lt());
-    __syncwarp();
-    if (valid && (__ffs(peers) - 1) == lane) warp_cnt[w][d] = before + __popc(peers);
-    __syncwarp();
-  }
-  __syncthreads();
-  // Thread = digit: turn per-warp counts into per-warp exclusive offsets.
-  uint32_t tile_count = 0;
-#pragma unroll
-  for (int ww = 0; ww < kSortThreads / 32; ++ww) {
-    const uint32_t c = warp_cnt[ww][tid];
-    warp_cnt[ww][tid] = tile_count;
-    tile_count += c;
-  }
-  // Publish, look back, publish the inclusive prefix.
-  volatile uint32_t* st = status + (size_t)pass * 256 * gridDim.x;
-  uint32_t prefix = 0;
-  if (tile == 0) {
-    st[tid] = kFlagP | tile_count;
-  } else {
-    st[(size_t)tile * 256 + tid] = kFlagA | tile_count;
-    // Walk back kLookBatch predecessors per round trip; stop at the first
-    // inclusive prefix.
-    bool done = false;
-    for (int64_t j0 = (int64_t)tile - 1; j0 >= 0 && !done; j0 -= kLookBatch) {
-      uint32_t sv[kLookBatch];
-#pragma unroll
-      for (int b = 0; b < kLookBatch; ++b) sv[b] = j0 - b >= 0 ? st[(size_t)(j0 - b) * 256 + tid] : (2u << 30);
-#pragma unroll
-      for (int b = 0; b < kLookBatch; ++b) {
-        if (done) break;
-        uint32_t sb = sv[b];
-        if ((sb & ~kValMask) == 0) sb = wait_flag32(st + (size_t)(j0 - b) * 256 + tid, err);
-        if (j0 - b >= 0) prefix += sb & kValMask;
-        if ((sb & ~kValMask) == kFlagP) done = true;
-      }
-    }
-    st[(size_t)tile * 256 + tid] = kFlagP | ((prefix + tile_count) & kValMask);
-  }
-  digit_base[tid] += prefix;
-  __syncthreads();
-#pragma unroll
-  for (int i = 0; i < kSortItems; ++i) {
-    const int64_t e = base + i * 32 + lane;
-    if (e < n) {
-      const uint32_t d = (uint32_t)((k[i] >> shift) & 0xff);
-      const uint32_t pos = digit_base[d] + warp_cnt[w][d] + rank[i];
-      keys_out[pos] = k[i];
-      vals_out[pos] = v[i];
-    }
-  }
+// One warp-round of inserts: lane l offers (f, i) if valid.  Lanes with equal
+// fingerprints are combined; the lowest such lane (smallest index) inserts.
+__device__ __forceinline__ void insert_row(uint64_t* keys, uint32_t* idx, int log2T, bool valid,
+                                           uint64_t f, uint32_t i) {
+  const unsigned act = __ballot_sync(0xffffffffu, valid);
+  if (!valid) return;
+  const unsigned peers = __match_any_sync(act, f);
+  if ((int)(__ffs(peers) - 1) != (int)(threadIdx.x & 31)) return;
+  const uint32_t s = insert_key(keys, f, log2T);
+  if (*reinterpret_cast<volatile uint32_t*>(idx + s) > i) atomicMin(idx + s, i);
 }
 
-// ---- 3./6. single-pass scans with decoupled look-back ---------------------------------------
-struct HeadPos {  // value(p) = p if the sorted key changes at p, else 0
-  const uint32_t* keys;
-  __device__ int32_t operator()(int64_t p) const {
-    return (p == 0 || keys[p] != keys[p - 1]) ? (int32_t)p : 0;
-  }
-};
-struct IsRep {  // value(i) = 1 if row i represents its group
-  const int32_t* rep;
-  __device__ int32_t operator()(int64_t i) const { return rep[i] == (int32_t)i ? 1 : 0; }
-};
-struct OpMax {
-  __device__ int32_t operator()(int32_t a, int32_t b) const { return a > b ? a : b; }
-  static constexpr int32_t identity = 0;
-};
-struct OpSum {
-  __device__ int32_t operator()(int32_t a, int32_t b) const { return a + b; }
-  static constexpr int32_t identity = 0;
-};
-
-template <class Src, class Op, bool kExclusive>
-__global__ void __launch_bounds__(kScanThreads) scan_kernel(Src src, int64_t n, int32_t* out,
-                                                            unsigned long long* status,
-                                                            uint32_t* tile_ctr,
-                                                            int32_t* total_out, unsigned* err) {
-  __shared__ uint32_t s_tile;
-  __shared__ int32_t s_warp[kScanThreads / 32];
-  __shared__ int32_t s_prefix;
-  const Op op;
-  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
-  if (tid == 0) s_tile = atomicAdd(tile_ctr, 1u);
-  __syncthreads();
-  const uint32_t tile = s_tile;
-  const int64_t base = (int64_t)tile * kScanTile + (int64_t)tid * kScanItems;
-  int32_t x[kScanItems];
-  int32_t run = Op::identity;
-#pragma unroll
-  for (int i = 0; i < kScanItems; ++i) {
-    const int64_t e = base + i;
-    x[i] = e < n ? src(e) : Op::identity;
-    run = op(run, x[i]);
-  }
-  // Warp-level inclusive scan of thread totals.
-  int32_t incl = run;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const int32_t y = __shfl_up_sync(0xffffffffu, incl, o);
-    if (lane >= o) incl = op(y, incl);
-  }
-  if (lane == 31) s_warp[w] = incl;
-  __syncthreads();
-  int32_t warp_prefix = Op::identity, tile_total = Op::identity;
-  for (int i = 0; i < kScanThreads / 32; ++i) {
-    if (i < w) warp_prefix = op(warp_prefix, s_warp[i]);
-    tile_total = op(tile_total, s_warp[i]);
-  }
-  int32_t thread_prefix = __shfl_up_sync(0xffffffffu, incl, 1);
-  if (lane == 0) thread_prefix = Op::identity;
-  thread_prefix = op(warp_prefix, thread_prefix);
-  if (tid == 0) {
-    volatile unsigned long long* st = status;
-    int32_t prefix = Op::identity;
-    if (tile == 0) {
-      st[0] = (2ull << 32) | (uint32_t)tile_total;
-    } else {
-      st[tile] = (1ull << 32) | (uint32_t)tile_total;
-      bool done = false;
-      for (int64_t j0 = (int64_t)tile - 1; j0 >= 0 && !done; j0 -= kLookBatch) {
-        unsigned long long sv[kLookBatch];
-#pragma unroll
-        for (int b = 0; b < kLookBatch; ++b) sv[b] = j0 - b >= 0 ? st[j0 - b] : (2ull << 32);
-#pragma unroll
-        for (int b = 0; b < kLookBatch; ++b) {
-          if (done) break;
-          unsigned long long sb = sv[b];
-          if ((sb >> 32) == 0) sb = wait_flag64(st + (j0 - b), err);
-          if (j0 - b >= 0) prefix = op((int32_t)(uint32_t)sb, prefix);
-          if ((sb >> 32) == 2ull) done = true;
-        }
-      }
-      st[tile] = (2ull << 32) | (uint32_t)op(prefix, tile_total);
-    }
-    s_prefix = prefix;
-    const int64_t tiles = (n + kScanTile - 1) / kScanTile;
-    if (total_out && (int64_t)tile == tiles - 1) *total_out = op(prefix, tile_total);
-  }
-  __syncthreads();
-  int32_t acc = op(s_prefix, thread_prefix);
-#pragma unroll
-  for (int i = 0; i < kScanItems; ++i) {
-    const int64_t e = base + i;
-    if (kExclusive) {
-      if (e < n) out[e] = acc;
-      acc = op(acc, x[i]);
-    } else {
-      acc = op(acc, x[i]);
-      if (e < n) out[e] = acc;
-    }
-  }
-}
-
-// ---- 4./5. full-row comparison -------------------------------------------------------------------
+// ---- row comparison ---------------------------------------------------------------------------
 __device__ __forceinline__ int32_t clamp_len(const int32_t* lens, int64_t r, int32_t stride,
                                              unsigned* err) {
   int32_t L = lens ? __ldg(lens + r) : stride;
@@ -353,52 +138,8 @@ __device__ __forceinline__ int32_t clamp_len(const int32_t* lens, int64_t r, int
   return L;
 }
 
-// Whole warp: are rows a and b equal (same length, same tokens below it)?
-template <bool VEC>
-__device__ bool rows_equal_warp(const int32_t* __restrict__ tokens, int32_t stride,
-                                const int32_t* __restrict__ lens, int64_t a, int64_t b,
-                                unsigned* err) {
-  const int lane = threadIdx.x & 31;
-  const int32_t la = clamp_len(lens, a, stride, err);
-  const int32_t lb = clamp_len(lens, b, stride, err);
-  if (la != lb) return false;
-  const int32_t* ra = tokens + a * (int64_t)stride;
-  const int32_t* rb = tokens + b * (int64_t)stride;
-  bool diff = false;
-  int32_t done = 0;
-  if (VEC) {
-    // Up to three 16-byte pieces of each row per lane in flight per round
-    // trip: a 384-token row is compared in one round trip.
-    const int32_t pieces = la >> 2;
-    const int4* pa = reinterpret_cast<const int4*>(ra);
-    const int4* pb = reinterpret_cast<const int4*>(rb);
-    for (int32_t j0 = 0; j0 < pieces; j0 += 96) {
-      int4 x[3], y[3];
-#pragma unroll
-      for (int u = 0; u < 3; ++u) {
-        const int32_t j = j0 + u * 32 + lane;
-        if (j < pieces) {
-          x[u] = __ldg(pa + j);
-          y[u] = __ldg(pb + j);
-        }
-      }
-#pragma unroll
-      for (int u = 0; u < 3; ++u) {
-        const int32_t j = j0 + u * 32 + lane;
-        if (j < pieces)
-          diff |= (x[u].x != y[u].x) | (x[u].y != y[u].y) | (x[u].z != y[u].z) | (x[u].w != y[u].w);
-      }
-    }
-    done = pieces << 2;
-  }
-  for (int32_t t = done + lane; t < la; t += 32) diff |= (__ldg(ra + t) != __ldg(rb + t));
-  return !__any_sync(0xffffffffu, diff);
-}
-
-// Verify: lane i of a warp loads the metadata of position p0+i (segment head,
-// row index, head row, both lengths) so the dependent lookups of 32 positions
-// share their round trips; then the two half-warps compare two pairs of rows
-// at a time, 16 lanes x up to 6 pieces of each row in flight.
+// Half-warp: do rows a and b differ in their first len tokens?  16 lanes, up
+// to six 16-byte pieces of each row per lane in flight per round trip.
 template <bool VEC>
 __device__ __forceinline__ bool half_rows_differ(const int32_t* __restrict__ tokens,
                                                  int32_t stride, int64_t a, int64_t b, int32_t len,
@@ -434,106 +175,265 @@ __device__ __forceinline__ bool half_rows_differ(const int32_t* __restrict__ tok
   return diff;
 }
 
+// Whole warp: lane l holds a pair (a, b) with `need` set if the rows must be
+// compared (their lengths, la, are equal).  Pairs are compared two at a time
+// (one per half-warp).  Returns, to each lane, whether its pair differs.
+template <bool VEC>
+__device__ __forceinline__ bool warp_pairs_differ(const int32_t* __restrict__ tokens,
+                                                  int32_t stride, bool need, int64_t a, int64_t b,
+                                                  int32_t la) {
+  const int lane = threadIdx.x & 31, half = lane >> 4, hl = lane & 15;
+  unsigned todo = __ballot_sync(0xffffffffu, need);
+  unsigned differ = 0u;
+  while (todo != 0u) {
+    const int j0 = __ffs(todo) - 1;
+    todo &= todo - 1;
+    int j1 = -1;
+    if (todo != 0u) {
+      j1 = __ffs(todo) - 1;
+      todo &= todo - 1;
+    }
+    const int j = half == 0 ? j0 : j1;
+    const int src = j < 0 ? 0 : j;
+    const int64_t aj = __shfl_sync(0xffffffffu, a, src);
+    const int64_t bj = __shfl_sync(0xffffffffu, b, src);
+    const int32_t lj = __shfl_sync(0xffffffffu, la, src);
+    const bool diff = j >= 0 && half_rows_differ<VEC>(tokens, stride, aj, bj, lj, hl);
+    const unsigned dm = __ballot_sync(0xffffffffu, diff);
+    if ((dm & 0xffffu) != 0u) differ |= 1u << j0;
+    if (j1 >= 0 && (dm >> 16) != 0u) differ |= 1u << j1;
+  }
+  return (differ >> lane) & 1u;
+}
+
+// Whole warp: are rows a and b equal (same length, same tokens below it)?
+template <bool VEC>
+__device__ bool rows_equal_warp(const int32_t* __restrict__ tokens, int32_t stride,
+                                const int32_t* __restrict__ lens, int64_t a, int64_t b,
+                                unsigned* err) {
+  const int lane = threadIdx.x & 31;
+  const int32_t la = clamp_len(lens, a, stride, err);
+  const int32_t lb = clamp_len(lens, b, stride, err);
+  if (la != lb) return false;
+  const int32_t* ra = tokens + a * (int64_t)stride;
+  const int32_t* rb = tokens + b * (int64_t)stride;
+  bool diff = false;
+  int32_t done = 0;
+  if (VEC) {
+    const int32_t pieces = la >> 2;
+    const int4* pa = reinterpret_cast<const int4*>(ra);
+    const int4* pb = reinterpret_cast<const int4*>(rb);
+    for (int32_t j = lane; j < pieces; j += 32) {
+      const int4 x = __ldg(pa + j), y = __ldg(pb + j);
+      diff |= (x.x != y.x) | (x.y != y.y) | (x.z != y.z) | (x.w != y.w);
+    }
+    done = pieces << 2;
+  }
+  for (int32_t t = done + lane; t < la; t += 32) diff |= (__ldg(ra + t) != __ldg(rb + t));
+  return !__any_sync(0xffffffffu, diff);
+}
+
+// Verify the 32 rows [p0, p0+32) of one warp against their tentative
+// representatives r (lane = row).  Returns, per lane, whether the row stays
+// merged with r (true for a row that is its own representative).
+template <bool VEC>
+__device__ __forceinline__ bool verify_warp(const int32_t* __restrict__ tokens, int32_t stride,
+                                            const int32_t* __restrict__ lens, bool valid,
+                                            int64_t a, int64_t r, unsigned* err) {
+  const bool self = !valid || r == a;
+  const int32_t la = valid ? clamp_len(lens, a, stride, err) : 0;
+  const int32_t lr = self ? la : clamp_len(lens, r, stride, err);
+  const bool need = !self && la == lr;
+  const bool differ = warp_pairs_differ<VEC>(tokens, stride, need, a, r, la);
+  return self || (need && !differ);
+}
+
+// Exact regrouping of the listed rows (rep == -1) by peeling; one block.
+// Listed rows differ from the representative of their fingerprint, so they
+// can only equal each other; the smallest unassigned row of each content
+// becomes its representative.  rep may be in shared or global memory.
+template <bool VEC>
+__device__ void peel_block(const uint64_t* __restrict__ fp, const int32_t* __restrict__ tokens,
+                           int32_t stride, const int32_t* __restrict__ lens, int32_t* rep,
+                           const int32_t* coll_list, uint32_t m, unsigned* err) {
+  __shared__ int32_t s_first;
+  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5, nw = blockDim.x >> 5;
+  for (;;) {
+    if (tid == 0) s_first = 0x7fffffff;
+    __syncthreads();
+    int32_t mine = 0x7fffffff;
+    for (uint32_t c = tid; c < m; c += blockDim.x) {
+      const int32_t a = coll_list[c];
+      if (*reinterpret_cast<volatile int32_t*>(rep + a) == -1 && a < mine) mine = a;
+    }
+    if (mine != 0x7fffffff) atomicMin(&s_first, mine);
+    __syncthreads();
+    const int32_t a0 = s_first;
+    if (a0 == 0x7fffffff) break;
+    const uint64_t f0 = fp[a0];
+    for (uint32_t c = w; c < m; c += nw) {
+      const int32_t b = coll_list[c];
+      if (b == a0 || *reinterpret_cast<volatile int32_t*>(rep + b) != -1 || fp[b] != f0) continue;
+      if (rows_equal_warp<VEC>(tokens, stride, lens, a0, b, err) && lane == 0) rep[b] = a0;
+    }
+    __syncthreads();
+    if (tid == 0) rep[a0] = a0;
+    __syncthreads();
+  }
+}
+
+// ---- multi-kernel path ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) insert_kernel(const uint64_t* __restrict__ fp, int64_t n,
+                                                     uint64_t* keys, uint32_t* idx, int log2T) {
+  for (int64_t base = (int64_t)blockIdx.x * blockDim.x; base < n;
+       base += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t i = base + threadIdx.x;
+    const bool valid = i < n;
+    insert_row(keys, idx, log2T, valid, valid ? __ldg(fp + i) : 0ull, (uint32_t)i);
+  }
+}
+
 template <bool VEC>
 __global__ void __launch_bounds__(256) verify_kernel(
-    const uint32_t* __restrict__ vals, const int32_t* __restrict__ seg_head, int64_t n,
-    const int32_t* __restrict__ tokens, int32_t stride, const int32_t* __restrict__ lens,
-    int32_t* __restrict__ rep, int32_t* coll_flag, int32_t* coll_list, uint32_t* coll_count,
-    unsigned* err) {
-  const int lane = threadIdx.x & 31, half = lane >> 4, hl = lane & 15;
+    const uint64_t* __restrict__ fp, int64_t n, const uint64_t* __restrict__ keys,
+    const uint32_t* __restrict__ idx, int log2T, const int32_t* __restrict__ tokens,
+    int32_t stride, const int32_t* __restrict__ lens, int32_t* __restrict__ rep,
+    int32_t* coll_list, uint32_t* ctr, unsigned* err) {
+  const int lane = threadIdx.x & 31;
   const int64_t warps = ((int64_t)gridDim.x * blockDim.x) >> 5;
   const int64_t w = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   for (int64_t p0 = w * 32; p0 < n; p0 += warps * 32) {
-    const int64_t p = p0 + lane;
-    const bool valid = p < n;
-    const int32_t h = valid ? seg_head[p] : 0;
-    const bool head = valid && h == (int32_t)p;
-    const int64_t a = valid ? (int64_t)vals[p] : 0;
-    const int64_t b = (valid && !head) ? (int64_t)vals[h] : a;
-    const int32_t la = valid ? clamp_len(lens, a, stride, err) : 0;
-    const int32_t lb = (valid && !head) ? clamp_len(lens, b, stride, err) : la;
-    bool need = valid && !head;
-    if (head) rep[a] = (int32_t)a;
-    if (need && la != lb) {               // different lengths: never equal
-      rep[a] = (int32_t)a;
-      if (atomicCAS(coll_flag + h, 0, 1) == 0) coll_list[atomicAdd(coll_count, 1u)] = h;
-      need = false;
+    const int64_t a = p0 + lane;
+    const bool valid = a < n;
+    int64_t r = a;
+    if (valid) {
+      const uint32_t v = idx[find_key(keys, __ldg(fp + a), log2T)];
+      if (v < (uint32_t)n) r = v;
+      else set_error(err, kErrInvalidArg);   // not reached: every row was inserted
     }
-    unsigned todo = __ballot_sync(0xffffffffu, need);
-    while (todo != 0u) {
-      const int j0 = __ffs(todo) - 1;
-      todo &= todo - 1;
-      int j1 = -1;
-      if (todo != 0u) {
-        j1 = __ffs(todo) - 1;
-        todo &= todo - 1;
-      }
-      const int j = half == 0 ? j0 : j1;
-      const int src = j < 0 ? 0 : j;
-      const int64_t aj = __shfl_sync(0xffffffffu, a, src);
-      const int64_t bj = __shfl_sync(0xffffffffu, b, src);
-      const int32_t lj = __shfl_sync(0xffffffffu, la, src);
-      const int32_t hj = __shfl_sync(0xffffffffu, h, src);
-      const bool diff = j >= 0 && half_rows_differ<VEC>(tokens, stride, aj, bj, lj, hl);
-      const unsigned dm = __ballot_sync(0xffffffffu, diff);
-      const bool eq = ((dm >> (half * 16)) & 0xffffu) == 0u;
-      if (j >= 0 && hl == 0) {
-        rep[aj] = eq ? (int32_t)bj : (int32_t)aj;
-        if (!eq && atomicCAS(coll_flag + hj, 0, 1) == 0) coll_list[atomicAdd(coll_count, 1u)] = hj;
+    const bool merged = verify_warp<VEC>(tokens, stride, lens, valid, a, r, err);
+    if (valid) {
+      rep[a] = merged ? (int32_t)r : -1;
+      if (!merged) coll_list[atomicAdd(ctr + kCtrColl, 1u)] = (int32_t)a;
+    }
+  }
+}
+
+template <bool VEC>
+__global__ void __launch_bounds__(1024) resolve_kernel(const uint64_t* __restrict__ fp,
+                                                       const int32_t* __restrict__ tokens,
+                                                       int32_t stride,
+                                                       const int32_t* __restrict__ lens,
+                                                       int32_t* rep, const int32_t* coll_list,
+                                                       const uint32_t* ctr, unsigned* err) {
+  const uint32_t m = ctr[kCtrColl];
+  if (m == 0) return;
+  peel_block<VEC>(fp, tokens, stride, lens, rep, coll_list, m, err);
+}
+
+// Single-pass exclusive sum-scan of "rep[i] == i" with decoupled look-back;
+// the last tile writes the total (the group count).
+__device__ __forceinline__ uint64_t wait_status(const volatile unsigned long long* p,
+                                                unsigned* err) {
+  unsigned long long s = *p;
+  if (s >> 32) return s;
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t it = 1;; ++it) {
+    s = *p;
+    if (s >> 32) return s;
+    if ((it & 31u) == 0) {
+      __nanosleep(64);
+      if (globaltimer_ns() - t0 > kWaitLimitNs) {
+        set_error(err, kErrTimeout);
+        return 2ull << 32;  // give up: treat as a zero prefix
       }
     }
   }
 }
 
-// Regroup the rows of each collided segment exactly.  Within a segment,
-// positions are in ascending row order (stable sort), so the first
-// unassigned position is the smallest unassigned row index.
-template <bool VEC>
-__global__ void __launch_bounds__(256) resolve_kernel(
-    const uint32_t* __restrict__ vals, const int32_t* __restrict__ seg_head, int64_t n,
-    const int32_t* __restrict__ tokens, int32_t stride, const int32_t* __restrict__ lens,
-    int32_t* rep, const int32_t* __restrict__ coll_list, const uint32_t* coll_count,
-    unsigned* err) {
-  __shared__ int64_t s_end;
-  __shared__ int32_t s_first;
-  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5, nw = blockDim.x >> 5;
-  const uint32_t count = *coll_count;
-  for (uint32_t c = blockIdx.x; c < count; c += gridDim.x) {
-    const int32_t h = coll_list[c];
-    if (tid == 0) s_end = n;
-    __syncthreads();
-    for (int64_t p = (int64_t)h + 1 + tid; p < n; p += blockDim.x) {
-      if (p >= s_end) break;
-      if (seg_head[p] != h) {
-        atomicMin(reinterpret_cast<unsigned long long*>(&s_end), (unsigned long long)p);
-        break;
-      }
+__global__ void __launch_bounds__(kScanThreads) scan_kernel(const int32_t* __restrict__ rep,
+                                                            int64_t n, int32_t* __restrict__ uid,
+                                                            unsigned long long* status,
+                                                            uint32_t* ctr, int32_t* total_out,
+                                                            unsigned* err) {
+  __shared__ uint32_t s_tile;
+  __shared__ int32_t s_warp[kScanThreads / 32];
+  __shared__ int32_t s_prefix;
+  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+  if (tid == 0) s_tile = atomicAdd(ctr + kCtrScan, 1u);
+  __syncthreads();
+  const uint32_t tile = s_tile;
+  const int64_t base = (int64_t)tile * kScanTile + (int64_t)tid * kScanItems;
+  int32_t x[kScanItems];
+  int32_t run = 0;
+#pragma unroll
+  for (int i = 0; i < kScanItems; i += 4) {
+    const int64_t e = base + i;
+    if (e + 3 < n) {
+      const int4 v = *reinterpret_cast<const int4*>(rep + e);
+      x[i] = v.x == (int32_t)e;
+      x[i + 1] = v.y == (int32_t)(e + 1);
+      x[i + 2] = v.z == (int32_t)(e + 2);
+      x[i + 3] = v.w == (int32_t)(e + 3);
+    } else {
+#pragma unroll
+      for (int j = 0; j < 4; ++j) x[i + j] = (e + j < n) ? (rep[e + j] == (int32_t)(e + j)) : 0;
     }
-    __syncthreads();
-    const int64_t end = s_end;
-    for (int64_t p = (int64_t)h + tid; p < end; p += blockDim.x) rep[vals[p]] = -1;
-    __syncthreads();
-    for (;;) {
-      if (tid == 0) s_first = 0x7fffffff;
-      __syncthreads();
-      for (int64_t p = (int64_t)h + tid; p < end; p += blockDim.x)
-        if (rep[vals[p]] == -1) {
-          atomicMin(&s_first, (int32_t)(p - h));
-          break;
+    run += x[i] + x[i + 1] + x[i + 2] + x[i + 3];
+  }
+  int32_t incl = run;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += y;
+  }
+  if (lane == 31) s_warp[w] = incl;
+  __syncthreads();
+  if (w == 0) {
+    const int32_t v = s_warp[lane];
+    int32_t iv = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int32_t y = __shfl_up_sync(0xffffffffu, iv, o);
+      if (lane >= o) iv += y;
+    }
+    s_warp[lane] = iv - v;  // exclusive warp offsets
+    if (lane == 31) {
+      const int32_t tile_total = iv;
+      volatile unsigned long long* st = status;
+      int32_t prefix = 0;
+      if (tile == 0) {
+        st[0] = (2ull << 32) | (uint32_t)tile_total;
+      } else {
+        st[tile] = (1ull << 32) | (uint32_t)tile_total;
+        bool done = false;
+        for (int64_t j0 = (int64_t)tile - 1; j0 >= 0 && !done; j0 -= kLookBatch) {
+          unsigned long long sv[kLookBatch];
+#pragma unroll
+          for (int b = 0; b < kLookBatch; ++b) sv[b] = j0 - b >= 0 ? st[j0 - b] : (2ull << 32);
+#pragma unroll
+          for (int b = 0; b < kLookBatch; ++b) {
+            if (done) break;
+            unsigned long long sb = sv[b];
+            if ((sb >> 32) == 0) sb = wait_status(st + (j0 - b), err);
+            if (j0 - b >= 0) prefix += (int32_t)(uint32_t)sb;
+            if ((sb >> 32) == 2ull) done = true;
+          }
         }
-      __syncthreads();
-      const int32_t first = s_first;
-      if (first == 0x7fffffff) break;
-      const int64_t r = vals[h + first];
-      for (int64_t p = (int64_t)h + first + w; p < end; p += nw) {
-        const int64_t a = vals[p];
-        const int32_t cur = __shfl_sync(0xffffffffu, lane == 0 ? rep[a] : 0, 0);
-        if (cur != -1) continue;
-        const bool eq = (a == r) || rows_equal_warp<VEC>(tokens, stride, lens, a, r, err);
-        if (eq && lane == 0) rep[a] = (int32_t)r;
+        st[tile] = (2ull << 32) | (uint32_t)(prefix + tile_total);
       }
-      __syncthreads();
+      s_prefix = prefix;
+      const int64_t tiles = (n + kScanTile - 1) / kScanTile;
+      if ((int64_t)tile == tiles - 1) *total_out = prefix + tile_total;
     }
+  }
+  __syncthreads();
+  int32_t acc = s_prefix + s_warp[w] + incl - run;
+#pragma unroll
+  for (int i = 0; i < kScanItems; ++i) {
+    const int64_t e = base + i;
+    if (e < n) uid[e] = acc;
+    acc += x[i];
   }
 }
 
@@ -552,11 +452,132 @@ __global__ void __launch_bounds__(256) finalize_kernel(const int32_t* __restrict
   }
 }
 
+// ---- single-launch path (n <= kSmallRows) ----------------------------------------------------
+// Dynamic shared memory: keys[T + 1], idx[T + 1], rep[n], uid[n] (T = 2^log2T).
+constexpr size_t small_smem(int64_t n) {
+  const size_t T1 = (size_t(1) << table_log2(n)) + 1;
+  return T1 * 8 + T1 * 4 + (size_t)n * 8 + 16;
+}
+
+template <bool VEC>
+__global__ void __launch_bounds__(kSmallThreads) unique_small_kernel(
+    const uint64_t* __restrict__ fp, int64_t n, const int32_t* __restrict__ tokens,
+    int32_t stride, const int32_t* __restrict__ lens, int32_t* __restrict__ n_unique,
+    int32_t* __restrict__ unique_idx, int32_t* __restrict__ inverse, uint32_t* ctr,
+    int32_t* coll_list, unsigned* err) {
+  extern __shared__ __align__(16) uint8_t sm[];
+  __shared__ bool s_last;
+  __shared__ int32_t s_warp[kSmallThreads / 32];
+  const int log2T = table_log2(n);
+  const uint32_t T1 = (1u << log2T) + 1u;
+  uint64_t* keys = reinterpret_cast<uint64_t*>(sm);
+  uint32_t* idx = reinterpret_cast<uint32_t*>(keys + T1);
+  int32_t* rep = reinterpret_cast<int32_t*>(idx + T1);
+  int32_t* uid = rep + n;
+  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+  constexpr int kWarps = kSmallThreads / 32;
+
+  // 1. the table for all rows (the same in every CTA)
+  for (uint32_t s = tid; s < T1; s += kSmallThreads) {
+    keys[s] = kEmpty;
+    idx[s] = kNoRow;
+  }
+  __syncthreads();
+  for (int64_t base = 0; base < n; base += kSmallThreads) {
+    const int64_t i = base + tid;
+    const bool valid = i < n;
+    insert_row(keys, idx, log2T, valid, valid ? __ldg(fp + i) : 0ull, (uint32_t)i);
+  }
+  __syncthreads();
+  for (int64_t i = tid; i < n; i += kSmallThreads) {
+    const uint32_t v = idx[find_key(keys, __ldg(fp + i), log2T)];
+    rep[i] = v < (uint32_t)n ? (int32_t)v : (int32_t)i;
+  }
+  __syncthreads();
+
+  // 2. verify this CTA's rows: warp-rounds of 32 rows, dealt round-robin
+  //    over the CTAs first, so every CTA gets a share
+  const int64_t rounds = (n + 31) / 32;
+  for (int64_t rd = (int64_t)w * gridDim.x + blockIdx.x; rd < rounds;
+       rd += (int64_t)gridDim.x * kWarps) {
+    const int64_t a = rd * 32 + lane;
+    const bool valid = a < n;
+    const int64_t r = valid ? rep[a] : a;
+    const bool merged = verify_warp<VEC>(tokens, stride, lens, valid, a, r, err);
+    if (valid && !merged) coll_list[atomicAdd(ctr + kCtrColl, 1u)] = (int32_t)a;
+  }
+
+  // 3. the last CTA to finish writes the outputs
+  __threadfence();
+  __syncthreads();
+  if (tid == 0) s_last = atomicAdd(ctr + kCtrDone, 1u) == gridDim.x - 1;
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  const uint32_t m = *reinterpret_cast<volatile uint32_t*>(ctr + kCtrColl);
+  for (uint32_t c = tid; c < m; c += kSmallThreads) rep[coll_list[c]] = -1;
+  __syncthreads();
+  if (m) peel_block<VEC>(fp, tokens, stride, lens, rep, coll_list, m, err);
+  __syncthreads();
+  // exclusive scan of rep[i] == i: contiguous items per thread
+  const int64_t per = (n + kSmallThreads - 1) / kSmallThreads;
+  const int64_t b0 = tid * per, b1 = min(n, b0 + per);
+  int32_t run = 0;
+  for (int64_t i = b0; i < b1; ++i) run += rep[i] == (int32_t)i;
+  int32_t incl = run;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += y;
+  }
+  if (lane == 31) s_warp[w] = incl;
+  __syncthreads();
+  int32_t off = 0, total = 0;
+  for (int i = 0; i < kWarps; ++i) {
+    off += i < w ? s_warp[i] : 0;
+    total += s_warp[i];
+  }
+  int32_t acc = off + incl - run;
+  for (int64_t i = b0; i < b1; ++i) {
+    uid[i] = acc;
+    acc += rep[i] == (int32_t)i;
+  }
+  __syncthreads();
+  for (int64_t i = tid; i < n; i += kSmallThreads) {
+    const int32_t r = rep[i];
+    inverse[i] = uid[r];
+    if (r == (int32_t)i) unique_idx[uid[i]] = (int32_t)i;
+  }
+  for (int64_t i = total + tid; i < n; i += kSmallThreads) unique_idx[i] = 0;
+  if (tid == 0) *n_unique = total;
+}
+
 unsigned grid_for(int64_t items, int per_block, int max_blocks) {
   int64_t b = (items + per_block - 1) / per_block;
   if (b < 1) b = 1;
   if (b > max_blocks) b = max_blocks;
   return (unsigned)b;
+}
+
+template <bool VEC>
+hs_status launch_small(const uint64_t* fp, const int32_t* tokens, int64_t n, int32_t stride,
+                       const int32_t* lens, int32_t* n_unique, int32_t* unique_idx,
+                       int32_t* inverse, uint32_t* ctr, int32_t* coll_list, unsigned* err,
+                       cudaStream_t stream) {
+  const size_t smem = small_smem(n);
+  static size_t configured = 0;
+  if (smem > 48 * 1024 && smem > configured) {
+    const cudaError_t e = cudaFuncSetAttribute(unique_small_kernel<VEC>,
+                                               cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               (int)small_smem(kSmallRows));
+    if (e != cudaSuccess) return cuda_fail(e, "unique smem attribute");
+    configured = small_smem(kSmallRows);
+  }
+  // One CTA per 2 warp-rounds of rows (they wait on memory), at most one per SM.
+  const unsigned grid = grid_for((n + 31) / 32, 2, num_sms());
+  unique_small_kernel<VEC><<<grid, kSmallThreads, smem, stream>>>(
+      fp, n, tokens, stride, lens, n_unique, unique_idx, inverse, ctr, coll_list, err);
+  return HS_OK;
 }
 
 }  // namespace
@@ -571,66 +592,50 @@ hs_status launch_unique_inverse(const uint64_t* fp, const int32_t* tokens, int64
   if (!err) return fail(HS_ERR_CUDA, "could not resolve the device error word");
   const Layout L = layout(n);
   char* w = static_cast<char*>(ws);
-  uint32_t* hist = reinterpret_cast<uint32_t*>(w + L.hist);
-  uint32_t* status = reinterpret_cast<uint32_t*>(w + L.status);
   uint32_t* ctr = reinterpret_cast<uint32_t*>(w + L.ctr);
-  int32_t* coll_flag = reinterpret_cast<int32_t*>(w + L.coll_flag);
-  uint32_t* coll_count = reinterpret_cast<uint32_t*>(w + L.coll_count);
-  auto* scan0 = reinterpret_cast<unsigned long long*>(w + L.scan_status0);
-  auto* scan1 = reinterpret_cast<unsigned long long*>(w + L.scan_status1);
-  uint32_t* keys[2] = {reinterpret_cast<uint32_t*>(w + L.keys0),
-                       reinterpret_cast<uint32_t*>(w + L.keys1)};
-  uint32_t* vals[2] = {reinterpret_cast<uint32_t*>(w + L.vals0),
-                       reinterpret_cast<uint32_t*>(w + L.vals1)};
-  int32_t* seg_head = reinterpret_cast<int32_t*>(w + L.seg_head);
+  auto* status = reinterpret_cast<unsigned long long*>(w + L.scan_status);
+  uint64_t* keys = reinterpret_cast<uint64_t*>(w + L.keys);
+  uint32_t* idx = reinterpret_cast<uint32_t*>(w + L.idx);
   int32_t* rep = reinterpret_cast<int32_t*>(w + L.rep);
   int32_t* uid = reinterpret_cast<int32_t*>(w + L.uid);
   int32_t* coll_list = reinterpret_cast<int32_t*>(w + L.coll_list);
+  const bool vec = ((reinterpret_cast<uintptr_t>(tokens) & 15u) == 0) && (stride % 4 == 0);
+  const int sms = num_sms();
 
   cudaError_t e = cudaMemsetAsync(w, 0, L.zero_end, stream);
   if (e != cudaSuccess) return cuda_fail(e, "workspace clear");
-  const int sms = num_sms();
-  const int64_t sort_tiles = (n + kSortTile - 1) / kSortTile;
-  const int64_t scan_tiles = (n + kScanTile - 1) / kScanTile;
-
-  sort_hist_kernel<<<grid_for(n, 256 * 8, sms * 4), 256, 0, stream>>>(fp, n, hist);
-  // Four passes; pass 0 reads the caller's fingerprints and implicit indices.
-  const uint32_t* kin = nullptr;
-  const uint32_t* vin = nullptr;
-  int out = 0;
-  for (int pass = 0; pass < kPasses; ++pass) {
-    onesweep_kernel<<<(unsigned)sort_tiles, kSortThreads, 0, stream>>>(
-        pass, pass == 0 ? fp : nullptr, kin, vin, keys[out], vals[out], n, hist, status, ctr, err);
-    kin = keys[out];
-    vin = vals[out];
-    out ^= 1;
+  if (n <= kSmallRows) {
+    const hs_status st =
+        vec ? launch_small<true>(fp, tokens, n, stride, lens, n_unique_dev, unique_idx, inverse,
+                                 ctr, coll_list, err, stream)
+            : launch_small<false>(fp, tokens, n, stride, lens, n_unique_dev, unique_idx, inverse,
+                                  ctr, coll_list, err, stream);
+    if (st != HS_OK) return st;
+    count_launches(1);
+    return cuda_fail(cudaGetLastError(), "unique_inverse launch");
   }
-  const uint32_t* skeys = kin;
-  const uint32_t* svals = vin;
-
-  scan_kernel<HeadPos, OpMax, false><<<(unsigned)scan_tiles, kScanThreads, 0, stream>>>(
-      HeadPos{skeys}, n, seg_head, scan0, ctr + 8, nullptr, err);
-
-  const bool vec = ((reinterpret_cast<uintptr_t>(tokens) & 15u) == 0) && (stride % 4 == 0);
-  const unsigned vgrid = grid_for(n, 256, sms * 8);   // one warp per 32 positions
+  e = cudaMemsetAsync(w + L.zero_end, 0xff, L.ones_end - L.zero_end, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "hash table clear");
+  insert_kernel<<<grid_for(n, 256, sms * 8), 256, 0, stream>>>(fp, n, keys, idx, L.log2T);
+  const unsigned vgrid = grid_for(n, 256, sms * 8);   // one warp per 32 rows
   if (vec)
-    verify_kernel<true><<<vgrid, 256, 0, stream>>>(svals, seg_head, n, tokens, stride, lens, rep,
-                                                   coll_flag, coll_list, coll_count, err);
+    verify_kernel<true><<<vgrid, 256, 0, stream>>>(fp, n, keys, idx, L.log2T, tokens, stride,
+                                                   lens, rep, coll_list, ctr, err);
   else
-    verify_kernel<false><<<vgrid, 256, 0, stream>>>(svals, seg_head, n, tokens, stride, lens,
-                                                    rep, coll_flag, coll_list, coll_count, err);
+    verify_kernel<false><<<vgrid, 256, 0, stream>>>(fp, n, keys, idx, L.log2T, tokens, stride,
+                                                    lens, rep, coll_list, ctr, err);
   if (vec)
-    resolve_kernel<true><<<(unsigned)sms, 256, 0, stream>>>(svals, seg_head, n, tokens, stride,
-                                                            lens, rep, coll_list, coll_count, err);
+    resolve_kernel<true><<<1, 1024, 0, stream>>>(fp, tokens, stride, lens, rep, coll_list, ctr,
+                                                 err);
   else
-    resolve_kernel<false><<<(unsigned)sms, 256, 0, stream>>>(svals, seg_head, n, tokens, stride,
-                                                             lens, rep, coll_list, coll_count,
-                                                             err);
-  scan_kernel<IsRep, OpSum, true><<<(unsigned)scan_tiles, kScanThreads, 0, stream>>>(
-      IsRep{rep}, n, uid, scan1, ctr + 9, n_unique_dev, err);
+    resolve_kernel<false><<<1, 1024, 0, stream>>>(fp, tokens, stride, lens, rep, coll_list, ctr,
+                                                  err);
+  const int64_t tiles = (n + kScanTile - 1) / kScanTile;
+  scan_kernel<<<(unsigned)tiles, kScanThreads, 0, stream>>>(rep, n, uid, status, ctr,
+                                                           n_unique_dev, err);
   finalize_kernel<<<grid_for(n, 256, sms * 8), 256, 0, stream>>>(rep, uid, n, n_unique_dev,
                                                                  unique_idx, inverse);
-  count_launches(10);  // hist, 4 radix passes, 2 scans, verify, resolve, finalize
+  count_launches(5);  // insert, verify, resolve, scan, finalize
   return cuda_fail(cudaGetLastError(), "unique_inverse launch");
 }
 
