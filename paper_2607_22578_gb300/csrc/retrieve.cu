@@ -573,6 +573,76 @@ __device__ __forceinline__ void unpack_key(uint64_t key, float& s, int32_t& idx)
   idx = (int32_t)(0xffffffffu - (uint32_t)key);
 }
 
+// Small kout: one warp per query runs a tournament over the sorted lists.
+// Lane l owns lists l, l+32, ...; it keeps each list's head and the entry
+// after it (prefetched) in registers.  Each round the warp takes the largest
+// head (keys are unique: a corpus row lives in exactly one list; padding
+// keys tie, and the lowest such lane advances), so kout rounds give the kout
+// best in order.
+constexpr int kMaxListsPerLane = 10;
+
+__global__ void __launch_bounds__(256) merge_warp_kernel(const Params p, float* __restrict__ out_s,
+                                                         int32_t* __restrict__ out_i,
+                                                         int32_t kout) {
+  const int64_t Q = query_count(p);
+  const SplitPlan sp = split_plan(Q, p.tiles, p.k, p.slots, p.cl);
+  const int k = p.k;
+  const int lists = 2 * sp.nsplit;
+  const int lane = threadIdx.x & 31;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t q = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; q < Q; q += nwarps) {
+    const float* __restrict__ ps = p.part_s + (size_t)q * lists * k;
+    const int32_t* __restrict__ pi = p.part_i + (size_t)q * lists * k;
+    uint64_t head[kMaxListsPerLane], next[kMaxListsPerLane];
+    int pos[kMaxListsPerLane];
+#pragma unroll
+    for (int j = 0; j < kMaxListsPerLane; ++j) {
+      const int l = j * 32 + lane;
+      pos[j] = 0;
+      head[j] = l < lists ? pack_key(ps[(size_t)l * k], pi[(size_t)l * k]) : 0ull;
+      next[j] = (l < lists && k > 1) ? pack_key(ps[(size_t)l * k + 1], pi[(size_t)l * k + 1]) : 0ull;
+    }
+    float my_s = -FLT_MAX;
+    int32_t my_i = -1;
+    for (int r = 0; r < kout; ++r) {
+      uint64_t best = 0ull;
+      int bj = 0;
+#pragma unroll
+      for (int j = 0; j < kMaxListsPerLane; ++j)
+        if (head[j] > best) {
+          best = head[j];
+          bj = j;
+        }
+      uint64_t mx = best;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const uint64_t y = __shfl_xor_sync(0xffffffffu, mx, o);
+        mx = y > mx ? y : mx;
+      }
+      const unsigned win = __ballot_sync(0xffffffffu, best == mx && mx != 0ull);
+      if (lane == r) {
+        if (mx != 0ull) unpack_key(mx, my_s, my_i);
+      }
+      if (win != 0u && lane == __ffs(win) - 1) {
+#pragma unroll
+        for (int j = 0; j < kMaxListsPerLane; ++j)
+          if (j == bj) {
+            const int l = j * 32 + lane;
+            ++pos[j];
+            head[j] = next[j];
+            next[j] = pos[j] + 1 < k ? pack_key(ps[(size_t)l * k + pos[j] + 1],
+                                                pi[(size_t)l * k + pos[j] + 1])
+                                     : 0ull;
+          }
+      }
+    }
+    if (lane < kout) {
+      out_s[(size_t)q * kout + lane] = my_s;
+      out_i[(size_t)q * kout + lane] = my_i;
+    }
+  }
+}
+
 // Lists of p.k entries per (query, split, half) -> the kout best per query.
 __global__ void __launch_bounds__(256) merge_kernel(const Params p, float* __restrict__ out_s,
                                                     int32_t* __restrict__ out_i, int32_t kout) {
@@ -800,6 +870,12 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
   prm.err = err;
   const int64_t mgrid = Qmax < sms * 8 ? Qmax : sms * 8;
   auto merge = [&](const Params& pm, int32_t kout) -> hs_status {
+    if (kout <= 32 && 2 * (int64_t)pm.slots <= 32 * kMaxListsPerLane) {
+      const int64_t blocks = (Qmax + 7) / 8;        // one warp per query
+      merge_warp_kernel<<<(unsigned)(blocks < sms * 16 ? blocks : sms * 16), 256, 0, stream>>>(
+          pm, scores_out, ids_out, kout);
+      return cuda_fail(cudaGetLastError(), "merge launch");
+    }
     const size_t msmem = (size_t)p2_for(max_splits(sms, pm.tiles, pm.k), pm.k) * 8;
     static size_t merge_configured = 0;
     if (msmem > 48 * 1024 && msmem > merge_configured) {
