@@ -44,8 +44,6 @@ WORKLOAD = ("rag_mix: 64 workflows x 32 queries (30% cross-workflow exact duplic
             "1434 merged) + 65,536 chunk rows x 256 int32 tokens (40% cross-workflow copies); "
             "corpus 1,048,576 x 768 bf16 unit-norm; top-10")
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
-KERNELS_PER_STEP = {  # kernels the library launches per call (hs_launch_count agrees)
-    "hs_fingerprint": 1, "hs_unique_inverse": 10, "hs_scatter_results": 1, "hs_retrieve_topk": 2}
 
 
 # ---------------------------------------------------------------- host logic
@@ -353,16 +351,20 @@ def gpu_arm(args, rank: int, local_rank: int, world: int) -> int:
                 "parallelism": "replicas: one independent stage per GPU (no exchange step)"},
             "dedup_rows_per_s": rows_total / (ms / 1e3),
             "queries_served_per_s": n_q * K * world / (ms / 1e3),
+            # The retrieval launches are timed inside K back-to-back steps (a
+            # long step, power-capped like a seconds-long GEMM loop), so the
+            # denominator is the sustained bf16 peak; the burst fraction is
+            # reported beside it.
             "roofline": {
-                "bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                "frac": achieved / peak, "traffic": traffic,
+                "bound": "tensor", "achieved": achieved, "peak": peak_s, "unit": "TFLOP/s",
+                "frac": achieved / peak_s, "traffic": traffic,
                 "kernel": "hs_retrieve_topk (retrieve_kernel + merge_kernel), %.3f ms/launch"
                           % ret_ms,
                 "algorithmic": "2 * %d merged queries * %d rows * %d dims = %.4g FLOP/launch"
                                % (n_u, N, d, flops),
-                "peak_source": "%s bf16 burst (MEASURED_PEAKS.json)" % peaks_kind
-                               if peaks_kind == "measured" else "fallback bf16 burst",
-                "frac_of_sustained": achieved / peak_s},
+                "peak_source": "%s bf16 sustained (MEASURED_PEAKS.json)" % peaks_kind
+                               if peaks_kind == "measured" else "fallback bf16 sustained",
+                "frac_of_burst": achieved / peak},
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h, "steps": Ke},
             "gpu_launches": int(launches),
