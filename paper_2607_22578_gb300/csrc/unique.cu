@@ -34,6 +34,7 @@ constexpr uint32_t kNoRow = 0xffffffffu;
 constexpr int kScanThreads = 1024;
 constexpr int kScanItems = 16;
 constexpr int kScanTile = kScanThreads * kScanItems;
+static_assert(kScanThreads % 32 == 0 && kScanThreads <= 1024, "scan block: whole warps, at most 32");
 constexpr int kLookBatch = 8;           // predecessor statuses read per round trip
 constexpr int64_t kSmallRows = 4096;    // single-launch path
 constexpr int kSmallThreads = 512;
@@ -390,14 +391,15 @@ __global__ void __launch_bounds__(kScanThreads) scan_kernel(const int32_t* __res
   if (lane == 31) s_warp[w] = incl;
   __syncthreads();
   if (w == 0) {
-    const int32_t v = s_warp[lane];
+    constexpr int kWarps = kScanThreads / 32;
+    const int32_t v = lane < kWarps ? s_warp[lane] : 0;
     int32_t iv = v;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
       const int32_t y = __shfl_up_sync(0xffffffffu, iv, o);
       if (lane >= o) iv += y;
     }
-    s_warp[lane] = iv - v;  // exclusive warp offsets
+    if (lane < kWarps) s_warp[lane] = iv - v;  // exclusive warp offsets
     if (lane == 31) {
       const int32_t tile_total = iv;
       volatile unsigned long long* st = status;
@@ -429,11 +431,20 @@ __global__ void __launch_bounds__(kScanThreads) scan_kernel(const int32_t* __res
   }
   __syncthreads();
   int32_t acc = s_prefix + s_warp[w] + incl - run;
+  int32_t u[kScanItems];
 #pragma unroll
   for (int i = 0; i < kScanItems; ++i) {
-    const int64_t e = base + i;
-    if (e < n) uid[e] = acc;
+    u[i] = acc;
     acc += x[i];
+  }
+  if (base + kScanItems <= n) {
+#pragma unroll
+    for (int i = 0; i < kScanItems; i += 4)
+      *reinterpret_cast<int4*>(uid + base + i) = make_int4(u[i], u[i + 1], u[i + 2], u[i + 3]);
+  } else {
+#pragma unroll
+    for (int i = 0; i < kScanItems; ++i)
+      if (base + i < n) uid[base + i] = u[i];
   }
 }
 
@@ -508,9 +519,11 @@ __global__ void __launch_bounds__(kSmallThreads) unique_small_kernel(
   }
 
   // 3. the last CTA to finish writes the outputs
-  __threadfence();
   __syncthreads();
-  if (tid == 0) s_last = atomicAdd(ctr + kCtrDone, 1u) == gridDim.x - 1;
+  if (tid == 0) {
+    __threadfence();
+    s_last = atomicAdd(ctr + kCtrDone, 1u) == gridDim.x - 1;
+  }
   __syncthreads();
   if (!s_last) return;
   __threadfence();
