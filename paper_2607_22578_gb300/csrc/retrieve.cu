@@ -93,7 +93,21 @@ struct Params {
   // query's final k-th best score, so it prunes without changing the result.
   const float* floor;
   int32_t floor_stride, floor_index;
+  // k <= 32: per-query shared floor, the largest k-th best score any list of
+  // the query has reached so far (order-preserving uint32 code of the float,
+  // 0 = none), raised with atomicMax and read once per tile by every list of
+  // the query.  Zeroed before each launch.
+  uint32_t* qfloor;
 };
+
+__device__ __forceinline__ uint32_t float_code(float f) {
+  const uint32_t u = __float_as_uint(f);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+__device__ __forceinline__ float code_float(uint32_t c) {
+  return __uint_as_float((c & 0x80000000u) ? (c ^ 0x80000000u) : ~c);
+}
 
 __host__ __device__ inline int64_t gcd64(int64_t a, int64_t b) {
   while (b) {
@@ -146,6 +160,19 @@ __device__ __forceinline__ void unit_coords(const SplitPlan& sp, int64_t tiles, 
   split = (int)(u / sp.groups);
   t0 = (int64_t)split * tiles / sp.nsplit;
   t1 = (int64_t)(split + 1) * tiles / sp.nsplit;
+}
+
+// Maximum of 32 scores as a 5-level tree (fmaxf is exact, so the order does
+// not change the result).
+__device__ __forceinline__ float chunk_max(const uint32_t (&r)[32]) {
+  float m[16];
+#pragma unroll
+  for (int j = 0; j < 16; ++j) m[j] = fmaxf(__uint_as_float(r[j]), __uint_as_float(r[j + 16]));
+#pragma unroll
+  for (int w = 8; w > 0; w >>= 1)
+#pragma unroll
+    for (int j = 0; j < w; ++j) m[j] = fmaxf(m[j], m[j + w]);
+  return m[0];
 }
 
 // Insert (s, idx) into a list sorted by score descending.  idx is larger than
@@ -426,13 +453,24 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (f > -FLT_MAX) floor_theta = nextafterf(f, -INFINITY);  // keep s >= f
       }
       float theta = floor_theta;
+      // Register list (k <= 32): KREG slots sorted descending, the first
+      // KREG - k holding +FLT_MAX sentinels that never move, so the last
+      // slot is always the k-th best score seen: the list's own threshold.
       float ls[KREG > 0 ? KREG : 1];
       int32_t li[KREG > 0 ? KREG : 1];
       int cnt = 0, cur = 0;
 #pragma unroll
       for (int i = 0; i < (KREG > 0 ? KREG : 1); ++i) {
-        ls[i] = -FLT_MAX;
+        ls[i] = (KREG > 0 && i < KREG - k) ? FLT_MAX : -FLT_MAX;
         li[i] = -1;
+      }
+      // The query's shared floor, as a threshold that keeps ties with it
+      // (another list may hold an equal score at a higher index).
+      uint32_t qf_seen = 0;
+      float qf_theta = -FLT_MAX;
+      if (KREG > 0 && valid_q && p.qfloor) {   // lists of other splits may have set it
+        qf_seen = *reinterpret_cast<volatile uint32_t*>(p.qfloor + q);
+        if (qf_seen) qf_theta = nextafterf(code_float(qf_seen), -INFINITY);
       }
       if (KREG == 0 && valid_q) {
         for (int i = 0; i < k; ++i) {
@@ -444,6 +482,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t acc = tile_i & 1u, aphase = (tile_i >> 1) & 1u;
         if (!mbar_wait(tfull + acc, aphase, abort_flag)) goto epi_done;
         tc_fence_after();
+        if (KREG > 0) theta = fmaxf(theta, qf_theta);
         const int64_t col0 = t * BN + half * kHalfCols;
         const bool tail = col0 + kHalfCols > p.N;
 #pragma unroll 1
@@ -462,9 +501,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int j = 0; j < 32; ++j) r[j] = __float_as_uint(-FLT_MAX);
           }
           if (KREG > 0) {
-            float mx = __uint_as_float(r[0]);
-#pragma unroll
-            for (int j = 1; j < 32; ++j) mx = fmaxf(mx, __uint_as_float(r[j]));
+            float mx = chunk_max(r);
             const bool any = mx > theta;
             if (__any_sync(0xffffffffu, any)) {
               uint32_t m = 0;
@@ -483,7 +520,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 m &= m - 1;
                 if (s > theta) {
                   list_insert<(KREG > 0 ? KREG : 1)>(ls, li, s, cbase + j);
-                  theta = ls[(KREG > 0 ? KREG : 1) - 1];
+                  theta = fmaxf(ls[(KREG > 0 ? KREG : 1) - 1], qf_theta);
                 }
               }
               __syncwarp();
@@ -491,9 +528,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           } else {
             // Same first test as above: a chunk whose maximum beats no
             // lane's threshold costs one max-reduction and a vote.
-            float mx = __uint_as_float(r[0]);
-#pragma unroll
-            for (int j = 1; j < 32; ++j) mx = fmaxf(mx, __uint_as_float(r[j]));
+            const float mx = chunk_max(r);
             if (__any_sync(0xffffffffu, mx > theta)) {
 #pragma unroll
               for (int j0 = 0; j0 < 32; j0 += 4) {
@@ -514,6 +549,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tc_fence_before();
         __syncwarp();
+        if (KREG > 0 && valid_q && p.qfloor) {
+          // Publish this list's k-th best if it raises the query's floor,
+          // and fetch the floor for the next tile.
+          const float kth = ls[(KREG > 0 ? KREG : 1) - 1];
+          const uint32_t mine = kth > -FLT_MAX ? float_code(kth) : 0u;
+          if (mine > qf_seen) atomicMax(p.qfloor + q, mine);
+          const uint32_t c = *reinterpret_cast<volatile uint32_t*>(p.qfloor + q);
+          if (c > qf_seen) {
+            qf_seen = c;
+            qf_theta = nextafterf(code_float(c), -INFINITY);  // keep s >= floor
+          }
+        }
         if (lane == 0) {
           if (CL == 1)
             mbar_arrive(tempty + acc);
@@ -528,9 +575,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (KREG > 0) {
 #pragma unroll
           for (int i = 0; i < (KREG > 0 ? KREG : 1); ++i)
-            if (i < k) {
-              os[i] = ls[i];
-              oi[i] = li[i];
+            if (i >= KREG - k) {
+              os[i - (KREG - k)] = ls[i];
+              oi[i - (KREG - k)] = li[i];
             }
         } else {
           flush_candidates(cand_s, cand_i, et, cnt, Ls, Li, k, cur, theta, floor_theta);
@@ -832,7 +879,8 @@ size_t retrieve_topk_workspace(int64_t Q, int64_t N, int32_t d, int32_t k) {
   const int64_t ns = max_splits(sms, (N + BN - 1) / BN, k);
   const size_t part = (((size_t)Q * 2 * ns * k * 4) + 255) & ~(size_t)255;
   const size_t list = k <= 32 ? 0 : ((((size_t)sms * kEpi * 2 * k * 4) + 255) & ~(size_t)255);
-  return 2 * part + 2 * list + 256;
+  const size_t qfloor = (((size_t)Q * 4) + 255) & ~(size_t)255;
+  return 2 * part + 2 * list + qfloor + 256;
 }
 
 // Qmax rows of `queries` are addressable; the kernels process the first
@@ -867,7 +915,11 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
   prm.part_i = reinterpret_cast<int32_t*>(w + part);
   prm.list_s = reinterpret_cast<float*>(w + 2 * part);
   prm.list_i = reinterpret_cast<int32_t*>(w + 2 * part + list);
+  prm.qfloor = reinterpret_cast<uint32_t*>(w + 2 * part + 2 * list);
   prm.err = err;
+  // The shared per-query floors of the register-list passes start empty.
+  const cudaError_t ze = cudaMemsetAsync(prm.qfloor, 0, (size_t)Qmax * 4, stream);
+  if (ze != cudaSuccess) return cuda_fail(ze, "floor clear");
   const int64_t mgrid = Qmax < sms * 8 ? Qmax : sms * 8;
   auto merge = [&](const Params& pm, int32_t kout) -> hs_status {
     if (kout <= 32 && 2 * (int64_t)pm.slots <= 32 * kMaxListsPerLane) {
