@@ -296,39 +296,40 @@ def gpu_arm(args, rank: int, local_rank: int, world: int) -> int:
 
     breakdown = rag_mix_breakdown(stage, tokens, queries, min(K, 50)) if args.breakdown else None
 
-    # End to end through the public API: pinned host inputs in, results out.
+    # End to end through the public API: every step copies its inputs from
+    # pinned host memory and its scores and ids back, and the host reads
+    # each step's results (HostFeed overlaps step i+1's input copy with
+    # step i's kernels; the host reads step i's results after submitting
+    # step i+1).
     h_tokens = torch.from_numpy(w["tokens"]).pin_memory()
     h_queries = torch.from_numpy(w["queries"].view(np.int16)).pin_memory()
-    d_tok = torch.empty_like(tokens)
-    d_q = torch.empty_like(queries)
-    h_s = torch.empty((n_q, k), dtype=torch.float32).pin_memory()
-    h_i = torch.empty((n_q, k), dtype=torch.int32).pin_memory()
+    feed = hs.HostFeed(stage, n_chunk, tokens.shape[1], n_q)
     Ke = max(1, min(K, 100))
 
-    def e2e_step():
-        d_tok.copy_(h_tokens, non_blocking=True)
-        d_q.view(torch.int16).copy_(h_queries, non_blocking=True)
-        _, (s, i, _) = stage.step(d_tok, d_q)
-        h_s.copy_(s, non_blocking=True)
-        h_i.copy_(i, non_blocking=True)
-        torch.cuda.current_stream().synchronize()   # the results are read on the host
-        return n_u
+    def e2e_run(steps):
+        prev, nu = None, 0
+        for _ in range(steps):
+            slot = feed.submit(h_tokens, h_queries)
+            if prev is not None:
+                nu += feed.fetch(prev)[2]
+            prev = slot
+        nu += feed.fetch(prev)[2]
+        return nu
 
-    for _ in range(3):
-        e2e_step()
+    e2e_run(3)
     barrier(world)
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record()
-    for _ in range(Ke):
-        nu = e2e_step()
+    feed.copy_stream.wait_stream(torch.cuda.current_stream())   # no copy before e0
+    nu_total = e2e_run(Ke)
     e1.record()
     torch.cuda.synchronize()
     barrier(world)
-    ems, emerged = reduce_over_ranks(e0.elapsed_time(e1), float(nu * Ke), world)
+    ems, emerged = reduce_over_ranks(e0.elapsed_time(e1), float(nu_total), world)
     e2e_value = emerged / (ems / 1e3)
     h2d = h_tokens.numel() * 4 + h_queries.numel() * 2
-    d2h = h_s.numel() * 4 + h_i.numel() * 4
+    d2h = feed.h_s[0].numel() * 4 + feed.h_i[0].numel() * 4 + 4
 
     flops = 2.0 * n_u * N * d
     achieved = flops / (ret_ms / 1e3) / 1e12

@@ -111,3 +111,63 @@ class EmbedRetrieveStage:
         scores = _lib.hs_scatter_results(s_u, inv, dst=self.scores[:Q])
         ids = _lib.hs_scatter_results(i_u, inv, dst=self.ids[:Q])
         return chunk, (scores, ids, nu)
+
+
+class HostFeed:
+    """Runs batches that live in (pinned) host memory through a stage, with
+    the next batch's host-to-device copy overlapping the current batch's
+    kernels.
+
+    Two device copies of the inputs alternate: batch i is copied on a copy
+    stream into buffer i % 2 once batch i - 2 (the last user of that buffer)
+    has finished, and the stage runs on the current stream after the copy.
+    Each batch's scores and ids are copied back into their own pinned host
+    buffers; ``fetch`` waits for that copy and returns them."""
+
+    def __init__(self, stage: EmbedRetrieveStage, chunk_rows: int, chunk_stride: int,
+                 n_queries: int):
+        dev = stage.device
+        self.stage = stage
+        self.copy_stream = torch.cuda.Stream(device=dev)
+        self.d_tok = [torch.empty((chunk_rows, chunk_stride), dtype=torch.int32, device=dev)
+                      for _ in range(2)]
+        self.d_q = [torch.empty((n_queries, stage.d), dtype=stage.corpus.dtype, device=dev)
+                    for _ in range(2)]
+        self.h_s = [torch.empty((n_queries, stage.k), dtype=torch.float32).pin_memory()
+                    for _ in range(2)]
+        self.h_i = [torch.empty((n_queries, stage.k), dtype=torch.int32).pin_memory()
+                    for _ in range(2)]
+        self.h_nu = [torch.empty(1, dtype=torch.int32).pin_memory() for _ in range(2)]
+        self.copied = [torch.cuda.Event() for _ in range(2)]
+        self.freed = [torch.cuda.Event() for _ in range(2)]
+        self.done = [torch.cuda.Event() for _ in range(2)]
+        self.used = [False, False]
+        self.count = 0
+
+    def submit(self, h_tokens: torch.Tensor, h_queries: torch.Tensor) -> int:
+        """Enqueue one batch (host tensors, pinned for an asynchronous copy).
+        Returns its slot for ``fetch``.  The slot's previous results must
+        have been fetched already."""
+        b = self.count % 2
+        self.count += 1
+        main = torch.cuda.current_stream(self.stage.device)
+        if self.used[b]:
+            self.copy_stream.wait_event(self.freed[b])
+        with torch.cuda.stream(self.copy_stream):
+            self.d_tok[b].copy_(h_tokens, non_blocking=True)
+            self.d_q[b].view(torch.int16).copy_(h_queries.view(torch.int16), non_blocking=True)
+            self.copied[b].record(self.copy_stream)
+        main.wait_event(self.copied[b])
+        _, (s, i, nu) = self.stage.step(self.d_tok[b], self.d_q[b])
+        self.freed[b].record(main)
+        self.h_s[b].copy_(s, non_blocking=True)
+        self.h_i[b].copy_(i, non_blocking=True)
+        self.h_nu[b].copy_(nu, non_blocking=True)
+        self.done[b].record(main)
+        self.used[b] = True
+        return b
+
+    def fetch(self, slot: int):
+        """Wait for a submitted batch; returns host (scores, ids, n_unique)."""
+        self.done[slot].synchronize()
+        return self.h_s[slot], self.h_i[slot], int(self.h_nu[slot][0])

@@ -245,3 +245,20 @@ def test_large_k_best_rows_outside_the_sample():
         C[N - 200 - 30 * q: N - 30 * q] = Q[q]
     gs, gi = gpu_topk(to_dev(Q), to_dev(C), k)
     parity(Q, C, k, gs, gi, range(nq))
+
+
+def test_shared_floor_keeps_ties_across_splits():
+    # 50 exact copies of each query spread over a corpus of many splits: every
+    # list that holds >= k copies raises the query's shared floor to the copy
+    # score, and lists elsewhere must still keep their copies (ties at the
+    # floor), so the top 10 are the 10 lowest-index copies.
+    nq, N, d, k = 6, 300000, 128, 10
+    Q, C = unit_pair(nq, N, d, 31)
+    rng = np.random.default_rng(7)
+    for q in range(nq):
+        pos = np.sort(rng.choice(N, size=50, replace=False))
+        C[pos] = Q[q]
+    gs, gi = gpu_topk(to_dev(Q), to_dev(C), k)
+    os_, oi = oracle.topk(Q, C, k)
+    assert (gi == oi).all()
+    parity(Q, C, k, gs, gi, range(nq))

@@ -58,3 +58,26 @@ def test_step_runs_both_paths_and_matches_separate_calls():
     s2, i2, _ = stage.retrieve(q)
     hs.hs_get_device_error()
     assert (s.cpu() == s2.cpu()).all() and (i.cpu() == i2.cpu()).all()
+
+
+def test_host_feed_matches_device_step():
+    import torch
+    w = configs.build_retrieval_mix(configs.TINY)
+    stage = hs.EmbedRetrieveStage(to_dev(w["corpus"]), w["k"], max_queries=len(w["queries"]),
+                                  max_chunk_rows=w["tokens"].shape[0])
+    s_ref, i_ref, nu_ref = stage.retrieve(to_dev(w["queries"]))
+    hs.hs_get_device_error()
+    s_ref, i_ref, nu_ref = s_ref.cpu(), i_ref.cpu(), int(nu_ref.item())
+    h_tok = torch.from_numpy(w["tokens"]).pin_memory()
+    h_q = torch.from_numpy(w["queries"].view(np.int16)).pin_memory()
+    feed = hs.HostFeed(stage, w["tokens"].shape[0], w["tokens"].shape[1], len(w["queries"]))
+    prev = None
+    for _ in range(5):                       # alternate both buffers twice over
+        slot = feed.submit(h_tok, h_q)
+        if prev is not None:
+            s, i, nu = feed.fetch(prev)
+            assert nu == nu_ref and torch.equal(s, s_ref) and torch.equal(i, i_ref)
+        prev = slot
+    s, i, nu = feed.fetch(prev)
+    hs.hs_get_device_error()
+    assert nu == nu_ref and torch.equal(s, s_ref) and torch.equal(i, i_ref)
