@@ -485,11 +485,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (KREG > 0) theta = fmaxf(theta, qf_theta);
         const int64_t col0 = t * BN + half * kHalfCols;
         const bool tail = col0 + kHalfCols > p.N;
-#pragma unroll 1
-        for (int c = 0; c < kHalfCols / 32; ++c) {
-          uint32_t r[32];
-          tmem_ld_32x32b_x32(tmem_base + lane_addr + acc * BN + half * kHalfCols + c * 32, r);
-          tmem_ld_wait();
+        // One 32-column chunk: mask columns past N / invalid queries, then
+        // the threshold test and candidate handling.
+        auto do_chunk = [&](uint32_t(&r)[32], int c) {
           const int32_t cbase = (int32_t)(col0 + c * 32);
           if (tail) {                           // zero-filled rows past N never qualify
 #pragma unroll
@@ -546,6 +544,17 @@ __global__ void __launch_bounds__(kThreads, 1)
               }
             }
           }
+                };
+        // Two chunks per TMEM round trip: both loads, one wait.
+#pragma unroll 1
+        for (int c = 0; c < kHalfCols / 32; c += 2) {
+          uint32_t ra[32], rb[32];
+          const uint32_t ta = tmem_base + lane_addr + acc * BN + half * kHalfCols + c * 32;
+          tmem_ld_32x32b_x32(ta, ra);
+          tmem_ld_32x32b_x32(ta + 32, rb);
+          tmem_ld_wait();
+          do_chunk(ra, c);
+          do_chunk(rb, c + 1);
         }
         tc_fence_before();
         __syncwarp();
