@@ -545,16 +545,24 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
           }
                 };
-        // Two chunks per TMEM round trip: both loads, one wait.
+        // Register lists: two chunks per TMEM round trip (both loads, one
+        // wait).  Large k keeps one, as its candidate path needs the registers.
 #pragma unroll 1
-        for (int c = 0; c < kHalfCols / 32; c += 2) {
-          uint32_t ra[32], rb[32];
+        for (int c = 0; c < kHalfCols / 32; c += (KREG > 0 ? 2 : 1)) {
           const uint32_t ta = tmem_base + lane_addr + acc * BN + half * kHalfCols + c * 32;
-          tmem_ld_32x32b_x32(ta, ra);
-          tmem_ld_32x32b_x32(ta + 32, rb);
-          tmem_ld_wait();
-          do_chunk(ra, c);
-          do_chunk(rb, c + 1);
+          uint32_t ra[32];
+          if (KREG > 0) {
+            uint32_t rb[32];
+            tmem_ld_32x32b_x32(ta, ra);
+            tmem_ld_32x32b_x32(ta + 32, rb);
+            tmem_ld_wait();
+            do_chunk(ra, c);
+            do_chunk(rb, c + 1);
+          } else {
+            tmem_ld_32x32b_x32(ta, ra);
+            tmem_ld_wait();
+            do_chunk(ra, c);
+          }
         }
         tc_fence_before();
         __syncwarp();

@@ -25,11 +25,15 @@ __device__ __forceinline__ void st_chunk<uint8_t>(uint8_t* p, const uint8_t& v) 
 template <>
 __device__ __forceinline__ uint8_t ld_chunk<uint8_t>(const uint8_t* p) { return *p; }
 
+// row = g / cpr as one 64x64 high multiply: with magic = floor((2^64 - 1) / cpr)
+// + 1 (the reciprocal rounded up), the quotient is exact for every g with
+// g * cpr < 2^64, which the host checks for the largest g.
 template <class T, int U>
 __global__ void __launch_bounds__(256) scatter_kernel(const T* __restrict__ src, int64_t n_src,
                                                       const int32_t* __restrict__ map,
                                                       int64_t n_rows, uint32_t cpr,
-                                                      T* __restrict__ dst, unsigned* err) {
+                                                      uint64_t magic, T* __restrict__ dst,
+                                                      unsigned* err) {
   const int64_t total = n_rows * (int64_t)cpr;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t g0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g0 < total; g0 += stride * U) {
@@ -41,7 +45,7 @@ __global__ void __launch_bounds__(256) scatter_kernel(const T* __restrict__ src,
       const int64_t g = g0 + (int64_t)u * stride;
       ok[u] = false;
       if (g < total) {
-        const int64_t row = g / cpr;
+        const int64_t row = magic ? (int64_t)__umul64hi((uint64_t)g, magic) : g / cpr;
         const int64_t c = g - row * cpr;
         const int32_t m = __ldg(map + row);
         if (m < 0 || (int64_t)m >= n_src) {
@@ -69,8 +73,13 @@ hs_status launch_typed(const void* src, int64_t n_src, int64_t row_bytes, const 
   const int64_t cap = (int64_t)num_sms() * 16;
   if (blocks > cap) blocks = cap;
   if (blocks < 1) blocks = 1;
+  // Reciprocal multiply when (total - 1) * cpr fits in 64 bits (else divide).
+  uint64_t magic = 0;
+  const unsigned __int128 span = (unsigned __int128)(uint64_t)(total > 0 ? total - 1 : 0) * (uint64_t)cpr;
+  if (cpr > 0 && (span >> 64) == 0) magic = ~0ull / (uint64_t)cpr + 1ull;
   scatter_kernel<T, U><<<(unsigned)blocks, 256, 0, stream>>>(
-      static_cast<const T*>(src), n_src, map, n_rows, (uint32_t)cpr, static_cast<T*>(dst), err);
+      static_cast<const T*>(src), n_src, map, n_rows, (uint32_t)cpr, magic, static_cast<T*>(dst),
+      err);
   count_launches(1);
   return cuda_fail(cudaGetLastError(), "scatter launch");
 }
