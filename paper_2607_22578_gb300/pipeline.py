@@ -47,6 +47,11 @@ class EmbedRetrieveStage:
         self.scores = torch.empty((mq, self.k), dtype=torch.float32, device=dev)
         self.ids = torch.empty((mq, self.k), **i32)
 
+    def capture(self, tokens: torch.Tensor, queries: torch.Tensor,
+                lens: torch.Tensor | None = None) -> "StepGraph":
+        """Capture ``step`` on these device buffers as a replayable CUDA graph."""
+        return StepGraph(self, tokens, queries, lens)
+
     def dedup_chunks(self, tokens: torch.Tensor, lens: torch.Tensor | None = None):
         """Fingerprint + exact unique of chunk rows.  Returns (n_unique_dev,
         unique_idx, inverse, fp) as device tensors."""
@@ -113,6 +118,35 @@ class EmbedRetrieveStage:
         return chunk, (scores, ids, nu)
 
 
+class StepGraph:
+    """One stage step captured as a CUDA graph on fixed device input buffers.
+
+    ``replay()`` enqueues the whole step — both dedup paths, the gather, the
+    retrieval and the result scatter, with the chunk path on its own branch —
+    as one graph launch on the current stream, so the host issues one call
+    instead of about twenty and the kernels follow each other without
+    per-launch gaps.  Refill ``tokens``/``queries`` (the captured buffers) in
+    place between replays; ``outputs`` are the stage's result buffers, which
+    every replay overwrites."""
+
+    def __init__(self, stage: "EmbedRetrieveStage", tokens: torch.Tensor,
+                 queries: torch.Tensor, lens: torch.Tensor | None = None):
+        self.tokens, self.queries, self.lens = tokens, queries, lens
+        # One eager step first: one-time host work (kernel attributes,
+        # occupancy queries) must not happen inside the capture.
+        stage.step(tokens, queries, lens)
+        torch.cuda.synchronize(stage.device)
+        self.graph = torch.cuda.CUDAGraph()
+        l0 = _lib.hs_launch_count()
+        with torch.cuda.graph(self.graph):
+            self.outputs = stage.step(tokens, queries, lens)
+        self.launches = _lib.hs_launch_count() - l0   # kernels per replay
+
+    def replay(self):
+        self.graph.replay()
+        return self.outputs
+
+
 class HostFeed:
     """Runs batches that live in (pinned) host memory through a stage, with
     the next batch's host-to-device copy overlapping the current batch's
@@ -125,14 +159,19 @@ class HostFeed:
     buffers; ``fetch`` waits for that copy and returns them."""
 
     def __init__(self, stage: EmbedRetrieveStage, chunk_rows: int, chunk_stride: int,
-                 n_queries: int):
+                 n_queries: int, graphs: bool = True):
         dev = stage.device
         self.stage = stage
         self.copy_stream = torch.cuda.Stream(device=dev)
-        self.d_tok = [torch.empty((chunk_rows, chunk_stride), dtype=torch.int32, device=dev)
+        self.d_tok = [torch.zeros((chunk_rows, chunk_stride), dtype=torch.int32, device=dev)
                       for _ in range(2)]
-        self.d_q = [torch.empty((n_queries, stage.d), dtype=stage.corpus.dtype, device=dev)
+        self.d_q = [torch.zeros((n_queries, stage.d), dtype=stage.corpus.dtype, device=dev)
                     for _ in range(2)]
+        # With graphs, each input buffer gets its captured step (nothing in a
+        # step depends on the data on the host side, so replays serve any
+        # contents of the buffers).
+        self.graphs = ([stage.capture(self.d_tok[b], self.d_q[b]) for b in range(2)]
+                       if graphs else None)
         self.h_s = [torch.empty((n_queries, stage.k), dtype=torch.float32).pin_memory()
                     for _ in range(2)]
         self.h_i = [torch.empty((n_queries, stage.k), dtype=torch.int32).pin_memory()
@@ -158,7 +197,10 @@ class HostFeed:
             self.d_q[b].view(torch.int16).copy_(h_queries.view(torch.int16), non_blocking=True)
             self.copied[b].record(self.copy_stream)
         main.wait_event(self.copied[b])
-        _, (s, i, nu) = self.stage.step(self.d_tok[b], self.d_q[b])
+        if self.graphs is not None:
+            _, (s, i, nu) = self.graphs[b].replay()
+        else:
+            _, (s, i, nu) = self.stage.step(self.d_tok[b], self.d_q[b])
         self.freed[b].record(main)
         self.h_s[b].copy_(s, non_blocking=True)
         self.h_i[b].copy_(i, non_blocking=True)

@@ -81,3 +81,32 @@ def test_host_feed_matches_device_step():
     s, i, nu = feed.fetch(prev)
     hs.hs_get_device_error()
     assert nu == nu_ref and torch.equal(s, s_ref) and torch.equal(i, i_ref)
+
+
+def test_step_graph_replays_match_eager_step():
+    import torch
+    w = configs.build_retrieval_mix(configs.TINY)
+    stage = hs.EmbedRetrieveStage(to_dev(w["corpus"]), w["k"], max_queries=len(w["queries"]),
+                                  max_chunk_rows=w["tokens"].shape[0])
+    t, q = to_dev(w["tokens"]), to_dev(w["queries"])
+    (cnu, cu, ci, _), (s, i, nu) = stage.step(t, q)
+    hs.hs_get_device_error()
+    ref = [x.cpu().clone() for x in (cnu, cu, ci, s, i, nu)]
+    g = hs.StepGraph(stage, t, q)
+    assert g.launches > 0
+    for _ in range(3):
+        (cnu, cu, ci, _), (s, i, nu) = g.replay()
+        hs.hs_get_device_error()
+        n = int(cnu.item())
+        got = [x.cpu() for x in (cnu, cu, ci, s, i, nu)]
+        assert torch.equal(got[0], ref[0]) and torch.equal(got[1][:n], ref[1][:n])
+        assert all(torch.equal(a, b) for a, b in zip(got[2:], ref[2:]))
+    # new contents in the captured buffers are picked up by the next replay
+    q2 = to_dev(w["queries"][::-1].copy())
+    q.copy_(q2)
+    _, (s2, i2, _) = g.replay()
+    s2, i2 = s2.cpu(), i2.cpu()          # host copies: retrieve() reuses the buffers
+    s3, i3, _ = stage.retrieve(q2)
+    hs.hs_get_device_error()
+    assert torch.equal(s2, s3.cpu()) and torch.equal(i2, i3.cpu())
+    assert not torch.equal(s2, ref[3])   # the reversed batch has different results
