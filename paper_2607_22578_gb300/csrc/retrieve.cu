@@ -752,6 +752,253 @@ __global__ void __launch_bounds__(256) merge_kernel(const Params p, float* __res
   }
 }
 
+// ---- K6s: small batches (at most 16 queries) -------------------------------------------
+// With few queries the query block of the main kernel is mostly padding and
+// is re-streamed with every corpus stage.  Here the roles are swapped: the
+// corpus tile is the MMA's M operand (128 rows) and the queries, padded to
+// 16, are its N operand, loaded once and kept in shared memory.  The ring
+// then carries only corpus boxes (10 stages of 16 KB), which is what an
+// HBM-bound pass needs.  TMEM holds four 128 x 16 fp32 accumulators.
+//
+// Epilogue (warps 2-5, one per TMEM lane quarter): thread = corpus row of the
+// tile, holding its 16 scores.  A score above its query's threshold is
+// appended to that query's candidate buffer in shared memory; after each
+// tile a warp merges each non-empty buffer with the query's sorted top-k list
+// (k rounds of a warp-wide maximum over packed (score, ~row) keys) and resets
+// the threshold to the new k-th best.  Each CTA covers a contiguous range of
+// 128-row tiles and writes one sorted list per query, in the layout of the
+// main kernel's lists, so the same merge kernel finishes the job.
+constexpr int SQ_N = 16;                    // queries per MMA (N)
+constexpr int SQ_BM = 128;                  // corpus rows per tile (M)
+constexpr int SQ_STAGES = 10;
+constexpr int SQ_MAXKB = 16;                // d <= 1024
+constexpr int SQ_TBUF = 4;                  // TMEM accumulators
+constexpr uint32_t SQ_TMEM_COLS = 64;       // SQ_TBUF * SQ_N
+constexpr int SQ_CAP = SQ_BM;               // candidates per query per tile: at most one per row
+constexpr int SQ_THREADS = 64 + 128;        // producer, MMA, 4 epilogue warps
+constexpr uint32_t SQ_ABYTES = SQ_BM * BK * 2;   // 16 KB
+constexpr uint32_t SQ_QBYTES = SQ_N * BK * 2;    // 2 KB per k-block
+constexpr size_t SQ_EPI_BYTES = (size_t)SQ_N * (SQ_CAP + 32) * 8 + SQ_N * 8;
+constexpr size_t SQ_SMEM = 1024 + (size_t)SQ_MAXKB * SQ_QBYTES + (size_t)SQ_STAGES * SQ_ABYTES +
+                           256 + SQ_EPI_BYTES;
+static_assert(SQ_SMEM <= 232448, "small-batch kernel shared memory");
+static_assert(8 * (2 * SQ_STAGES + 1 + 2 * SQ_TBUF) + 8 <= 256, "small-batch barrier area");
+
+__global__ void __launch_bounds__(SQ_THREADS, 1)
+    retrieve_small_kernel(const __grid_constant__ CUtensorMap tmap_q,
+                          const __grid_constant__ CUtensorMap tmap_c, const Params p,
+                          int64_t tiles128) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  uint8_t* sQ = smem;
+  uint8_t* sA = sQ + SQ_MAXKB * SQ_QBYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sA + SQ_STAGES * SQ_ABYTES);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + SQ_STAGES;
+  uint64_t* qfull = bars + 2 * SQ_STAGES;
+  uint64_t* tfull = qfull + 1;
+  uint64_t* tempty = tfull + SQ_TBUF;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + SQ_TBUF);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  uint64_t* lists = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(bars) + 256);  // [16][32]
+  uint64_t* cands = lists + SQ_N * 32;                                                    // [16][128]
+  float* theta = reinterpret_cast<float*>(cands + SQ_N * SQ_CAP);                          // [16]
+  int32_t* cnt = reinterpret_cast<int32_t*>(theta + SQ_N);                                 // [16]
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < SQ_STAGES; ++s) {
+      mbar_init(full + s, 1);
+      mbar_init(empty + s, 1);
+    }
+    mbar_init(qfull, 1);
+    for (int b = 0; b < SQ_TBUF; ++b) {
+      mbar_init(tfull + b, 1);
+      mbar_init(tempty + b, 4);
+    }
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    prefetch_tmap(&tmap_q);
+    prefetch_tmap(&tmap_c);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, SQ_TMEM_COLS);
+    tmem_relinquish();
+  }
+  for (int i = threadIdx.x; i < SQ_N * 32; i += SQ_THREADS) lists[i] = 0ull;
+  if (threadIdx.x < SQ_N) {
+    theta[threadIdx.x] = -FLT_MAX;
+    cnt[threadIdx.x] = 0;
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const int64_t Q = query_count(p);
+  const int k = p.k;
+  const int64_t t0 = (int64_t)blockIdx.x * tiles128 / gridDim.x;
+  const int64_t t1 = (int64_t)(blockIdx.x + 1) * tiles128 / gridDim.x;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0 && Q > 0) {
+      const uint64_t pol_c = policy_evict_first();
+      mbar_arrive_expect_tx(qfull, (uint32_t)p.kb_count * SQ_QBYTES);
+      for (int kb = 0; kb < p.kb_count; ++kb)
+        tma_load_2d(sQ + kb * SQ_QBYTES, &tmap_q, qfull, kb * BK, 0);
+      uint32_t stage = 0, phase = 0;
+      for (int64_t t = t0; t < t1; ++t) {
+        for (int kb = 0; kb < p.kb_count; ++kb) {
+          if (!mbar_wait(empty + stage, phase ^ 1u, abort_flag)) goto sq_producer_done;
+          mbar_arrive_expect_tx(full + stage, SQ_ABYTES);
+          tma_load_2d_hint(sA + stage * SQ_ABYTES, &tmap_c, full + stage, kb * BK,
+                           (int32_t)(t * SQ_BM), pol_c);
+          if (++stage == SQ_STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+    sq_producer_done:;
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0 && Q > 0) {
+      constexpr uint32_t idesc = idesc_bf16_f32(SQ_BM, SQ_N);
+      uint32_t stage = 0, phase = 0, tile_i = 0;
+      if (!mbar_wait(qfull, 0u, abort_flag)) goto sq_mma_done;
+      tc_fence_after();
+      for (int64_t t = t0; t < t1; ++t, ++tile_i) {
+        const uint32_t b = tile_i % SQ_TBUF, bphase = (tile_i / SQ_TBUF) & 1u;
+        if (!mbar_wait(tempty + b, bphase ^ 1u, abort_flag)) goto sq_mma_done;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + b * SQ_N;
+        for (int kb = 0; kb < p.kb_count; ++kb) {
+          if (!mbar_wait(full + stage, phase, abort_flag)) goto sq_mma_done;
+          tc_fence_after();
+          const uint64_t a0 = smem_desc_k_sw128(smem_u32(sA + stage * SQ_ABYTES));
+          const uint64_t b0 = smem_desc_k_sw128(smem_u32(sQ + kb * SQ_QBYTES));
+#pragma unroll
+          for (int kk = 0; kk < BK / UK; ++kk)
+            umma_bf16(d_tmem, a0 + (uint64_t)(kk * UK * 2 / 16), b0 + (uint64_t)(kk * UK * 2 / 16),
+                      idesc, (kb | kk) != 0 ? 1u : 0u);
+          umma_commit(empty + stage);
+          if (++stage == SQ_STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        umma_commit(tfull + b);
+      }
+    sq_mma_done:;
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int ew = warp - 2;                     // 0..3, merges queries q = ew (mod 4)
+    const int quarter = warp & 3;                // TMEM lanes [32*quarter, 32*quarter+32)
+    const uint32_t lane_addr = (uint32_t)(quarter * 32) << 16;
+    const int nq = (int)(Q < SQ_N ? Q : SQ_N);
+    uint32_t tile_i = 0;
+    for (int64_t t = t0; t < t1 && nq > 0; ++t, ++tile_i) {
+      const uint32_t b = tile_i % SQ_TBUF, bphase = (tile_i / SQ_TBUF) & 1u;
+      // On a timeout every later wait fails at once; the named barriers
+      // below stay paired because all four warps walk every tile.
+      const bool ok = mbar_wait(tfull + b, bphase, abort_flag);
+      tc_fence_after();
+      uint32_t r[16];
+      tmem_ld_32x32b_x16(tmem_base + lane_addr + b * SQ_N, r);
+      tmem_ld_wait();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(tempty + b);
+      const int64_t row = t * SQ_BM + quarter * 32 + lane;
+      if (ok && row < p.N) {
+#pragma unroll
+        for (int q = 0; q < SQ_N; ++q) {
+          const float sc = __uint_as_float(r[q]);
+          if (q < nq && sc > theta[q]) {
+            const int slot = atomicAdd(cnt + q, 1);
+            if (slot < SQ_CAP) cands[q * SQ_CAP + slot] = pack_key(sc, (int32_t)row);
+          }
+        }
+      }
+      named_bar_sync(1, 128);
+      // Merge: list (k sorted keys) + candidates -> the k best, per query.
+      for (int q = ew; q < nq; q += 4) {
+        const int c = min(cnt[q], SQ_CAP);
+        if (c == 0) continue;
+        uint64_t held[1 + SQ_CAP / 32];
+        held[0] = lane < k ? lists[q * 32 + lane] : 0ull;
+#pragma unroll
+        for (int j = 0; j < SQ_CAP / 32; ++j) {
+          const int e = j * 32 + lane;
+          held[1 + j] = e < c ? cands[q * SQ_CAP + e] : 0ull;
+        }
+        uint64_t mine = 0ull;
+        for (int rd = 0; rd < k; ++rd) {
+          uint64_t best = held[0];
+          int bj = 0;
+#pragma unroll
+          for (int j = 1; j < 1 + SQ_CAP / 32; ++j)
+            if (held[j] > best) {
+              best = held[j];
+              bj = j;
+            }
+          uint64_t mx = best;
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) {
+            const uint64_t y = __shfl_xor_sync(0xffffffffu, mx, o);
+            mx = y > mx ? y : mx;
+          }
+          if (lane == rd) mine = mx;
+          if (mx == 0ull) continue;
+          const unsigned win = __ballot_sync(0xffffffffu, best == mx);
+          if (lane == __ffs(win) - 1) {
+#pragma unroll
+            for (int j = 0; j < 1 + SQ_CAP / 32; ++j)
+              if (j == bj) held[j] = 0ull;
+          }
+        }
+        if (lane < k) lists[q * 32 + lane] = mine;
+        const uint64_t kth = __shfl_sync(0xffffffffu, mine, k - 1);
+        if (lane == 0) {
+          float sk = -FLT_MAX;
+          int32_t ik;
+          if (kth != 0ull) unpack_key(kth, sk, ik);
+          theta[q] = sk;
+          cnt[q] = 0;
+        }
+      }
+      named_bar_sync(1, 128);
+    }
+    // This CTA's list per query (list index = blockIdx.x of 2 * nsplit).
+    const int nlists = (int)gridDim.x;
+    for (int q = ew; q < nq; q += 4) {
+      if (lane < k) {
+        const uint64_t key = lists[q * 32 + lane];
+        float sc = -FLT_MAX;
+        int32_t id = -1;
+        if (key != 0ull) unpack_key(key, sc, id);
+        const size_t o = ((size_t)q * nlists + blockIdx.x) * k + lane;
+        p.part_s[o] = sc;
+        p.part_i[o] = id;
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem_base, SQ_TMEM_COLS);
+  }
+  if (threadIdx.x == 0 && *abort_flag) set_error(p.err, kErrTimeout);
+}
+
 // ---- host side ---------------------------------------------------------------------------
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
@@ -957,7 +1204,28 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
     return cuda_fail(cudaGetLastError(), "merge launch");
   };
   hs_status st;
-  if (k <= 16) {
+  if (Qmax <= SQ_N && k <= 32 && prm.kb_count <= SQ_MAXKB) {
+    // Small batch: corpus as the M operand, queries resident (swap-AB).
+    CUtensorMap mq16, mc128;
+    if (!make_map(&mq16, queries, Qmax, d, SQ_N) || !make_map(&mc128, corpus, N, d, SQ_BM))
+      return fail(HS_ERR_CUDA, "cuTensorMapEncodeTiled failed (driver entry point or arguments)");
+    static bool sq_configured = false;
+    if (!sq_configured) {
+      const cudaError_t e = cudaFuncSetAttribute(
+          retrieve_small_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SQ_SMEM);
+      if (e != cudaSuccess) return cuda_fail(e, "retrieve smem attribute");
+      sq_configured = true;
+    }
+    // Lists per query = 2 * nsplit of the plan the merge kernel recomputes
+    // (one query block, one group: nsplit = min(slots, tiles, 8192 / k)).
+    prm.slots = (int32_t)std::max<int64_t>(1, sms / 2);
+    prm.cl = 1;
+    const SplitPlan sp = split_plan(1, tiles, k, prm.slots, 1);
+    const int64_t grid = 2 * (int64_t)sp.nsplit;
+    retrieve_small_kernel<<<(unsigned)grid, SQ_THREADS, SQ_SMEM, stream>>>(
+        mq16, mc128, prm, (N + SQ_BM - 1) / SQ_BM);
+    st = cuda_fail(cudaGetLastError(), "retrieve launch");
+  } else if (k <= 16) {
     st = launch_variant<16>(corpus, N, d, mq, prm, stream);
   } else if (k <= 32) {
     st = launch_variant<32>(corpus, N, d, mq, prm, stream);

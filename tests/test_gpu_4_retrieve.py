@@ -262,3 +262,35 @@ def test_shared_floor_keeps_ties_across_splits():
     os_, oi = oracle.topk(Q, C, k)
     assert (gi == oi).all()
     parity(Q, C, k, gs, gi, range(nq))
+
+
+@pytest.mark.parametrize("nq,N,d,k", [
+    (1, 50000, 768, 10),      # one query, ragged last 128-row tile
+    (16, 20000, 1024, 32),    # a full batch of 16, largest k and d of the small path
+    (7, 777, 72, 5),          # d not a multiple of 64, few tiles
+    (2, 130, 128, 1),         # two tiles, k = 1
+])
+def test_small_batch_path(nq, N, d, k):
+    Q, C = unit_pair(nq, N, d, nq * 11 + N)
+    gs, gi = gpu_topk(to_dev(Q), to_dev(C), k)
+    parity(Q, C, k, gs, gi, range(nq))
+
+
+def test_small_batch_ties_and_device_count():
+    nq, N, d, k = 16, 60000, 256, 10
+    Q, C = unit_pair(nq, N, d, 41)
+    rng = np.random.default_rng(5)
+    for q in range(nq):
+        C[np.sort(rng.choice(N, size=25, replace=False))] = Q[q]
+    Qd, Cd = to_dev(Q), to_dev(C)
+    os_, oi = oracle.topk(Q, C, k)
+    gs, gi = gpu_topk(Qd, Cd, k)
+    assert (gi == oi).all()
+    for cnt_ in (0, 5, 16):
+        s = torch.full((nq, k), -7.0, device="cuda")
+        i = torch.full((nq, k), -7, dtype=torch.int32, device="cuda")
+        hs.hs_retrieve_topk_n(Qd, torch.tensor([cnt_], dtype=torch.int32, device="cuda"), Cd, k,
+                              out=(s, i))
+        hs.hs_get_device_error()
+        assert (i[:cnt_].cpu().numpy() == oi[:cnt_]).all()
+        assert (i[cnt_:] == -7).all()
