@@ -195,7 +195,7 @@ __device__ __forceinline__ void list_insert(float (&ls)[KREG], int32_t (&li)[KRE
 
 // ---- large-k helpers (per thread, serial) ---------------------------------------------
 __device__ void flush_candidates(float* cs, int32_t* ci, int et, int& cnt, float* Ls, int32_t* Li,
-                                 int k, int& cur, float& theta, float floor_theta) {
+                                 int k, int& cur, float& theta, float floor_theta, float& kth) {
   if (cnt == 0) return;
   // Stable insertion sort of the buffer, score descending (buffer order is
   // ascending corpus index, so ties keep the lower index first).
@@ -273,7 +273,8 @@ __device__ void flush_candidates(float* cs, int32_t* ci, int et, int& cnt, float
     }
   }
   cur ^= 1;
-  theta = fmaxf(last, floor_theta);  // the k-th entry of the new list, not below the floor
+  kth = last;                        // the k-th entry of the new list (-FLT_MAX if not full)
+  theta = fmaxf(last, floor_theta);  // ... not below the floor
   cnt = 0;
 }
 
@@ -468,7 +469,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       // (another list may hold an equal score at a higher index).
       uint32_t qf_seen = 0;
       float qf_theta = -FLT_MAX;
-      if (KREG > 0 && valid_q && p.qfloor) {   // lists of other splits may have set it
+      float list_kth = -FLT_MAX;               // large k: this list's k-th best so far
+      if (valid_q && p.qfloor) {               // lists of other splits may have set it
         qf_seen = *reinterpret_cast<volatile uint32_t*>(p.qfloor + q);
         if (qf_seen) qf_theta = nextafterf(code_float(qf_seen), -INFINITY);
       }
@@ -482,7 +484,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t acc = tile_i & 1u, aphase = (tile_i >> 1) & 1u;
         if (!mbar_wait(tfull + acc, aphase, abort_flag)) goto epi_done;
         tc_fence_after();
-        if (KREG > 0) theta = fmaxf(theta, qf_theta);
+        theta = fmaxf(theta, qf_theta);
         const int64_t col0 = t * BN + half * kHalfCols;
         const bool tail = col0 + kHalfCols > p.N;
         // One 32-column chunk: mask columns past N / invalid queries, then
@@ -540,7 +542,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                   }
                 }
                 if (__any_sync(0xffffffffu, cnt > kCap - 4))
-                  flush_candidates(cand_s, cand_i, et, cnt, Ls, Li, k, cur, theta, floor_theta);
+                  flush_candidates(cand_s, cand_i, et, cnt, Ls, Li, k, cur, theta,
+                                   fmaxf(floor_theta, qf_theta), list_kth);
               }
             }
           }
@@ -566,10 +569,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tc_fence_before();
         __syncwarp();
-        if (KREG > 0 && valid_q && p.qfloor) {
+        if (valid_q && p.qfloor) {
           // Publish this list's k-th best if it raises the query's floor,
           // and fetch the floor for the next tile.
-          const float kth = ls[(KREG > 0 ? KREG : 1) - 1];
+          const float kth = KREG > 0 ? ls[(KREG > 0 ? KREG : 1) - 1] : list_kth;
           const uint32_t mine = kth > -FLT_MAX ? float_code(kth) : 0u;
           if (mine > qf_seen) atomicMax(p.qfloor + q, mine);
           const uint32_t c = *reinterpret_cast<volatile uint32_t*>(p.qfloor + q);
@@ -597,7 +600,8 @@ __global__ void __launch_bounds__(kThreads, 1)
               oi[i - (KREG - k)] = li[i];
             }
         } else {
-          flush_candidates(cand_s, cand_i, et, cnt, Ls, Li, k, cur, theta, floor_theta);
+          flush_candidates(cand_s, cand_i, et, cnt, Ls, Li, k, cur, theta,
+                           fmaxf(floor_theta, qf_theta), list_kth);
           for (int i = 0; i < k; ++i) {
             os[i] = Ls[(size_t)cur * k + i];
             oi[i] = Li[(size_t)cur * k + i];
@@ -1252,6 +1256,9 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
       prm.floor = scores_out;
       prm.floor_stride = k;
       prm.floor_index = k - 1;
+      // Pass 1's shared floors bound 32nd-best scores, not k-th best: clear.
+      const cudaError_t ze2 = cudaMemsetAsync(prm.qfloor, 0, (size_t)Qmax * 4, stream);
+      if (ze2 != cudaSuccess) return cuda_fail(ze2, "floor clear");
     }
     st = launch_variant<0>(corpus, N, d, mq, prm, stream);
   }
