@@ -162,17 +162,24 @@ __device__ __forceinline__ void unit_coords(const SplitPlan& sp, int64_t tiles, 
   t1 = (int64_t)(split + 1) * tiles / sp.nsplit;
 }
 
-// Maximum of 32 scores as a 5-level tree (fmaxf is exact, so the order does
-// not change the result).
+__device__ __forceinline__ float max3f(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
+
+// Maximum of 32 scores as a tree of three-input maxima (17 operations; the
+// maximum is exact, so the order does not change the result).
 __device__ __forceinline__ float chunk_max(const uint32_t (&r)[32]) {
-  float m[16];
+  float m[11];
 #pragma unroll
-  for (int j = 0; j < 16; ++j) m[j] = fmaxf(__uint_as_float(r[j]), __uint_as_float(r[j + 16]));
-#pragma unroll
-  for (int w = 8; w > 0; w >>= 1)
-#pragma unroll
-    for (int j = 0; j < w; ++j) m[j] = fmaxf(m[j], m[j + w]);
-  return m[0];
+  for (int j = 0; j < 10; ++j)
+    m[j] = max3f(__uint_as_float(r[3 * j]), __uint_as_float(r[3 * j + 1]),
+                 __uint_as_float(r[3 * j + 2]));
+  m[10] = fmaxf(__uint_as_float(r[30]), __uint_as_float(r[31]));
+  const float a = max3f(m[0], m[1], m[2]), b = max3f(m[3], m[4], m[5]);
+  const float c = max3f(m[6], m[7], m[8]), e = fmaxf(m[9], m[10]);
+  return fmaxf(max3f(a, b, c), e);
 }
 
 // Insert (s, idx) into a list sorted by score descending.  idx is larger than
