@@ -453,6 +453,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       unit_coords(sp, p.tiles, u, rank, CL, qb, split, t0, t1);
       const int64_t q = (int64_t)qb * BM + row;
       const bool valid_q = q < Q;
+      const bool warp_has_query = __any_sync(0xffffffffu, valid_q);
       // Large k: start from the query's floor (a lower bound on its final k-th
       // best score), so only scores that can still make the top k are kept.
       float floor_theta = -FLT_MAX;
@@ -503,13 +504,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int j = 0; j < 32; ++j)
               if ((int64_t)cbase + j >= p.N) r[j] = __float_as_uint(-FLT_MAX);
           }
-          if (!valid_q) {
-#pragma unroll
-            for (int j = 0; j < 32; ++j) r[j] = __float_as_uint(-FLT_MAX);
-          }
           if (KREG > 0) {
             float mx = chunk_max(r);
-            const bool any = mx > theta;
+            const bool any = valid_q && mx > theta;   // padding query rows never insert
             if (__any_sync(0xffffffffu, any)) {
               uint32_t m = 0;
               if (any) {
@@ -536,13 +533,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             // Same first test as above: a chunk whose maximum beats no
             // lane's threshold costs one max-reduction and a vote.
             const float mx = chunk_max(r);
-            if (__any_sync(0xffffffffu, mx > theta)) {
+            if (__any_sync(0xffffffffu, valid_q && mx > theta)) {
 #pragma unroll
               for (int j0 = 0; j0 < 32; j0 += 4) {
 #pragma unroll
                 for (int j = j0; j < j0 + 4; ++j) {
                   const float s = __uint_as_float(r[j]);
-                  if (s > theta) {
+                  if (valid_q && s > theta) {
                     cand_s[cnt * kEpi + et] = s;
                     cand_i[cnt * kEpi + et] = cbase + j;
                     ++cnt;
@@ -557,8 +554,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                 };
         // Register lists: two chunks per TMEM round trip (both loads, one
         // wait).  Large k keeps one, as its candidate path needs the registers.
+        // A warp whose 32 query rows are all padding has nothing to read.
 #pragma unroll 1
-        for (int c = 0; c < kHalfCols / 32; c += (KREG > 0 ? 2 : 1)) {
+        for (int c = 0; c < kHalfCols / 32 && warp_has_query; c += (KREG > 0 ? 2 : 1)) {
           const uint32_t ta = tmem_base + lane_addr + acc * BN + half * kHalfCols + c * 32;
           uint32_t ra[32];
           if (KREG > 0) {
@@ -1236,6 +1234,10 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
     retrieve_small_kernel<<<(unsigned)grid, SQ_THREADS, SQ_SMEM, stream>>>(
         mq16, mc128, prm, (N + SQ_BM - 1) / SQ_BM);
     st = cuda_fail(cudaGetLastError(), "retrieve launch");
+  } else if (k <= 8) {
+    st = launch_variant<8>(corpus, N, d, mq, prm, stream);
+  } else if (k <= 12) {
+    st = launch_variant<12>(corpus, N, d, mq, prm, stream);
   } else if (k <= 16) {
     st = launch_variant<16>(corpus, N, d, mq, prm, stream);
   } else if (k <= 32) {
