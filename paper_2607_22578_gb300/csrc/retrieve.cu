@@ -495,8 +495,38 @@ __global__ void __launch_bounds__(kThreads, 1)
         theta = fmaxf(theta, qf_theta);
         const int64_t col0 = t * BN + half * kHalfCols;
         const bool tail = col0 + kHalfCols > p.N;
-        // One 32-column chunk: mask columns past N / invalid queries, then
-        // the threshold test and candidate handling.
+        // Register lists: the candidates of the staged chunk (if any) of every
+        // lane, inserted in one converged loop (the warp pays for the largest
+        // candidate count of a lane); thresholds are re-read per insert.
+        bool pending = false;
+        int32_t pending_base = 0;
+        auto drain = [&]() {
+          uint32_t m = 0;
+          if (pending) {
+#pragma unroll
+            for (int v = 0; v < 8; ++v) {
+              const uint4 x = reinterpret_cast<const uint4*>(stage_f)[v * kEpi + et];
+              m |= (__uint_as_float(x.x) > theta ? 1u : 0u) << (4 * v);
+              m |= (__uint_as_float(x.y) > theta ? 1u : 0u) << (4 * v + 1);
+              m |= (__uint_as_float(x.z) > theta ? 1u : 0u) << (4 * v + 2);
+              m |= (__uint_as_float(x.w) > theta ? 1u : 0u) << (4 * v + 3);
+            }
+          }
+          const int most = __reduce_max_sync(0xffffffffu, (unsigned)__popc(m));
+          for (int it = 0; it < most; ++it) {
+            const int j = m ? __ffs(m) - 1 : 0;
+            const float sc = m ? stage_f[((j >> 2) * kEpi + et) * 4 + (j & 3)] : -FLT_MAX;
+            m &= m - 1;
+            if (sc > theta) {
+              list_insert<(KREG > 0 ? KREG : 1)>(ls, li, sc, pending_base + j);
+              theta = fmaxf(ls[(KREG > 0 ? KREG : 1) - 1], qf_theta);
+            }
+          }
+          pending = false;
+          __syncwarp();
+        };
+        // One 32-column chunk: mask columns past N, then the threshold test
+        // and candidate handling.
         auto do_chunk = [&](uint32_t(&r)[32], int c) {
           const int32_t cbase = (int32_t)(col0 + c * 32);
           if (tail) {                           // zero-filled rows past N never qualify
@@ -505,9 +535,27 @@ __global__ void __launch_bounds__(kThreads, 1)
               if ((int64_t)cbase + j >= p.N) r[j] = __float_as_uint(-FLT_MAX);
           }
           if (KREG > 0) {
-            float mx = chunk_max(r);
+            // A chunk with a candidate is staged in the lane's slot; drain()
+            // inserts the staged candidates of all lanes in one converged
+            // loop.  Long lists (32 slots, costly inserts) defer it to the end
+            // of the tile, so the lanes' candidates of several chunks share
+            // one pass (a lane whose slot is taken drains first); short lists
+            // drain at once.
+            const float mx = chunk_max(r);
             const bool any = valid_q && mx > theta;   // padding query rows never insert
-            if (__any_sync(0xffffffffu, any)) {
+            if (KREG >= 32) {
+              if (__any_sync(0xffffffffu, any && pending)) drain();
+              if (any) {
+#pragma unroll
+                for (int v = 0; v < 8; ++v)
+                  reinterpret_cast<uint4*>(stage_f)[v * kEpi + et] =
+                      make_uint4(r[4 * v], r[4 * v + 1], r[4 * v + 2], r[4 * v + 3]);
+                pending = true;
+                pending_base = cbase;
+              }
+            } else if (__any_sync(0xffffffffu, any)) {
+              // Short lists: this chunk's candidates at once, the mask built
+              // from the registers.
               uint32_t m = 0;
               if (any) {
 #pragma unroll
@@ -520,10 +568,10 @@ __global__ void __launch_bounds__(kThreads, 1)
               const int most = __reduce_max_sync(0xffffffffu, (unsigned)__popc(m));
               for (int it = 0; it < most; ++it) {
                 const int j = m ? __ffs(m) - 1 : 0;
-                const float s = m ? stage_f[((j >> 2) * kEpi + et) * 4 + (j & 3)] : -FLT_MAX;
+                const float sc = m ? stage_f[((j >> 2) * kEpi + et) * 4 + (j & 3)] : -FLT_MAX;
                 m &= m - 1;
-                if (s > theta) {
-                  list_insert<(KREG > 0 ? KREG : 1)>(ls, li, s, cbase + j);
+                if (sc > theta) {
+                  list_insert<(KREG > 0 ? KREG : 1)>(ls, li, sc, cbase + j);
                   theta = fmaxf(ls[(KREG > 0 ? KREG : 1) - 1], qf_theta);
                 }
               }
@@ -572,6 +620,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             do_chunk(ra, c);
           }
         }
+        if (KREG >= 32 && __any_sync(0xffffffffu, pending)) drain();
         tc_fence_before();
         __syncwarp();
         if (valid_q && p.qfloor) {
