@@ -294,3 +294,15 @@ def test_small_batch_ties_and_device_count():
         hs.hs_get_device_error()
         assert (i[:cnt_].cpu().numpy() == oi[:cnt_]).all()
         assert (i[cnt_:] == -7).all()
+
+
+@pytest.mark.parametrize("nq,N,d,k", [
+    (4, 40, 128, 10),         # small-batch path, corpus shorter than one 128-row tile
+    (300, 200, 256, 10),      # CTA pairs, corpus shorter than one 256-row tile
+    (260, 300, 64, 20),       # CTA pairs, 2 tiles, odd query-block count, 32-slot lists
+    (129, 1000, 768, 12),     # two query blocks (one pair), 12-slot lists, k = 12
+])
+def test_tiny_corpus_edges(nq, N, d, k):
+    Q, C = unit_pair(nq, N, d, nq + 3 * N)
+    gs, gi = gpu_topk(to_dev(Q), to_dev(C), k)
+    parity(Q, C, k, gs, gi, range(nq))
