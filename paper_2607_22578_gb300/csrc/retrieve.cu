@@ -600,14 +600,15 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
           }
                 };
-        // Register lists: two chunks per TMEM round trip (both loads, one
-        // wait).  Large k keeps one, as its candidate path needs the registers.
+        // Lists of up to 16 slots: two chunks per TMEM round trip (both loads,
+        // one wait).  Longer lists and large k keep one: they need the
+        // registers.
         // A warp whose 32 query rows are all padding has nothing to read.
 #pragma unroll 1
-        for (int c = 0; c < kHalfCols / 32 && warp_has_query; c += (KREG > 0 ? 2 : 1)) {
+        for (int c = 0; c < kHalfCols / 32 && warp_has_query; c += (KREG > 0 && KREG < 32 ? 2 : 1)) {
           const uint32_t ta = tmem_base + lane_addr + acc * BN + half * kHalfCols + c * 32;
           uint32_t ra[32];
-          if (KREG > 0) {
+          if (KREG > 0 && KREG < 32) {
             uint32_t rb[32];
             tmem_ld_32x32b_x32(ta, ra);
             tmem_ld_32x32b_x32(ta + 32, rb);
