@@ -540,6 +540,17 @@ def row_batch_sweep(args, dev, peaks) -> dict:
                 lat.append(e0.elapsed_time(e1))
                 ret.append(r0.elapsed_time(r1))
                 nus.append(nu)
+        # The same batches through the captured query path (one launch).
+        graph = hs.RetrieveGraph(stage, B)
+        glat = []
+        for i, q in enumerate(batches):
+            e0, e1 = _ev(), _ev()
+            e0.record()
+            graph.run(q)
+            e1.record()
+            torch.cuda.synchronize()
+            if i >= 3:
+                glat.append(e0.elapsed_time(e1))
         hs.hs_get_device_error()
         qu = float(np.mean(nus))
         t_ret = float(np.mean(ret))
@@ -548,6 +559,9 @@ def row_batch_sweep(args, dev, peaks) -> dict:
             "merged_queries_mean": qu, "latency_ms_p50": float(np.percentile(lat, 50)),
             "latency_ms_p99": float(np.percentile(lat, 99)),
             "queries_per_s": B * len(lat) / (sum(lat) / 1e3),
+            "graph_latency_ms_p50": float(np.percentile(glat, 50)),
+            "graph_latency_ms_p99": float(np.percentile(glat, 99)),
+            "graph_queries_per_s": B * len(glat) / (sum(glat) / 1e3),
             "retrieval": _roof(rb, 2.0 * qu * N * d, t_ret, peaks)}
         del batches
     return out

@@ -9,7 +9,7 @@ from ._lib import (HS_ERR_CUDA, HS_ERR_INVALID_ARG, HS_ERR_TIMEOUT, HS_ERR_UNSUP
                    hs_retrieve_topk_workspace, hs_scatter_results, hs_unique_inverse,
                    hs_unique_inverse_noalloc,
                    hs_unique_inverse_workspace, hs_version, library_path, load)
-from .pipeline import EmbedRetrieveStage, HostFeed, StepGraph
+from .pipeline import EmbedRetrieveStage, HostFeed, RetrieveGraph, StepGraph
 
 __all__ = [
     "HS_OK", "HS_ERR_INVALID_ARG", "HS_ERR_UNSUPPORTED", "HS_ERR_CUDA", "HS_ERR_WORKSPACE",

@@ -147,6 +147,35 @@ class StepGraph:
         return self.outputs
 
 
+class RetrieveGraph:
+    """The query path of a stage — fingerprint, unique, gather, retrieval,
+    result scatter — captured as one CUDA graph for batches of exactly
+    ``n_queries`` queries (serving pads batches to a few such sizes).
+
+    ``run(queries)`` copies the batch into the captured input buffer and
+    replays the graph: one launch for the whole path instead of one host
+    call per kernel.  Returns the stage's (scores, ids, n_unique) buffers,
+    which the next run overwrites."""
+
+    def __init__(self, stage: "EmbedRetrieveStage", n_queries: int):
+        if n_queries > stage.max_queries:
+            raise ValueError("batch larger than the stage's max_queries")
+        self.queries = torch.zeros((n_queries, stage.d), dtype=stage.corpus.dtype,
+                                   device=stage.device)
+        stage.retrieve(self.queries)           # one-time host work outside the capture
+        torch.cuda.synchronize(stage.device)
+        self.graph = torch.cuda.CUDAGraph()
+        l0 = _lib.hs_launch_count()
+        with torch.cuda.graph(self.graph):
+            self.outputs = stage.retrieve(self.queries)
+        self.launches = _lib.hs_launch_count() - l0
+
+    def run(self, queries: torch.Tensor):
+        self.queries.copy_(queries, non_blocking=True)
+        self.graph.replay()
+        return self.outputs
+
+
 class HostFeed:
     """Runs batches that live in (pinned) host memory through a stage, with
     the next batch's host-to-device copy overlapping the current batch's

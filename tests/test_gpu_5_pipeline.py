@@ -110,3 +110,17 @@ def test_step_graph_replays_match_eager_step():
     hs.hs_get_device_error()
     assert torch.equal(s2, s3.cpu()) and torch.equal(i2, i3.cpu())
     assert not torch.equal(s2, ref[3])   # the reversed batch has different results
+
+
+def test_retrieve_graph_matches_eager_retrieve():
+    import torch
+    w = configs.build_retrieval_mix(configs.TINY)
+    stage = hs.EmbedRetrieveStage(to_dev(w["corpus"]), w["k"], max_queries=len(w["queries"]))
+    g = hs.RetrieveGraph(stage, len(w["queries"]))
+    for qs in (w["queries"], w["queries"][::-1].copy()):
+        qd = to_dev(qs)
+        s, i, nu = g.run(qd)
+        s, i, nu = s.cpu(), i.cpu(), int(nu.item())
+        s2, i2, nu2 = stage.retrieve(qd)
+        hs.hs_get_device_error()
+        assert nu == int(nu2.item()) and torch.equal(s, s2.cpu()) and torch.equal(i, i2.cpu())
