@@ -612,7 +612,7 @@ def rag_mix_breakdown(stage, tokens, queries, K: int) -> dict:
     import paper_2607_22578_gb300 as hs
     from paper_2607_22578_gb300 import _lib
     names = ["chunk_fingerprint", "chunk_unique", "query_fingerprint", "query_unique",
-             "gather_unique_queries", "retrieve_topk", "scatter_results"]
+             "gather_unique_queries", "retrieve_topk_fanout"]
     acc = {n: 0.0 for n in names}
     Q = queries.shape[0]
     for _ in range(K):
@@ -629,12 +629,9 @@ def rag_mix_breakdown(stage, tokens, queries, K: int) -> dict:
         ev[4].record()
         uq = _lib.hs_scatter_results(queries, uidx, dst=stage.uq[:Q])
         ev[5].record()
-        s_u, i_u = _lib.hs_retrieve_topk_n(uq, nu, stage.corpus, stage.k, workspace=stage.ws_r,
-                                           out=(stage.s_u[:Q], stage.i_u[:Q]))
+        _lib.hs_retrieve_topk_fanout(uq, nu, inv, stage.corpus, stage.k, workspace=stage.ws_r,
+                                     out=(stage.scores[:Q], stage.ids[:Q]))
         ev[6].record()
-        _lib.hs_scatter_results(s_u, inv, dst=stage.scores[:Q])
-        _lib.hs_scatter_results(i_u, inv, dst=stage.ids[:Q])
-        ev[7].record()
         torch.cuda.synchronize()
         for i, n in enumerate(names):
             acc[n] += ev[i].elapsed_time(ev[i + 1])

@@ -7,6 +7,9 @@
  *   hs_unique_inverse   merge exactly-equal rows into unique nodes + inverse map
  *   hs_retrieve_topk    score merged queries against a corpus, keep top-k
  *   hs_scatter_results  fan each kept result back out to every merged row
+ * and two fused forms for latency-bound batches:
+ *   hs_merge_queries         fingerprint + merge + gather of a query batch
+ *   hs_retrieve_topk_fanout  retrieval whose results go to every merged row
  *
  * Conventions shared by every call
  *   - Pointers named *_dev or documented as device pointers must be device
@@ -51,6 +54,9 @@ typedef enum {
 
 /* Largest k accepted by hs_retrieve_topk. */
 #define HS_TOPK_MAX_K 1024
+
+/* Largest batch accepted by hs_merge_queries. */
+#define HS_MERGE_QUERIES_MAX 256
 
 /* Human-readable description of the last error returned on this host
  * thread ("" if none).  The string stays valid until the next hs_* call on
@@ -203,6 +209,69 @@ hs_status hs_retrieve_topk_n(const uint16_t* queries, int64_t max_queries,
                              int64_t n_corpus, int32_t dim, int32_t k, float* scores_out,
                              int32_t* ids_out, void* workspace, size_t workspace_bytes,
                              hs_stream_t stream);
+
+/*
+ * hs_retrieve_topk_fanout — hs_retrieve_topk_n whose results go straight to
+ * every row merged into each query: row o of scores_out / ids_out holds the
+ * top-k of query inverse[o].
+ *
+ * Paper: Section 3.3 (I) and Appendix A.2: a merged node executes once and
+ * its output flows to the downstream nodes of every node merged into it.
+ * The result equals hs_retrieve_topk_n followed by hs_scatter_results of the
+ * scores and of the ids with map = inverse, without the intermediate
+ * per-query rows: the final merge of the retrieval writes the fanned-out
+ * rows itself.
+ *
+ * n_queries_dev  device int32 scalar or NULL (NULL: max_queries queries).
+ * inverse        device int32 [n_out]; an entry outside [0, query count)
+ *                sets the device error word (HS_ERR_INVALID_ARG) and leaves
+ *                that output row unwritten.
+ * n_out          >= 0 (0: nothing enqueued); max_queries >= 1 if n_out > 0.
+ * scores_out     device float [n_out, k]; ids_out device int32 [n_out, k].
+ * Every other argument is as for hs_retrieve_topk_n (same workspace size).
+ */
+hs_status hs_retrieve_topk_fanout(const uint16_t* queries, int64_t max_queries,
+                                  const int32_t* n_queries_dev, const int32_t* inverse,
+                                  int64_t n_out, const uint16_t* corpus, int64_t n_corpus,
+                                  int32_t dim, int32_t k, float* scores_out, int32_t* ids_out,
+                                  void* workspace, size_t workspace_bytes, hs_stream_t stream);
+
+/*
+ * hs_merge_queries — the query side of a small batch in one launch:
+ * fingerprint, exact merge and gather of the unique query vectors.
+ *
+ * Paper: Section 3.3, Eq. 2 (the signature of a node) and "Dynamic Fusion
+ * and Reuse Mechanism" (I) (a node equal to one already in the window is
+ * merged into it); Appendix A.2 (merge sets M(v*) executed once).
+ * The outputs are exactly those of
+ *   hs_fingerprint(queries as int32 words, n_queries, dim / 2, NULL,
+ *                  seed_state, fp_out)
+ *   hs_unique_inverse(fp, ..., n_unique_dev, unique_idx_out, inverse_out)
+ *   hs_scatter_results(queries, unique_idx_out -> unique_queries_out)
+ * with the gather limited to the first *n_unique_dev rows.  One kernel, no
+ * workspace: meant for the latency-bound batches of an online stage.
+ *
+ * queries             device bf16 bits (uint16) [n_queries, dim] row-major,
+ *                     16-byte aligned.
+ * n_queries           0 <= n_queries <= HS_MERGE_QUERIES_MAX (0 writes
+ *                     *n_unique_dev = 0 and nothing else).
+ * dim                 8 <= dim <= 16384, dim % 8 == 0.
+ * seed_state          FNV-1a seed, as for hs_fingerprint.
+ * fp_in               device uint64 [n_queries] or NULL.  NULL: fingerprints
+ *                     are computed here.  Otherwise these fingerprints are
+ *                     used as given (they must be equal for equal rows, as
+ *                     hs_unique_inverse requires; for instance fingerprints
+ *                     carried from an earlier stage).
+ * fp_out              device uint64 [n_queries] or NULL: the fingerprints used.
+ * n_unique_dev, unique_idx_out, inverse_out   as for hs_unique_inverse.
+ * unique_queries_out  device uint16 [n_queries, dim], 16-byte aligned, not
+ *                     overlapping queries: row u < *n_unique_dev is
+ *                     queries[unique_idx_out[u]]; later rows are untouched.
+ */
+hs_status hs_merge_queries(const uint16_t* queries, int64_t n_queries, int32_t dim,
+                           uint64_t seed_state, const uint64_t* fp_in, uint64_t* fp_out,
+                           int32_t* n_unique_dev, int32_t* unique_idx_out, int32_t* inverse_out,
+                           uint16_t* unique_queries_out, hs_stream_t stream);
 
 /*
  * hs_scatter_results — row gather/scatter: dst[i, :] = src[map[i], :].

@@ -25,6 +25,7 @@ HS_ERR_WORKSPACE = 4
 HS_ERR_TIMEOUT = 5
 HS_FNV64_OFFSET_BASIS = 0xCBF29CE484222325
 HS_TOPK_MAX_K = 1024
+HS_MERGE_QUERIES_MAX = 256
 
 _STATUS = {0: "HS_OK", 1: "HS_ERR_INVALID_ARG", 2: "HS_ERR_UNSUPPORTED", 3: "HS_ERR_CUDA",
            4: "HS_ERR_WORKSPACE", 5: "HS_ERR_TIMEOUT"}
@@ -72,6 +73,11 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
             lib.hs_retrieve_topk.restype = st
             lib.hs_retrieve_topk_n.argtypes = [P, i64, P, P, i64, i32, i32, P, P, P, sz, P]
             lib.hs_retrieve_topk_n.restype = st
+            lib.hs_retrieve_topk_fanout.argtypes = [P, i64, P, P, i64, P, i64, i32, i32, P, P,
+                                                    P, sz, P]
+            lib.hs_retrieve_topk_fanout.restype = st
+            lib.hs_merge_queries.argtypes = [P, i64, i32, u64, P, P, P, P, P, P, P]
+            lib.hs_merge_queries.restype = st
             lib.hs_scatter_results.argtypes = [P, i64, i64, P, i64, P, P]
             lib.hs_scatter_results.restype = st
             lib.hs_get_device_error.argtypes = [P]
@@ -240,6 +246,74 @@ def hs_retrieve_topk_n(queries: torch.Tensor, n_queries_dev: torch.Tensor, corpu
                                      k, _ptr(scores), _ptr(ids), _ptr(workspace),
                                      workspace.numel(), _stream(stream)))
     return scores, ids
+
+
+def hs_retrieve_topk_fanout(queries: torch.Tensor, n_queries_dev: torch.Tensor | None,
+                            inverse: torch.Tensor, corpus: torch.Tensor, k: int,
+                            workspace: torch.Tensor | None = None, out: tuple | None = None,
+                            stream=None):
+    """Retrieval whose results go to every merged row: row o of the returned
+    (scores [n_out, k], ids [n_out, k]) is the top-k of query inverse[o]
+    (n_out = inverse.numel()).  n_queries_dev (device int32 scalar) or None
+    gives the query count, as for hs_retrieve_topk_n."""
+    _cuda(queries, "queries")
+    _cuda(corpus, "corpus")
+    _cuda(inverse, "inverse")
+    if inverse.dtype != torch.int32:
+        raise TypeError("inverse must be int32")
+    if n_queries_dev is not None:
+        _cuda(n_queries_dev, "n_queries_dev")
+        if n_queries_dev.dtype != torch.int32:
+            raise TypeError("n_queries_dev must be int32")
+    if queries.element_size() != 2 or corpus.element_size() != 2:
+        raise TypeError("queries and corpus must hold bf16 (2-byte) elements")
+    Q, d = queries.shape
+    N, d2 = corpus.shape
+    if d != d2:
+        raise ValueError("dimension mismatch")
+    n_out = inverse.numel()
+    dev = queries.device
+    if out is None:
+        out = (torch.empty((n_out, k), dtype=torch.float32, device=dev),
+               torch.empty((n_out, k), dtype=torch.int32, device=dev))
+    scores, ids = out
+    if workspace is None:
+        workspace = torch.empty(hs_retrieve_topk_workspace(Q, N, d, k), dtype=torch.uint8,
+                                device=dev)
+    _check(load().hs_retrieve_topk_fanout(_ptr(queries), Q, _ptr(n_queries_dev), _ptr(inverse),
+                                          n_out, _ptr(corpus), N, d, k, _ptr(scores), _ptr(ids),
+                                          _ptr(workspace), workspace.numel(), _stream(stream)))
+    return scores, ids
+
+
+def hs_merge_queries(queries: torch.Tensor, seed_state: int = HS_FNV64_OFFSET_BASIS,
+                     fp_in: torch.Tensor | None = None, out: tuple | None = None, stream=None):
+    """Fingerprint, exact merge and gather of a query batch (at most
+    HS_MERGE_QUERIES_MAX rows of bf16 vectors) in one launch.  Returns
+    (fp [n] int64, n_unique_dev [1] int32, unique_idx [n] int32,
+    inverse [n] int32, unique_queries [n, dim]); the first n_unique rows of
+    unique_queries are the unique query vectors.  ``out`` may supply those
+    five tensors preallocated; ``fp_in`` replaces the computed fingerprints."""
+    _cuda(queries, "queries")
+    if queries.element_size() != 2 or queries.dim() != 2:
+        raise TypeError("queries must be a 2-D tensor of bf16 (2-byte) elements")
+    n, d = queries.shape
+    dev = queries.device
+    if fp_in is not None:
+        _cuda(fp_in, "fp_in")
+        if fp_in.dtype != torch.int64 or fp_in.numel() != n:
+            raise TypeError("fp_in must be int64 [n]")
+    if out is None:
+        out = (torch.empty(max(n, 1), dtype=torch.int64, device=dev),
+               torch.empty(1, dtype=torch.int32, device=dev),
+               torch.empty(max(n, 1), dtype=torch.int32, device=dev),
+               torch.empty(max(n, 1), dtype=torch.int32, device=dev),
+               torch.empty((max(n, 1), d), dtype=queries.dtype, device=dev))
+    fp, nu, uidx, inv, uq = out
+    _check(load().hs_merge_queries(_ptr(queries), n, d, seed_state & (2**64 - 1), _ptr(fp_in),
+                                   _ptr(fp), _ptr(nu), _ptr(uidx), _ptr(inv), _ptr(uq),
+                                   _stream(stream)))
+    return fp[:n], nu, uidx[:n], inv[:n], uq[:n]
 
 
 def hs_scatter_results(src: torch.Tensor, mapping: torch.Tensor, dst: torch.Tensor | None = None,

@@ -16,8 +16,10 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libhs.so")
-SOURCES = ["api.cu", "fingerprint.cu", "unique.cu", "scatter.cu", "retrieve.cu"]
-HEADERS = [os.path.join(CSRC, "hs_internal.cuh"), os.path.join(ROOT, "include", "hs.h")]
+SOURCES = ["api.cu", "fingerprint.cu", "unique.cu", "scatter.cu", "retrieve.cu",
+           "query_merge.cu"]
+HEADERS = [os.path.join(CSRC, h) for h in ("hs_internal.cuh", "fnv.cuh", "row_table.cuh")] + \
+    [os.path.join(ROOT, "include", "hs.h")]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC",
                 "--expt-relaxed-constexpr", "-Xptxas", "-warn-spills"]

@@ -17,8 +17,11 @@ hs_status launch_unique_inverse(const uint64_t*, const int32_t*, int64_t, int32_
                                 const int32_t*, int32_t*, int32_t*, int32_t*, void*,
                                 cudaStream_t);
 size_t retrieve_topk_workspace(int64_t, int64_t, int32_t, int32_t);
-hs_status launch_retrieve_topk(const uint16_t*, int64_t, const int32_t*, const uint16_t*, int64_t,
-                               int32_t, int32_t, float*, int32_t*, void*, size_t, cudaStream_t);
+hs_status launch_retrieve_topk(const uint16_t*, int64_t, const int32_t*, const int32_t*, int64_t,
+                               const uint16_t*, int64_t, int32_t, int32_t, float*, int32_t*,
+                               void*, size_t, cudaStream_t);
+hs_status launch_merge_queries(const uint16_t*, int64_t, int32_t, uint64_t, const uint64_t*,
+                               uint64_t*, int32_t*, int32_t*, int32_t*, uint16_t*, cudaStream_t);
 hs_status launch_scatter(const void*, int64_t, int64_t, const int32_t*, int64_t, void*,
                          cudaStream_t);
 
@@ -145,16 +148,23 @@ size_t hs_retrieve_topk_workspace(int64_t n_queries, int64_t n_corpus, int32_t d
 }
 
 static hs_status retrieve_common(const uint16_t* queries, int64_t n_queries,
-                                 const int32_t* n_queries_dev, const uint16_t* corpus,
-                                 int64_t n_corpus, int32_t dim, int32_t k, float* scores_out,
-                                 int32_t* ids_out, void* workspace, size_t workspace_bytes,
-                                 hs_stream_t stream) {
+                                 const int32_t* n_queries_dev, const int32_t* inverse,
+                                 int64_t n_out, const uint16_t* corpus, int64_t n_corpus,
+                                 int32_t dim, int32_t k, float* scores_out, int32_t* ids_out,
+                                 void* workspace, size_t workspace_bytes, hs_stream_t stream) {
   if (n_queries < 0) return fail(HS_ERR_INVALID_ARG, "n_queries < 0");
   if (n_corpus < 1 || n_corpus > 0x7fffffffLL)
     return fail(HS_ERR_INVALID_ARG, "n_corpus outside [1, 2^31 - 1]");
   if (dim < 8 || dim % 8 != 0) return fail(HS_ERR_INVALID_ARG, "dim must be >= 8 and a multiple of 8");
   if (k < 1 || (int64_t)k > n_corpus || k > HS_TOPK_MAX_K)
     return fail(HS_ERR_INVALID_ARG, "k outside [1, min(n_corpus, %d)]", HS_TOPK_MAX_K);
+  if (inverse) {
+    if (n_out < 0 || n_out > 0x7fffffffLL)
+      return fail(HS_ERR_INVALID_ARG, "n_out outside [0, 2^31 - 1]");
+    if (n_out == 0) return HS_OK;
+    if (n_queries == 0) return fail(HS_ERR_INVALID_ARG, "n_out > 0 rows but no queries");
+    if (!aligned(inverse, 4)) return fail(HS_ERR_INVALID_ARG, "inverse misaligned");
+  }
   if (n_queries == 0) return HS_OK;
   if (n_queries > 0x7fffffffLL) return fail(HS_ERR_INVALID_ARG, "n_queries >= 2^31");
   if (!queries || !corpus || !scores_out || !ids_out)
@@ -167,8 +177,8 @@ static hs_status retrieve_common(const uint16_t* queries, int64_t n_queries,
     return fail(HS_ERR_WORKSPACE, "workspace NULL or not 256-byte aligned");
   if (n_queries_dev && !aligned(n_queries_dev, 4))
     return fail(HS_ERR_INVALID_ARG, "n_queries_dev misaligned");
-  return launch_retrieve_topk(queries, n_queries, n_queries_dev, corpus, n_corpus, dim, k,
-                              scores_out, ids_out, workspace, workspace_bytes,
+  return launch_retrieve_topk(queries, n_queries, n_queries_dev, inverse, n_out, corpus,
+                              n_corpus, dim, k, scores_out, ids_out, workspace, workspace_bytes,
                               reinterpret_cast<cudaStream_t>(stream));
 }
 
@@ -177,8 +187,8 @@ hs_status hs_retrieve_topk(const uint16_t* queries, int64_t n_queries, const uin
                            int32_t* ids_out, void* workspace, size_t workspace_bytes,
                            hs_stream_t stream) {
   clear_msg();
-  return retrieve_common(queries, n_queries, nullptr, corpus, n_corpus, dim, k, scores_out,
-                         ids_out, workspace, workspace_bytes, stream);
+  return retrieve_common(queries, n_queries, nullptr, nullptr, 0, corpus, n_corpus, dim, k,
+                         scores_out, ids_out, workspace, workspace_bytes, stream);
 }
 
 hs_status hs_retrieve_topk_n(const uint16_t* queries, int64_t max_queries,
@@ -188,8 +198,52 @@ hs_status hs_retrieve_topk_n(const uint16_t* queries, int64_t max_queries,
                              hs_stream_t stream) {
   clear_msg();
   if (!n_queries_dev) return fail(HS_ERR_INVALID_ARG, "n_queries_dev is NULL");
-  return retrieve_common(queries, max_queries, n_queries_dev, corpus, n_corpus, dim, k,
-                         scores_out, ids_out, workspace, workspace_bytes, stream);
+  return retrieve_common(queries, max_queries, n_queries_dev, nullptr, 0, corpus, n_corpus, dim,
+                         k, scores_out, ids_out, workspace, workspace_bytes, stream);
+}
+
+hs_status hs_retrieve_topk_fanout(const uint16_t* queries, int64_t max_queries,
+                                  const int32_t* n_queries_dev, const int32_t* inverse,
+                                  int64_t n_out, const uint16_t* corpus, int64_t n_corpus,
+                                  int32_t dim, int32_t k, float* scores_out, int32_t* ids_out,
+                                  void* workspace, size_t workspace_bytes, hs_stream_t stream) {
+  clear_msg();
+  if (n_out < 0 || n_out > 0x7fffffffLL)
+    return fail(HS_ERR_INVALID_ARG, "n_out outside [0, 2^31 - 1]");
+  if (n_out == 0) return HS_OK;
+  if (!inverse) return fail(HS_ERR_INVALID_ARG, "inverse is NULL");
+  return retrieve_common(queries, max_queries, n_queries_dev, inverse, n_out, corpus, n_corpus,
+                         dim, k, scores_out, ids_out, workspace, workspace_bytes, stream);
+}
+
+hs_status hs_merge_queries(const uint16_t* queries, int64_t n_queries, int32_t dim,
+                           uint64_t seed_state, const uint64_t* fp_in, uint64_t* fp_out,
+                           int32_t* n_unique_dev, int32_t* unique_idx_out, int32_t* inverse_out,
+                           uint16_t* unique_queries_out, hs_stream_t stream) {
+  clear_msg();
+  if (n_queries < 0 || n_queries > HS_MERGE_QUERIES_MAX)
+    return fail(HS_ERR_INVALID_ARG, "n_queries outside [0, %d]", HS_MERGE_QUERIES_MAX);
+  if (dim < 8 || dim % 8 != 0 || dim > 16384)
+    return fail(HS_ERR_INVALID_ARG, "dim must be a multiple of 8 in [8, 16384]");
+  if (!n_unique_dev || !aligned(n_unique_dev, 4))
+    return fail(HS_ERR_INVALID_ARG, "n_unique_dev NULL or misaligned");
+  if (n_queries > 0) {
+    if (!queries || !unique_idx_out || !inverse_out || !unique_queries_out)
+      return fail(HS_ERR_INVALID_ARG, "NULL input or output pointer");
+    if (!aligned(queries, 16) || !aligned(unique_queries_out, 16))
+      return fail(HS_ERR_INVALID_ARG, "queries/unique_queries_out must be 16-byte aligned");
+    if (!aligned(unique_idx_out, 4) || !aligned(inverse_out, 4) || (fp_in && !aligned(fp_in, 8)) ||
+        (fp_out && !aligned(fp_out, 8)))
+      return fail(HS_ERR_INVALID_ARG, "misaligned pointer");
+    const uintptr_t q0 = reinterpret_cast<uintptr_t>(queries);
+    const uintptr_t u0 = reinterpret_cast<uintptr_t>(unique_queries_out);
+    const uintptr_t bytes = (uintptr_t)n_queries * (uintptr_t)dim * 2u;
+    if (q0 < u0 + bytes && u0 < q0 + bytes)
+      return fail(HS_ERR_INVALID_ARG, "queries and unique_queries_out overlap");
+  }
+  return launch_merge_queries(queries, n_queries, dim, seed_state, fp_in, fp_out, n_unique_dev,
+                              unique_idx_out, inverse_out, unique_queries_out,
+                              reinterpret_cast<cudaStream_t>(stream));
 }
 
 hs_status hs_scatter_results(const void* src, int64_t n_src, int64_t row_bytes,

@@ -100,6 +100,14 @@ struct Params {
   uint32_t* qfloor;
 };
 
+// Rows the merge writes: with inv NULL one per query (row q = query q);
+// otherwise n_out rows, row o holding the results of query inv[o] — the
+// fan-out of each merged query's results to every row merged into it.
+struct OutRows {
+  const int32_t* inv;
+  int64_t n_out;
+};
+
 __device__ __forceinline__ uint32_t float_code(float f) {
   const uint32_t u = __float_as_uint(f);
   return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
@@ -706,14 +714,20 @@ constexpr int kMaxListsPerLane = 10;
 
 __global__ void __launch_bounds__(256) merge_warp_kernel(const Params p, float* __restrict__ out_s,
                                                          int32_t* __restrict__ out_i,
-                                                         int32_t kout) {
+                                                         int32_t kout, OutRows rows) {
   const int64_t Q = query_count(p);
   const SplitPlan sp = split_plan(Q, p.tiles, p.k, p.slots, p.cl);
   const int k = p.k;
   const int lists = 2 * sp.nsplit;
   const int lane = threadIdx.x & 31;
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  for (int64_t q = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; q < Q; q += nwarps) {
+  const int64_t R = rows.inv ? rows.n_out : Q;
+  for (int64_t o = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; o < R; o += nwarps) {
+    const int64_t q = rows.inv ? (int64_t)__ldg(rows.inv + o) : o;
+    if (q < 0 || q >= Q) {                         // warp-uniform
+      if (lane == 0) set_error(p.err, kErrInvalidArg);
+      continue;
+    }
     const float* __restrict__ ps = p.part_s + (size_t)q * lists * k;
     const int32_t* __restrict__ pi = p.part_i + (size_t)q * lists * k;
     uint64_t head[kMaxListsPerLane], next[kMaxListsPerLane];
@@ -760,15 +774,18 @@ __global__ void __launch_bounds__(256) merge_warp_kernel(const Params p, float* 
       }
     }
     if (lane < kout) {
-      out_s[(size_t)q * kout + lane] = my_s;
-      out_i[(size_t)q * kout + lane] = my_i;
+      out_s[(size_t)o * kout + lane] = my_s;
+      out_i[(size_t)o * kout + lane] = my_i;
     }
   }
 }
 
 // Lists of p.k entries per (query, split, half) -> the kout best per query.
+// With out_i NULL only the kout-th best score of each query is written, to
+// out_s[q] (the floor of the second large-k pass).
 __global__ void __launch_bounds__(256) merge_kernel(const Params p, float* __restrict__ out_s,
-                                                    int32_t* __restrict__ out_i, int32_t kout) {
+                                                    int32_t* __restrict__ out_i, int32_t kout,
+                                                    OutRows rows) {
   extern __shared__ uint64_t keys[];
   const int64_t Q = query_count(p);
   const SplitPlan sp = split_plan(Q, p.tiles, p.k, p.slots, p.cl);
@@ -779,7 +796,13 @@ __global__ void __launch_bounds__(256) merge_kernel(const Params p, float* __res
   while (p2 < m) p2 <<= 1;
   const float* __restrict__ part_s = p.part_s;
   const int32_t* __restrict__ part_i = p.part_i;
-  for (int64_t q = blockIdx.x; q < Q; q += gridDim.x) {
+  const int64_t R = rows.inv ? rows.n_out : Q;
+  for (int64_t o = blockIdx.x; o < R; o += gridDim.x) {
+    const int64_t q = rows.inv ? (int64_t)__ldg(rows.inv + o) : o;
+    if (q < 0 || q >= Q) {                         // block-uniform
+      if (threadIdx.x == 0) set_error(p.err, kErrInvalidArg);
+      continue;
+    }
     const float* ps = part_s + (size_t)q * m;
     const int32_t* pi = part_i + (size_t)q * m;
     for (int e = threadIdx.x; e < p2; e += blockDim.x) keys[e] = e < m ? pack_key(ps[e], pi[e]) : 0ull;
@@ -800,12 +823,21 @@ __global__ void __launch_bounds__(256) merge_kernel(const Params p, float* __res
         __syncthreads();
       }
     }
-    for (int j = threadIdx.x; j < kout; j += blockDim.x) {
-      float s = -FLT_MAX;
-      int32_t idx = -1;
-      if (j < m) unpack_key(keys[j], s, idx);
-      out_s[(size_t)q * kout + j] = s;
-      out_i[(size_t)q * kout + j] = idx;
+    if (!out_i) {
+      if (threadIdx.x == 0) {
+        float s = -FLT_MAX;
+        int32_t idx = -1;
+        if (kout - 1 < m) unpack_key(keys[kout - 1], s, idx);
+        out_s[o] = s;
+      }
+    } else {
+      for (int j = threadIdx.x; j < kout; j += blockDim.x) {
+        float s = -FLT_MAX;
+        int32_t idx = -1;
+        if (j < m) unpack_key(keys[j], s, idx);
+        out_s[(size_t)o * kout + j] = s;
+        out_i[(size_t)o * kout + j] = idx;
+      }
     }
     __syncthreads();
   }
@@ -1203,16 +1235,17 @@ size_t retrieve_topk_workspace(int64_t Q, int64_t N, int32_t d, int32_t k) {
   const size_t part = (((size_t)Q * 2 * ns * k * 4) + 255) & ~(size_t)255;
   const size_t list = k <= 32 ? 0 : ((((size_t)sms * kEpi * 2 * k * 4) + 255) & ~(size_t)255);
   const size_t qfloor = (((size_t)Q * 4) + 255) & ~(size_t)255;
-  return 2 * part + 2 * list + qfloor + 256;
+  return 2 * part + 2 * list + 2 * qfloor + 256;   // shared floors + large-k floors
 }
 
 // Qmax rows of `queries` are addressable; the kernels process the first
 // count of them, count = *count_dev (clamped to [0, Qmax]) or Qmax if
-// count_dev is NULL.
+// count_dev is NULL.  With inv NULL, scores_out / ids_out get one row per
+// query; otherwise n_out rows, row o holding the results of query inv[o].
 hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int32_t* count_dev,
-                               const uint16_t* corpus, int64_t N, int32_t d, int32_t k,
-                               float* scores_out, int32_t* ids_out, void* ws, size_t ws_bytes,
-                               cudaStream_t stream) {
+                               const int32_t* inv, int64_t n_out, const uint16_t* corpus,
+                               int64_t N, int32_t d, int32_t k, float* scores_out,
+                               int32_t* ids_out, void* ws, size_t ws_bytes, cudaStream_t stream) {
   unsigned* err = device_error_word();
   if (!err) return fail(HS_ERR_CUDA, "could not resolve the device error word");
   const int64_t sms = num_sms();
@@ -1238,19 +1271,29 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
   prm.part_i = reinterpret_cast<int32_t*>(w + part);
   prm.list_s = reinterpret_cast<float*>(w + 2 * part);
   prm.list_i = reinterpret_cast<int32_t*>(w + 2 * part + list);
+  const size_t qfloor_bytes = (((size_t)Qmax * 4) + 255) & ~(size_t)255;
   prm.qfloor = reinterpret_cast<uint32_t*>(w + 2 * part + 2 * list);
+  float* kth = reinterpret_cast<float*>(w + 2 * part + 2 * list + qfloor_bytes);
   prm.err = err;
-  // The shared per-query floors of the register-list passes start empty.
-  const cudaError_t ze = cudaMemsetAsync(prm.qfloor, 0, (size_t)Qmax * 4, stream);
-  if (ze != cudaSuccess) return cuda_fail(ze, "floor clear");
-  const int64_t mgrid = Qmax < sms * 8 ? Qmax : sms * 8;
-  auto merge = [&](const Params& pm, int32_t kout) -> hs_status {
-    if (kout <= 32 && 2 * (int64_t)pm.slots <= 32 * kMaxListsPerLane) {
-      const int64_t blocks = (Qmax + 7) / 8;        // one warp per query
+  const bool small = Qmax <= SQ_N && k <= 32 && prm.kb_count <= SQ_MAXKB;
+  if (!small) {
+    // The shared per-query floors of the register-list passes start empty.
+    const cudaError_t ze = cudaMemsetAsync(prm.qfloor, 0, (size_t)Qmax * 4, stream);
+    if (ze != cudaSuccess) return cuda_fail(ze, "floor clear");
+  }
+  const OutRows rows{inv, n_out};
+  const int64_t R = inv ? n_out : Qmax;             // rows the final merge writes
+  auto merge = [&](const Params& pm, int32_t kout, float* os, int32_t* oi,
+                   OutRows orows) -> hs_status {
+    const int64_t nr = orows.inv ? orows.n_out : Qmax;
+    if (nr == 0) return HS_OK;
+    if (oi && kout <= 32 && 2 * (int64_t)pm.slots <= 32 * kMaxListsPerLane) {
+      const int64_t blocks = (nr + 7) / 8;          // one warp per row
       merge_warp_kernel<<<(unsigned)(blocks < sms * 16 ? blocks : sms * 16), 256, 0, stream>>>(
-          pm, scores_out, ids_out, kout);
+          pm, os, oi, kout, orows);
       return cuda_fail(cudaGetLastError(), "merge launch");
     }
+    const int64_t mgrid = nr < sms * 8 ? nr : sms * 8;
     const size_t msmem = (size_t)p2_for(max_splits(sms, pm.tiles, pm.k), pm.k) * 8;
     static size_t merge_configured = 0;
     if (msmem > 48 * 1024 && msmem > merge_configured) {
@@ -1259,11 +1302,11 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
       if (e != cudaSuccess) return cuda_fail(e, "merge smem attribute");
       merge_configured = msmem;
     }
-    merge_kernel<<<(unsigned)mgrid, 256, msmem, stream>>>(pm, scores_out, ids_out, kout);
+    merge_kernel<<<(unsigned)mgrid, 256, msmem, stream>>>(pm, os, oi, kout, orows);
     return cuda_fail(cudaGetLastError(), "merge launch");
   };
   hs_status st;
-  if (Qmax <= SQ_N && k <= 32 && prm.kb_count <= SQ_MAXKB) {
+  if (small) {
     // Small batch: corpus as the M operand, queries resident (swap-AB).
     CUtensorMap mq16, mc128;
     if (!make_map(&mq16, queries, Qmax, d, SQ_N) || !make_map(&mc128, corpus, N, d, SQ_BM))
@@ -1299,8 +1342,7 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
     // most the query's final k-th best: a floor.  Pass 2 runs the large-k
     // kernel over the whole corpus keeping only scores >= the floor, which
     // leaves few candidates per list.  Both passes' lists go through the
-    // same workspace; the floor is staged in scores_out and overwritten by
-    // the final merge.
+    // same workspace; the floors (one score per query) are staged in it.
     if (tiles >= 64) {
       Params p1 = prm;
       p1.tiles = tiles / 8;
@@ -1309,12 +1351,12 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
       p1.floor = nullptr;
       st = launch_variant<32>(corpus, N, d, mq, p1, stream);
       if (st != HS_OK) return st;
-      st = merge(p1, k);
+      st = merge(p1, k, kth, nullptr, OutRows{nullptr, 0});
       if (st != HS_OK) return st;
       count_launches(2);
-      prm.floor = scores_out;
-      prm.floor_stride = k;
-      prm.floor_index = k - 1;
+      prm.floor = kth;
+      prm.floor_stride = 1;
+      prm.floor_index = 0;
       // Pass 1's shared floors bound 32nd-best scores, not k-th best: clear.
       const cudaError_t ze2 = cudaMemsetAsync(prm.qfloor, 0, (size_t)Qmax * 4, stream);
       if (ze2 != cudaSuccess) return cuda_fail(ze2, "floor clear");
@@ -1322,9 +1364,9 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
     st = launch_variant<0>(corpus, N, d, mq, prm, stream);
   }
   if (st != HS_OK) return st;
-  st = merge(prm, k);
+  st = merge(prm, k, scores_out, ids_out, rows);
   if (st != HS_OK) return st;
-  count_launches(2);  // retrieve_kernel + merge_kernel
+  count_launches(R > 0 ? 2 : 1);  // retrieve_kernel + merge_kernel
   return HS_OK;
 }
 

@@ -2,12 +2,16 @@
 
 Composition of the C-ABI calls only (no arithmetic here):
   chunks:  hs_fingerprint -> hs_unique_inverse      (merge duplicate chunk nodes)
-  queries: hs_fingerprint -> hs_unique_inverse      (merge duplicate query nodes,
-           -> hs_scatter_results (gather unique)     Section 3.3 (I))
-           -> hs_retrieve_topk_n                    (one retrieval per merged node)
-           -> hs_scatter_results (fan results back to every originating query)
+  queries: hs_merge_queries                         (merge duplicate query nodes,
+             (batches up to HS_MERGE_QUERIES_MAX;    Section 3.3 (I): fingerprint,
+              larger ones: hs_fingerprint ->          unique and gather in one
+              hs_unique_inverse ->                    launch)
+              hs_scatter_results gathering the unique rows)
+           -> hs_retrieve_topk_fanout               (one retrieval per merged node,
+                                                     results written to every
+                                                     originating query)
 Nothing here synchronises with the host: the merged-query count stays in
-device memory (hs_retrieve_topk_n reads it when its kernels run), and the
+device memory (the retrieval reads it when its kernels run), and the
 unique-index tail beyond that count is a valid row map, so the gather can
 always cover the whole batch.  Buffers are allocated once per stage.
 """
@@ -42,8 +46,6 @@ class EmbedRetrieveStage:
         self.q_fp = torch.empty(mq, dtype=torch.int64, device=dev)
         self.c_fp = torch.empty(mc, dtype=torch.int64, device=dev)
         self.uq = torch.empty((mq, self.d), dtype=corpus.dtype, device=dev)
-        self.s_u = torch.empty((mq, self.k), dtype=torch.float32, device=dev)
-        self.i_u = torch.empty((mq, self.k), **i32)
         self.scores = torch.empty((mq, self.k), dtype=torch.float32, device=dev)
         self.ids = torch.empty((mq, self.k), **i32)
 
@@ -70,19 +72,34 @@ class EmbedRetrieveStage:
         Q, d = queries.shape
         if Q > self.max_queries:
             raise ValueError("batch larger than max_queries")
+        nu, inv, uq = self._merge_queries(queries)
+        return self._retrieve_merged(uq, nu, inv, events) + (nu,)
+
+    def _merge_queries(self, queries: torch.Tensor):
+        """Merged query nodes of a batch: (n_unique_dev, inverse, unique
+        query rows)."""
+        Q = queries.shape[0]
+        nu_b, uidx_b, inv_b = self.q_out
+        if Q <= _lib.HS_MERGE_QUERIES_MAX:
+            _, nu, _, inv, uq = _lib.hs_merge_queries(
+                queries, out=(self.q_fp[:Q], nu_b, uidx_b[:Q], inv_b[:Q], self.uq[:Q]))
+            return nu, inv, uq
         qi32 = queries.view(torch.int32)
         fp = _lib.hs_fingerprint(qi32, fp_out=self.q_fp[:Q])
         nu, uidx, inv = _lib.hs_unique_inverse(fp, qi32, workspace=self.ws_q, out=self.q_out)
         uq = _lib.hs_scatter_results(queries, uidx, dst=self.uq[:Q])
+        return nu, inv, uq
+
+    def _retrieve_merged(self, uq, nu, inv, events):
+        Q = inv.shape[0]
         if events is not None:
             events[0].record()
-        s_u, i_u = _lib.hs_retrieve_topk_n(uq, nu, self.corpus, self.k, workspace=self.ws_r,
-                                           out=(self.s_u[:Q], self.i_u[:Q]))
+        scores, ids = _lib.hs_retrieve_topk_fanout(uq, nu, inv, self.corpus, self.k,
+                                                   workspace=self.ws_r,
+                                                   out=(self.scores[:Q], self.ids[:Q]))
         if events is not None:
             events[1].record()
-        scores = _lib.hs_scatter_results(s_u, inv, dst=self.scores[:Q])
-        ids = _lib.hs_scatter_results(i_u, inv, dst=self.ids[:Q])
-        return scores, ids, nu
+        return scores, ids
 
     def step(self, tokens: torch.Tensor, queries: torch.Tensor,
              lens: torch.Tensor | None = None, events: tuple | None = None):
@@ -101,20 +118,11 @@ class EmbedRetrieveStage:
         with torch.cuda.stream(self._side):
             chunk = self.dedup_chunks(tokens, lens)
         self._join.record(self._side)
-        Q = queries.shape[0]
-        qi32 = queries.view(torch.int32)
-        fp = _lib.hs_fingerprint(qi32, fp_out=self.q_fp[:Q])
-        nu, uidx, inv = _lib.hs_unique_inverse(fp, qi32, workspace=self.ws_q, out=self.q_out)
-        uq = _lib.hs_scatter_results(queries, uidx, dst=self.uq[:Q])
+        if queries.shape[0] > self.max_queries:
+            raise ValueError("batch larger than max_queries")
+        nu, inv, uq = self._merge_queries(queries)
         main.wait_event(self._join)      # retrieval occupies every SM: chunk work first
-        if events is not None:
-            events[0].record()
-        s_u, i_u = _lib.hs_retrieve_topk_n(uq, nu, self.corpus, self.k, workspace=self.ws_r,
-                                           out=(self.s_u[:Q], self.i_u[:Q]))
-        if events is not None:
-            events[1].record()
-        scores = _lib.hs_scatter_results(s_u, inv, dst=self.scores[:Q])
-        ids = _lib.hs_scatter_results(i_u, inv, dst=self.ids[:Q])
+        scores, ids = self._retrieve_merged(uq, nu, inv, events)
         return chunk, (scores, ids, nu)
 
 

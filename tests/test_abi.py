@@ -50,6 +50,14 @@ def test_host_only_calls_without_gpu():
     assert rc == _lib.HS_ERR_INVALID_ARG and b"k outside" in lib.hs_last_error()
     rc = lib.hs_unique_inverse(None, None, 1 << 30, 4, None, None, None, None, None, 0, None)
     assert rc == _lib.HS_ERR_INVALID_ARG
+    rc = lib.hs_merge_queries(None, _lib.HS_MERGE_QUERIES_MAX + 1, 768, 0, None, None, None,
+                              None, None, None, None)
+    assert rc == _lib.HS_ERR_INVALID_ARG and b"n_queries" in lib.hs_last_error()
+    rc = lib.hs_merge_queries(None, 4, 12, 0, None, None, None, None, None, None, None)
+    assert rc == _lib.HS_ERR_INVALID_ARG and b"dim" in lib.hs_last_error()
+    rc = lib.hs_retrieve_topk_fanout(None, 4, None, None, 4, None, 10, 64, 3, None, None, None,
+                                     0, None)
+    assert rc == _lib.HS_ERR_INVALID_ARG and b"inverse" in lib.hs_last_error()
 
 
 def test_binding_names_match_header():
