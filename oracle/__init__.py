@@ -2,8 +2,8 @@
 
 Plain, slow CPU implementations of what the GPU library computes; see
 ``hs_oracle.cpp`` for the definition each function follows and the paper
-passage it comes from (Section 3.3 Eq. 2 and "Dynamic Fusion and Reuse
-Mechanism"; Appendix A.2; Section 4.1 "Workloads").
+passage it comes from (Section 3.3 Eq. 2, "Dynamic Fusion and Reuse
+Mechanism" and Eq. 3; Appendix A.2; Section 4.1 "Workloads").
 
 Only the tests, ``__graft_entry__.smoke()`` and the benchmark's CPU-baseline
 leg may import this package.  The library under ``paper_2607_22578_gb300``
@@ -58,6 +58,8 @@ def _load():
             lib.oracle_pair_scores.restype = None
             lib.oracle_scatter.argtypes = [P, i64, i64, P, i64, P]
             lib.oracle_scatter.restype = ctypes.c_int
+            lib.oracle_segment_sum.argtypes = [P, P, i64, i64, P]
+            lib.oracle_segment_sum.restype = ctypes.c_int
             _lib = lib
     return _lib
 
@@ -143,3 +145,17 @@ def scatter(src: np.ndarray, mapping: np.ndarray) -> np.ndarray:
     if rc:
         raise IndexError("map entry outside [0, n_src)")
     return dst
+
+
+def segment_sum(phi: np.ndarray, inverse: np.ndarray, n_groups: int) -> np.ndarray:
+    """out[u] = sum of phi[i] over rows with inverse[i] == u (fp64, ascending
+    row order): the priority contribution of a fused node (Section 3.3,
+    Eq. 3)."""
+    phi = np.ascontiguousarray(phi, dtype=np.float64)
+    inverse = np.ascontiguousarray(inverse, dtype=np.int32)
+    assert phi.shape == inverse.shape
+    out = np.empty(max(int(n_groups), 1), dtype=np.float64)
+    rc = _load().oracle_segment_sum(_ptr(phi), _ptr(inverse), phi.size, int(n_groups), _ptr(out))
+    if rc:
+        raise IndexError("inverse entry outside [0, n_groups)")
+    return out[: int(n_groups)].copy()

@@ -25,6 +25,11 @@
 //   oracle_scatter
 //       result sharing: the output of the kept node flows to every merged
 //       node (Section 3.3 (I); Appendix A.2), dst[i] = src[map[i]].
+//   oracle_segment_sum
+//       the reuse-driven priority of a fused node (Section 3.3, "Reuse-Driven
+//       Priority Adjustment", Eq. 3): phi(v*) is the sum of phi(v) over the
+//       logical nodes v merged into v*, i.e. out[u] = sum of phi[i] over the
+//       rows i with inverse[i] = u, added in fp64 in ascending row order.
 //
 // Parity pins for these functions live in tests/ (published FNV vectors,
 // brute-force pairwise comparison, hand-computed top-k, library special
@@ -219,6 +224,19 @@ int oracle_scatter(const uint8_t* src, int64_t n_src, int64_t row_bytes,
   for (int64_t i = 0; i < n; ++i) {
     if (map[i] < 0 || (int64_t)map[i] >= n_src) return 1;
     std::memcpy(dst + i * row_bytes, src + (int64_t)map[i] * row_bytes, (size_t)row_bytes);
+  }
+  return 0;
+}
+
+// out[u] = sum over rows i with inverse[i] == u of phi[i], for u in
+// [0, n_groups); a group without rows sums to 0.  Returns 0, or 1 if some
+// inverse entry is outside [0, n_groups).
+int oracle_segment_sum(const double* phi, const int32_t* inverse, int64_t n, int64_t n_groups,
+                       double* out) {
+  for (int64_t u = 0; u < n_groups; ++u) out[u] = 0.0;
+  for (int64_t i = 0; i < n; ++i) {
+    if (inverse[i] < 0 || (int64_t)inverse[i] >= n_groups) return 1;
+    out[inverse[i]] += phi[i];
   }
   return 0;
 }
