@@ -460,8 +460,11 @@ def row_dedup_heavy(args, dev, peaks) -> dict:
             torch.empty(n, dtype=torch.int32, device=dev),
             torch.empty(n, dtype=torch.int32, device=dev))
     dst = torch.empty((n, W), dtype=torch.uint8, device=dev)
+    # per-row priority contributions (Eq. 3), summed per merged node after the step
+    phi = torch.rand(n, dtype=torch.float64, device=dev)
+    phi_u = torch.empty(n, dtype=torch.float64, device=dev)
     K = max(1, args.steps)
-    evs = [[_ev() for _ in range(4)] for _ in range(K)]
+    evs = [[_ev() for _ in range(5)] for _ in range(K)]
 
     def step(e=None):
         if e: e[0].record()
@@ -471,6 +474,8 @@ def row_dedup_heavy(args, dev, peaks) -> dict:
         if e: e[2].record()
         hs.hs_scatter_results(payload, outs[2], dst=dst)
         if e: e[3].record()
+        hs.hs_segment_sum(phi, outs[2], n, n_groups_dev=outs[0], out=phi_u)
+        if e: e[4].record()
 
     for _ in range(args.warmup):
         step()
@@ -484,6 +489,7 @@ def row_dedup_heavy(args, dev, peaks) -> dict:
     t_fp = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
     t_un = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
     t_sc = statistics.mean(e[2].elapsed_time(e[3]) for e in evs)
+    t_ss = statistics.mean(e[3].elapsed_time(e[4]) for e in evs)
     t_all = statistics.mean(e[0].elapsed_time(e[3]) for e in evs)
     L = w["lens"].astype(np.int64)
     sizes = np.bincount(gi, minlength=n_u)
@@ -492,6 +498,7 @@ def row_dedup_heavy(args, dev, peaks) -> dict:
     fp_bytes = tok_bytes + 4 * n + 8 * n
     un_bytes = 4 * int(L[multi].sum()) + 8 * n + 8 * n
     sc_bytes = n_u * W + n * W + 4 * n
+    ss_bytes = 8 * n + 4 * n + 8 * n_u
     return {
         "workload": "dedup_heavy: 400,000 rows x 512 int32 (lens U[64,512], Zipf(1.1) over "
                     "100,000 distinct) -> %d unique; scatter %d B per row" % (n_u, W),
@@ -500,7 +507,12 @@ def row_dedup_heavy(args, dev, peaks) -> dict:
         "kernels": {
             "hs_fingerprint": _roof(fp_bytes, None, t_fp, peaks),
             "hs_unique_inverse": _roof(un_bytes, None, t_un, peaks),
-            "hs_scatter_results": _roof(sc_bytes, None, t_sc, peaks)},
+            "hs_scatter_results": _roof(sc_bytes, None, t_sc, peaks),
+            "hs_segment_sum": _roof(ss_bytes, None, t_ss, peaks)},
+        "segment_sum_note": "priority contribution per merged node (Eq. 3) over the same "
+                            "inverse map, timed after the step and not part of its value; bytes: "
+                            "phi (fp64) + inverse in, one fp64 per merged node out; the output "
+                            "clear of the remaining %d entries is not counted" % (n - n_u),
         "bytes_note": "fingerprint: valid token bytes + lens + fp; unique: full-row verify "
                       "re-read of every row in a group of size >= 2 + fp in + unique_idx/inverse "
                       "out (sort scratch is L2-resident and not counted); scatter: unique rows "

@@ -7,9 +7,11 @@
  *   hs_unique_inverse   merge exactly-equal rows into unique nodes + inverse map
  *   hs_retrieve_topk    score merged queries against a corpus, keep top-k
  *   hs_scatter_results  fan each kept result back out to every merged row
- * and two fused forms for latency-bound batches:
+ * two fused forms for latency-bound batches:
  *   hs_merge_queries         fingerprint + merge + gather of a query batch
  *   hs_retrieve_topk_fanout  retrieval whose results go to every merged row
+ * and the scheduling weight of the merged nodes:
+ *   hs_segment_sum           priority contribution of each fused node (Eq. 3)
  *
  * Conventions shared by every call
  *   - Pointers named *_dev or documented as device pointers must be device
@@ -293,6 +295,37 @@ hs_status hs_merge_queries(const uint16_t* queries, int64_t n_queries, int32_t d
 hs_status hs_scatter_results(const void* src, int64_t n_src, int64_t row_bytes,
                              const int32_t* map, int64_t n_rows, void* dst,
                              hs_stream_t stream);
+
+/*
+ * hs_segment_sum — priority contribution of each fused node: the sum of the
+ * contributions of the rows merged into it.
+ *
+ * Paper: Section 3.3, "Reuse-Driven Priority Adjustment", Eq. 3:
+ * phi(v*) = sum over v in M(v*) of phi(v), so that a node shared by many
+ * queries is scheduled with their combined weight.  With the inverse map of
+ * hs_unique_inverse (or hs_merge_queries):
+ *   out[u] = sum of phi[i] over the rows i with inverse[i] == u,
+ * for u < count, count = min(*n_groups_dev, max_groups), or max_groups if
+ * n_groups_dev is NULL; out[u] = 0 for count <= u < max_groups.
+ *
+ * Additions are fp64 in an unspecified order: for a group of m rows the
+ * result is within (m-1)u/(1-(m-1)u) * sum|phi| of the exact sum
+ * (u = 2^-53); sums whose partial sums are all representable (integers
+ * below 2^53, for instance) are exact.
+ *
+ * phi           device double [n_rows], 8-byte aligned.
+ * inverse       device int32 [n_rows]; an entry outside [0, count) sets the
+ *               device error word (HS_ERR_INVALID_ARG) and that row is left
+ *               out of every sum.
+ * n_rows        >= 0.
+ * n_groups_dev  device int32 scalar or NULL.
+ * max_groups    0 <= max_groups < 2^31 (>= 1 when n_rows > 0).
+ * out           device double [max_groups], 8-byte aligned; every entry is
+ *               written.
+ */
+hs_status hs_segment_sum(const double* phi, const int32_t* inverse, int64_t n_rows,
+                         const int32_t* n_groups_dev, int64_t max_groups, double* out,
+                         hs_stream_t stream);
 
 /*
  * hs_get_device_error — synchronise `stream`, then read and clear the

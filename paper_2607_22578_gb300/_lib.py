@@ -78,6 +78,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
             lib.hs_retrieve_topk_fanout.restype = st
             lib.hs_merge_queries.argtypes = [P, i64, i32, u64, P, P, P, P, P, P, P]
             lib.hs_merge_queries.restype = st
+            lib.hs_segment_sum.argtypes = [P, P, i64, P, i64, P, P]
+            lib.hs_segment_sum.restype = st
             lib.hs_scatter_results.argtypes = [P, i64, i64, P, i64, P, P]
             lib.hs_scatter_results.restype = st
             lib.hs_get_device_error.argtypes = [P]
@@ -330,6 +332,29 @@ def hs_scatter_results(src: torch.Tensor, mapping: torch.Tensor, dst: torch.Tens
     _check(load().hs_scatter_results(_ptr(src), src.shape[0], row_bytes, _ptr(mapping), n,
                                      _ptr(dst), _stream(stream)))
     return dst
+
+
+def hs_segment_sum(phi: torch.Tensor, inverse: torch.Tensor, max_groups: int,
+                   n_groups_dev: torch.Tensor | None = None, out: torch.Tensor | None = None,
+                   stream=None) -> torch.Tensor:
+    """out[u] = sum of phi[i] over rows with inverse[i] == u (float64
+    [max_groups]; entries past the group count, n_groups_dev[0] if given,
+    are 0): the priority contribution of each fused node."""
+    _cuda(phi, "phi")
+    _cuda(inverse, "inverse")
+    if phi.dtype != torch.float64 or inverse.dtype != torch.int32:
+        raise TypeError("phi must be float64 and inverse int32")
+    if phi.numel() != inverse.numel():
+        raise ValueError("phi and inverse differ in length")
+    if n_groups_dev is not None:
+        _cuda(n_groups_dev, "n_groups_dev")
+        if n_groups_dev.dtype != torch.int32:
+            raise TypeError("n_groups_dev must be int32")
+    if out is None:
+        out = torch.empty(max(int(max_groups), 1), dtype=torch.float64, device=phi.device)
+    _check(load().hs_segment_sum(_ptr(phi), _ptr(inverse), phi.numel(), _ptr(n_groups_dev),
+                                 int(max_groups), _ptr(out), _stream(stream)))
+    return out[: int(max_groups)]
 
 
 def hs_launch_count() -> int:

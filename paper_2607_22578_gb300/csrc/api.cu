@@ -20,6 +20,8 @@ size_t retrieve_topk_workspace(int64_t, int64_t, int32_t, int32_t);
 hs_status launch_retrieve_topk(const uint16_t*, int64_t, const int32_t*, const int32_t*, int64_t,
                                const uint16_t*, int64_t, int32_t, int32_t, float*, int32_t*,
                                void*, size_t, cudaStream_t);
+hs_status launch_segment_sum(const double*, const int32_t*, int64_t, const int32_t*, int64_t,
+                             double*, cudaStream_t);
 hs_status launch_merge_queries(const uint16_t*, int64_t, int32_t, uint64_t, const uint64_t*,
                                uint64_t*, int32_t*, int32_t*, int32_t*, uint16_t*, cudaStream_t);
 hs_status launch_scatter(const void*, int64_t, int64_t, const int32_t*, int64_t, void*,
@@ -260,6 +262,24 @@ hs_status hs_scatter_results(const void* src, int64_t n_src, int64_t row_bytes,
   if (s0 < d1 && d0 < s1) return fail(HS_ERR_INVALID_ARG, "src and dst overlap");
   return launch_scatter(src, n_src, row_bytes, map, n_rows, dst,
                         reinterpret_cast<cudaStream_t>(stream));
+}
+
+hs_status hs_segment_sum(const double* phi, const int32_t* inverse, int64_t n_rows,
+                         const int32_t* n_groups_dev, int64_t max_groups, double* out,
+                         hs_stream_t stream) {
+  clear_msg();
+  if (n_rows < 0) return fail(HS_ERR_INVALID_ARG, "n_rows < 0");
+  if (max_groups < 0 || max_groups > 0x7fffffffLL)
+    return fail(HS_ERR_INVALID_ARG, "max_groups outside [0, 2^31 - 1]");
+  if (max_groups > 0 && !out) return fail(HS_ERR_INVALID_ARG, "out is NULL");
+  if (n_rows > 0 && (!phi || !inverse)) return fail(HS_ERR_INVALID_ARG, "NULL input pointer");
+  if (!aligned(phi, 8) || !aligned(out, 8) || !aligned(inverse, 4) ||
+      (n_groups_dev && !aligned(n_groups_dev, 4)))
+    return fail(HS_ERR_INVALID_ARG, "misaligned pointer (phi/out 8 B, inverse/count 4 B)");
+  if (n_rows > 0 && max_groups == 0)
+    return fail(HS_ERR_INVALID_ARG, "rows given but max_groups is 0");
+  return launch_segment_sum(phi, inverse, n_rows, n_groups_dev, max_groups, out,
+                            reinterpret_cast<cudaStream_t>(stream));
 }
 
 hs_status hs_get_device_error(hs_stream_t stream) {
