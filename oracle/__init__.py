@@ -3,7 +3,8 @@
 Plain, slow CPU implementations of what the GPU library computes; see
 ``hs_oracle.cpp`` for the definition each function follows and the paper
 passage it comes from (Section 3.3 Eq. 2, "Dynamic Fusion and Reuse
-Mechanism" and Eq. 3; Appendix A.2; Section 4.1 "Workloads").
+Mechanism" and Eq. 3; Appendix A.2; Section 4.1 "Workloads", retrieval and
+rerank).
 
 Only the tests, ``__graft_entry__.smoke()`` and the benchmark's CPU-baseline
 leg may import this package.  The library under ``paper_2607_22578_gb300``
@@ -58,6 +59,8 @@ def _load():
             lib.oracle_pair_scores.restype = None
             lib.oracle_scatter.argtypes = [P, i64, i64, P, i64, P]
             lib.oracle_scatter.restype = ctypes.c_int
+            lib.oracle_rerank.argtypes = [P, i64, P, i64, i32, P, i32, i32, P, P]
+            lib.oracle_rerank.restype = ctypes.c_int
             lib.oracle_segment_sum.argtypes = [P, P, i64, i64, P]
             lib.oracle_segment_sum.restype = ctypes.c_int
             _lib = lib
@@ -159,3 +162,23 @@ def segment_sum(phi: np.ndarray, inverse: np.ndarray, n_groups: int) -> np.ndarr
     if rc:
         raise IndexError("inverse entry outside [0, n_groups)")
     return out[: int(n_groups)].copy()
+
+
+def rerank(rq: np.ndarray, rc: np.ndarray, cand: np.ndarray, k2: int):
+    """Second-stage rerank of retrieved candidates (Section 4.1, RAG with
+    rerank): fp64 inner products of bf16 rerank vectors over cand[q, :]
+    (negative entries absent), ordered by descending score, ties to the lower
+    id; returns the first k2 (scores fp64, ids int32)."""
+    rq = np.ascontiguousarray(rq, dtype=np.uint16)
+    rc = np.ascontiguousarray(rc, dtype=np.uint16)
+    cand = np.ascontiguousarray(cand, dtype=np.int32)
+    nq, d = rq.shape
+    assert rc.shape[1] == d and cand.shape[0] == nq
+    k1 = cand.shape[1]
+    scores = np.empty((nq, k2), dtype=np.float64)
+    ids = np.empty((nq, k2), dtype=np.int32)
+    rc_ = _load().oracle_rerank(_ptr(rq), nq, _ptr(rc), rc.shape[0], d, _ptr(cand), k1, k2,
+                                _ptr(scores), _ptr(ids))
+    if rc_:
+        raise IndexError("candidate id outside [0, n_rc)")
+    return scores, ids

@@ -30,12 +30,20 @@
 //       Priority Adjustment", Eq. 3): phi(v*) is the sum of phi(v) over the
 //       logical nodes v merged into v*, i.e. out[u] = sum of phi[i] over the
 //       rows i with inverse[i] = u, added in fp64 in ascending row order.
+//   oracle_rerank
+//       the second stage of the RAG-with-rerank workflow (Section 4.1,
+//       "Workloads": a reranker scores the initial top-12 chunks and the
+//       top-8 by those scores are kept).  The reranker model is absent, so
+//       its score is an exact fp64 inner product of bf16 rerank vectors; the
+//       candidates of a query are ordered by descending score, ties to the
+//       lower corpus index, and the first k2 kept.
 //
 // Parity pins for these functions live in tests/ (published FNV vectors,
 // brute-force pairwise comparison, hand-computed top-k, library special
 // cases, generator ground truth).
 
 #include <algorithm>
+#include <cmath>
 #include <cstdint>
 #include <cstring>
 #include <numeric>
@@ -224,6 +232,38 @@ int oracle_scatter(const uint8_t* src, int64_t n_src, int64_t row_bytes,
   for (int64_t i = 0; i < n; ++i) {
     if (map[i] < 0 || (int64_t)map[i] >= n_src) return 1;
     std::memcpy(dst + i * row_bytes, src + (int64_t)map[i] * row_bytes, (size_t)row_bytes);
+  }
+  return 0;
+}
+
+// For each query q: the candidates cand[q, 0:k1] (entries < 0 are absent)
+// scored by the fp64 inner product of rq[q] and rc[id], ordered by (score
+// descending, id ascending), the first k2 written to scores_out / ids_out
+// (-inf / -1 past the number of present candidates).  Returns 0, or 1 if a
+// candidate id is >= n_rc.
+int oracle_rerank(const uint16_t* rq, int64_t nq, const uint16_t* rc, int64_t n_rc, int32_t d,
+                  const int32_t* cand, int32_t k1, int32_t k2, double* scores_out,
+                  int32_t* ids_out) {
+  for (int64_t q = 0; q < nq; ++q) {
+    std::vector<std::pair<double, int32_t>> c;
+    for (int32_t j = 0; j < k1; ++j) {
+      const int32_t id = cand[q * k1 + j];
+      if (id < 0) continue;
+      if ((int64_t)id >= n_rc) return 1;
+      double s = 0.0;
+      for (int32_t t = 0; t < d; ++t)
+        s += bf16_to_double(rq[q * d + t]) * bf16_to_double(rc[(int64_t)id * d + t]);
+      c.push_back({s, id});
+    }
+    std::sort(c.begin(), c.end(), [](const std::pair<double, int32_t>& a,
+                                     const std::pair<double, int32_t>& b) {
+      return a.first != b.first ? a.first > b.first : a.second < b.second;
+    });
+    for (int32_t j = 0; j < k2; ++j) {
+      const bool have = j < (int32_t)c.size();
+      scores_out[q * k2 + j] = have ? c[j].first : -INFINITY;
+      ids_out[q * k2 + j] = have ? c[j].second : -1;
+    }
   }
   return 0;
 }
