@@ -616,6 +616,61 @@ def row_large_corpus(args, dev, peaks) -> dict:
             "retrieval": _roof(2.0 * N * d, 2.0 * Q * N * d, ms, peaks)}
 
 
+def row_rerank(args, dev, peaks) -> dict:
+    """RAG with rerank (Section 4.1): the merged RAG-mix queries retrieve
+    their top-12 from the 1,048,576 x 768 corpus, then a second stage
+    rescores those 12 with 1024-dim rerank vectors and keeps the top-8."""
+    import torch
+
+    import paper_2607_22578_gb300 as hs
+    from synth import configs
+    w = configs.build_retrieval_mix(configs.RAG_MIX, seed=args.seed)
+    corpus = _dev_array(w["corpus"], dev)
+    q = _dev_array(w["queries"], dev)
+    N, d = w["corpus"].shape
+    Q = q.shape[0]
+    del w
+    d2, k1, k2 = 1024, 12, 8
+    g = torch.Generator(device=dev).manual_seed(args.seed + 17)
+    rc = torch.nn.functional.normalize(torch.randn(N, d2, device=dev, generator=g), dim=1)
+    rc = rc.to(torch.bfloat16)
+    rq_all = torch.nn.functional.normalize(torch.randn(Q, d2, device=dev, generator=g), dim=1)
+    rq_all = rq_all.to(torch.bfloat16)
+    _, nu, uidx, inv, uq = hs.hs_merge_queries(q) if Q <= hs.HS_MERGE_QUERIES_MAX else (None,) * 5
+    if nu is None:
+        fp = hs.hs_fingerprint(q.view(torch.int32))
+        nu, uidx, inv = hs.hs_unique_inverse(fp, q.view(torch.int32))
+        uq = hs.hs_scatter_results(q, uidx)
+    rq = hs.hs_scatter_results(rq_all, uidx)            # rerank vectors of the merged queries
+    s12, i12 = hs.hs_retrieve_topk_n(uq, nu, corpus, k1)
+    torch.cuda.synchronize()
+    Qu = int(nu.item())
+    outs = (torch.empty((Q, k2), dtype=torch.float32, device=dev),
+            torch.empty((Q, k2), dtype=torch.int32, device=dev))
+    for _ in range(3):
+        hs.hs_rerank_topk(rq, rc, i12, k2, n_queries_dev=nu, inverse=inv, out=outs)
+    torch.cuda.synchronize()
+    K = max(3, args.steps)
+    e0, e1 = _ev(), _ev()
+    e0.record()
+    for _ in range(K):
+        hs.hs_rerank_topk(rq, rc, i12, k2, n_queries_dev=nu, inverse=inv, out=outs)
+    e1.record()
+    torch.cuda.synchronize()
+    hs.hs_get_device_error()
+    ms = e0.elapsed_time(e1) / K
+    # every output row gathers its query's k1 candidate rows (merged
+    # duplicates re-read rows that are then in L2)
+    bytes_ = Q * (k1 * d2 * 2 + d2 * 2 + k1 * 4 + 4 + k2 * 8)
+    return {"workload": "rerank: %d queries (%d merged), top-%d of a %d x %d corpus rescored "
+                        "with %d-dim rerank vectors (%d x %d bf16), top-%d kept"
+                        % (Q, Qu, k1, N, d, d2, N, d2, k2),
+            "metric": "reranked queries/s", "value": Q / (ms / 1e3), "steps": K,
+            "kernels": {"hs_rerank_topk": _roof(bytes_, None, ms, peaks)},
+            "bytes_note": "per output row: k1 candidate rows + the rerank query row + "
+                          "candidate ids + map entry + k2 results"}
+
+
 def rag_mix_breakdown(stage, tokens, queries, K: int) -> dict:
     """Per-phase device time of the RAG-mix step (the same calls as the
     pipeline, with events between them)."""
@@ -657,7 +712,7 @@ def rows_arm(args) -> int:
     dev = torch.device("cuda", 0)
     peaks, kind = load_peaks()
     fn = {"dedup_heavy": row_dedup_heavy, "batch_sweep": row_batch_sweep,
-          "large_corpus": row_large_corpus}[args.workload]
+          "large_corpus": row_large_corpus, "rerank": row_rerank}[args.workload]
     line = fn(args, dev, peaks)
     line["peaks"] = {"hbm_gbs": peaks["hbm_gbs"], "bf16_tflops": peaks["bf16_tflops"],
                      "source": kind}
@@ -676,7 +731,7 @@ def main() -> int:
                     help="seconds of host time for the oracle baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--workload", default="rag_mix",
-                    choices=["rag_mix", "dedup_heavy", "batch_sweep", "large_corpus"],
+                    choices=["rag_mix", "dedup_heavy", "batch_sweep", "large_corpus", "rerank"],
                     help="rag_mix is the headline step; the others measure the other "
                          "rows of the hot-path table (one GPU)")
     ap.add_argument("--k", type=int, default=0, help="override k (large_corpus only)")

@@ -10,6 +10,8 @@
  * two fused forms for latency-bound batches:
  *   hs_merge_queries         fingerprint + merge + gather of a query batch
  *   hs_retrieve_topk_fanout  retrieval whose results go to every merged row
+ * the second retrieval stage of the rerank workflow:
+ *   hs_rerank_topk           rescore the retrieved candidates, keep the best
  * and the scheduling weight of the merged nodes:
  *   hs_segment_sum           priority contribution of each fused node (Eq. 3)
  *
@@ -295,6 +297,43 @@ hs_status hs_merge_queries(const uint16_t* queries, int64_t n_queries, int32_t d
 hs_status hs_scatter_results(const void* src, int64_t n_src, int64_t row_bytes,
                              const int32_t* map, int64_t n_rows, void* dst,
                              hs_stream_t stream);
+
+/*
+ * hs_rerank_topk — second retrieval stage: rescore each query's retrieved
+ * candidates and keep the best k2.
+ *
+ * Paper: Section 4.1, "Workloads", RAG with rerank: a reranker scores the
+ * initial top-12 chunks and the top-8 by those scores are kept.  The
+ * reranker model is not part of this library; its score is the inner
+ * product of bf16 rerank vectors accumulated in fp32:
+ *   s[q, j] = sum_t rerank_queries[q, t] * rerank_corpus[candidates[q, j], t]
+ * and query q keeps the k2 candidates first in (score descending, corpus
+ * index ascending), written in that order.
+ *
+ * rerank_queries  device bf16 bits (uint16) [max_queries, dim], 16-byte
+ *                 aligned rows.
+ * n_queries_dev   device int32 scalar or NULL: queries processed =
+ *                 min(*n_queries_dev, max_queries), or max_queries if NULL.
+ * rerank_corpus   device bf16 bits [n_corpus, dim], 16-byte aligned.
+ * dim             8 <= dim <= 65536, dim % 8 == 0.
+ * candidates      device int32 [max_queries, k1] (e.g. the ids of
+ *                 hs_retrieve_topk with k = k1).  A negative entry is an
+ *                 absent candidate; an entry >= n_corpus sets the device
+ *                 error word (HS_ERR_INVALID_ARG) and counts as absent.
+ * k1, k2          1 <= k2 <= k1 <= 32.
+ * inverse, n_out  NULL: one output row per query.  Otherwise n_out output
+ *                 rows, row o holding the result of query inverse[o] (the
+ *                 fan-out to every merged row, as hs_retrieve_topk_fanout);
+ *                 an entry outside [0, query count) sets the device error
+ *                 word and leaves that row unwritten.
+ * scores_out      device float [rows, k2]; ids_out device int32 [rows, k2].
+ *                 Entries past the number of present candidates are -inf / -1.
+ */
+hs_status hs_rerank_topk(const uint16_t* rerank_queries, int64_t max_queries,
+                         const int32_t* n_queries_dev, const uint16_t* rerank_corpus,
+                         int64_t n_corpus, int32_t dim, const int32_t* candidates, int32_t k1,
+                         int32_t k2, const int32_t* inverse, int64_t n_out, float* scores_out,
+                         int32_t* ids_out, hs_stream_t stream);
 
 /*
  * hs_segment_sum — priority contribution of each fused node: the sum of the

@@ -78,6 +78,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
             lib.hs_retrieve_topk_fanout.restype = st
             lib.hs_merge_queries.argtypes = [P, i64, i32, u64, P, P, P, P, P, P, P]
             lib.hs_merge_queries.restype = st
+            lib.hs_rerank_topk.argtypes = [P, i64, P, P, i64, i32, P, i32, i32, P, i64, P, P, P]
+            lib.hs_rerank_topk.restype = st
             lib.hs_segment_sum.argtypes = [P, P, i64, P, i64, P, P]
             lib.hs_segment_sum.restype = st
             lib.hs_scatter_results.argtypes = [P, i64, i64, P, i64, P, P]
@@ -332,6 +334,45 @@ def hs_scatter_results(src: torch.Tensor, mapping: torch.Tensor, dst: torch.Tens
     _check(load().hs_scatter_results(_ptr(src), src.shape[0], row_bytes, _ptr(mapping), n,
                                      _ptr(dst), _stream(stream)))
     return dst
+
+
+def hs_rerank_topk(rerank_queries: torch.Tensor, rerank_corpus: torch.Tensor,
+                   candidates: torch.Tensor, k2: int, n_queries_dev: torch.Tensor | None = None,
+                   inverse: torch.Tensor | None = None, out: tuple | None = None, stream=None):
+    """Rescore each query's candidates (int32 [Q, k1] corpus ids) by the
+    inner product of bf16 rerank vectors and keep the best k2.  Returns
+    (scores fp32, ids int32), one row per query, or one per entry of
+    ``inverse`` (row o = query inverse[o]) when it is given."""
+    _cuda(rerank_queries, "rerank_queries")
+    _cuda(rerank_corpus, "rerank_corpus")
+    _cuda(candidates, "candidates")
+    if rerank_queries.element_size() != 2 or rerank_corpus.element_size() != 2:
+        raise TypeError("rerank vectors must hold bf16 (2-byte) elements")
+    if candidates.dtype != torch.int32 or candidates.dim() != 2:
+        raise TypeError("candidates must be int32 [Q, k1]")
+    Q, d = rerank_queries.shape
+    N, d2 = rerank_corpus.shape
+    if d != d2:
+        raise ValueError("dimension mismatch")
+    if candidates.shape[0] != Q:
+        raise ValueError("candidates must have one row per query")
+    k1 = candidates.shape[1]
+    for t, name in ((n_queries_dev, "n_queries_dev"), (inverse, "inverse")):
+        if t is not None:
+            _cuda(t, name)
+            if t.dtype != torch.int32:
+                raise TypeError("%s must be int32" % name)
+    rows = inverse.numel() if inverse is not None else Q
+    dev = rerank_queries.device
+    if out is None:
+        out = (torch.empty((rows, k2), dtype=torch.float32, device=dev),
+               torch.empty((rows, k2), dtype=torch.int32, device=dev))
+    scores, ids = out
+    _check(load().hs_rerank_topk(_ptr(rerank_queries), Q, _ptr(n_queries_dev),
+                                 _ptr(rerank_corpus), N, d, _ptr(candidates), k1, int(k2),
+                                 _ptr(inverse), rows if inverse is not None else 0, _ptr(scores),
+                                 _ptr(ids), _stream(stream)))
+    return scores, ids
 
 
 def hs_segment_sum(phi: torch.Tensor, inverse: torch.Tensor, max_groups: int,

@@ -22,6 +22,9 @@ hs_status launch_retrieve_topk(const uint16_t*, int64_t, const int32_t*, const i
                                void*, size_t, cudaStream_t);
 hs_status launch_segment_sum(const double*, const int32_t*, int64_t, const int32_t*, int64_t,
                              double*, cudaStream_t);
+hs_status launch_rerank(const uint16_t*, int64_t, const int32_t*, const uint16_t*, int64_t, int32_t,
+                        const int32_t*, int32_t, int32_t, const int32_t*, int64_t, float*,
+                        int32_t*, cudaStream_t);
 hs_status launch_merge_queries(const uint16_t*, int64_t, int32_t, uint64_t, const uint64_t*,
                                uint64_t*, int32_t*, int32_t*, int32_t*, uint16_t*, cudaStream_t);
 hs_status launch_scatter(const void*, int64_t, int64_t, const int32_t*, int64_t, void*,
@@ -262,6 +265,37 @@ hs_status hs_scatter_results(const void* src, int64_t n_src, int64_t row_bytes,
   if (s0 < d1 && d0 < s1) return fail(HS_ERR_INVALID_ARG, "src and dst overlap");
   return launch_scatter(src, n_src, row_bytes, map, n_rows, dst,
                         reinterpret_cast<cudaStream_t>(stream));
+}
+
+hs_status hs_rerank_topk(const uint16_t* rerank_queries, int64_t max_queries,
+                         const int32_t* n_queries_dev, const uint16_t* rerank_corpus,
+                         int64_t n_corpus, int32_t dim, const int32_t* candidates, int32_t k1,
+                         int32_t k2, const int32_t* inverse, int64_t n_out, float* scores_out,
+                         int32_t* ids_out, hs_stream_t stream) {
+  clear_msg();
+  if (max_queries < 0 || max_queries > 0x7fffffffLL)
+    return fail(HS_ERR_INVALID_ARG, "max_queries outside [0, 2^31 - 1]");
+  if (n_corpus < 1 || n_corpus > 0x7fffffffLL)
+    return fail(HS_ERR_INVALID_ARG, "n_corpus outside [1, 2^31 - 1]");
+  if (dim < 8 || dim % 8 != 0 || dim > 65536)
+    return fail(HS_ERR_INVALID_ARG, "dim must be a multiple of 8 in [8, 65536]");
+  if (k1 < 1 || k1 > 32 || k2 < 1 || k2 > k1)
+    return fail(HS_ERR_INVALID_ARG, "need 1 <= k2 <= k1 <= 32");
+  if (inverse && (n_out < 0 || n_out > 0x7fffffffLL))
+    return fail(HS_ERR_INVALID_ARG, "n_out outside [0, 2^31 - 1]");
+  const int64_t rows = inverse ? n_out : max_queries;
+  if (rows == 0) return HS_OK;
+  if (max_queries == 0) return fail(HS_ERR_INVALID_ARG, "output rows but no queries");
+  if (!rerank_queries || !rerank_corpus || !candidates || !scores_out || !ids_out)
+    return fail(HS_ERR_INVALID_ARG, "NULL input or output pointer");
+  if (!aligned(rerank_queries, 16) || !aligned(rerank_corpus, 16))
+    return fail(HS_ERR_INVALID_ARG, "rerank vectors must be 16-byte aligned");
+  if (!aligned(candidates, 4) || !aligned(scores_out, 4) || !aligned(ids_out, 4) ||
+      (inverse && !aligned(inverse, 4)) || (n_queries_dev && !aligned(n_queries_dev, 4)))
+    return fail(HS_ERR_INVALID_ARG, "misaligned pointer");
+  return launch_rerank(rerank_queries, max_queries, n_queries_dev, rerank_corpus, n_corpus, dim,
+                       candidates, k1, k2, inverse, n_out, scores_out, ids_out,
+                       reinterpret_cast<cudaStream_t>(stream));
 }
 
 hs_status hs_segment_sum(const double* phi, const int32_t* inverse, int64_t n_rows,

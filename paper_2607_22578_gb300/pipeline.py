@@ -10,6 +10,9 @@ Composition of the C-ABI calls only (no arithmetic here):
            -> hs_retrieve_topk_fanout               (one retrieval per merged node,
                                                      results written to every
                                                      originating query)
+  rerank:  hs_retrieve_topk_n -> hs_scatter_results (rerank vectors of the
+           merged queries) -> hs_rerank_topk        (top-k rescored, best kept,
+                                                     fanned out; Section 4.1)
 Nothing here synchronises with the host: the merged-query count stays in
 device memory (the retrieval reads it when its kernels run), and the
 unique-index tail beyond that count is a valid row map, so the gather can
@@ -26,7 +29,8 @@ class EmbedRetrieveStage:
     """Holds the resident corpus and reusable buffers for repeated batches."""
 
     def __init__(self, corpus: torch.Tensor, k: int, max_queries: int,
-                 max_chunk_rows: int = 0):
+                 max_chunk_rows: int = 0, rerank_corpus: torch.Tensor | None = None,
+                 rerank_k: int = 0):
         if not corpus.is_cuda:
             raise TypeError("corpus must be resident on the GPU")
         self.corpus = corpus
@@ -48,6 +52,19 @@ class EmbedRetrieveStage:
         self.uq = torch.empty((mq, self.d), dtype=corpus.dtype, device=dev)
         self.scores = torch.empty((mq, self.k), dtype=torch.float32, device=dev)
         self.ids = torch.empty((mq, self.k), **i32)
+        # second stage (RAG with rerank): k candidates rescored, rerank_k kept
+        self.rerank_corpus, self.rerank_k = rerank_corpus, int(rerank_k)
+        if rerank_corpus is not None:
+            if not rerank_corpus.is_cuda or rerank_corpus.shape[0] != self.N:
+                raise ValueError("rerank_corpus must be on the GPU, one row per corpus row")
+            if not 1 <= self.rerank_k <= self.k:
+                raise ValueError("need 1 <= rerank_k <= k")
+            self.s_u = torch.empty((mq, self.k), dtype=torch.float32, device=dev)
+            self.i_u = torch.empty((mq, self.k), **i32)
+            self.rq_u = torch.empty((mq, rerank_corpus.shape[1]), dtype=rerank_corpus.dtype,
+                                    device=dev)
+            self.r_scores = torch.empty((mq, self.rerank_k), dtype=torch.float32, device=dev)
+            self.r_ids = torch.empty((mq, self.rerank_k), **i32)
 
     def capture(self, tokens: torch.Tensor, queries: torch.Tensor,
                 lens: torch.Tensor | None = None) -> "StepGraph":
@@ -74,6 +91,27 @@ class EmbedRetrieveStage:
             raise ValueError("batch larger than max_queries")
         nu, inv, uq = self._merge_queries(queries)
         return self._retrieve_merged(uq, nu, inv, events) + (nu,)
+
+    def retrieve_rerank(self, queries: torch.Tensor, rerank_queries: torch.Tensor):
+        """RAG with rerank (Section 4.1): merged retrieval of the top-k, then
+        the k candidates of each merged query rescored with its rerank
+        vector (the representative's row of ``rerank_queries``) and the best
+        rerank_k kept, fanned out to every query.  Returns (scores [Q,
+        rerank_k], ids [Q, rerank_k], n_unique_dev)."""
+        if self.rerank_corpus is None:
+            raise ValueError("stage built without a rerank corpus")
+        Q = queries.shape[0]
+        if Q > self.max_queries or rerank_queries.shape[0] != Q:
+            raise ValueError("batch larger than max_queries or rerank rows differ")
+        nu, inv, uq = self._merge_queries(queries)
+        uidx = self.q_out[1][:Q]
+        _lib.hs_retrieve_topk_n(uq, nu, self.corpus, self.k, workspace=self.ws_r,
+                                out=(self.s_u[:Q], self.i_u[:Q]))
+        rq = _lib.hs_scatter_results(rerank_queries, uidx, dst=self.rq_u[:Q])
+        scores, ids = _lib.hs_rerank_topk(rq, self.rerank_corpus, self.i_u[:Q], self.rerank_k,
+                                          n_queries_dev=nu, inverse=inv,
+                                          out=(self.r_scores[:Q], self.r_ids[:Q]))
+        return scores, ids, nu
 
     def _merge_queries(self, queries: torch.Tensor):
         """Merged query nodes of a batch: (n_unique_dev, inverse, unique
