@@ -182,3 +182,21 @@ def rerank(rq: np.ndarray, rc: np.ndarray, cand: np.ndarray, k2: int):
     if rc_:
         raise IndexError("candidate id outside [0, n_rc)")
     return scores, ids
+
+
+def cache_reuse(batches):
+    """Asynchronous cache reuse across batches (Section 3.3, "Dynamic Fusion
+    and Reuse Mechanism" (II)) with unbounded capacity: a node of a later
+    batch that equals a node completed in an earlier batch takes that
+    node's result instead of executing.  ``batches`` is a sequence of 2-D
+    arrays of rows (the merged nodes of each batch); returns, per batch, a
+    bool array: True where the row equals a row of an earlier batch."""
+    seen = set()
+    out = []
+    for rows in batches:
+        rows = np.ascontiguousarray(rows)
+        hit = np.array([r.tobytes() in seen for r in rows], dtype=bool)
+        for r in rows:
+            seen.add(r.tobytes())
+        out.append(hit)
+    return out

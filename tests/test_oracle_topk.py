@@ -128,3 +128,4 @@ def test_bad_k_is_rejected():
         oracle.topk(Q, C, 3)
     with pytest.raises(ValueError):
         oracle.topk(Q, C, 0)
+
