@@ -12,6 +12,8 @@
  *   hs_retrieve_topk_fanout  retrieval whose results go to every merged row
  * the second retrieval stage of the rerank workflow:
  *   hs_rerank_topk           rescore the retrieved candidates, keep the best
+ * reuse of results across batches:
+ *   hs_cache_lookup / hs_cache_insert   a device-resident result cache
  * and the scheduling weight of the merged nodes:
  *   hs_segment_sum           priority contribution of each fused node (Eq. 3)
  *
@@ -334,6 +336,90 @@ hs_status hs_rerank_topk(const uint16_t* rerank_queries, int64_t max_queries,
                          int64_t n_corpus, int32_t dim, const int32_t* candidates, int32_t k1,
                          int32_t k2, const int32_t* inverse, int64_t n_out, float* scores_out,
                          int32_t* ids_out, hs_stream_t stream);
+
+/*
+ * Result cache — asynchronous cache reuse across batches.
+ *
+ * Paper: Section 3.3, "Dynamic Fusion and Reuse Mechanism" (II): a node
+ * that matches a node completed earlier takes its result instead of being
+ * executed.  Here the nodes are merged queries and the result is their
+ * retrieval top-k.  The cache lives in device memory the caller provides
+ * (hs_cache_bytes) and keeps `capacity` entries or more: sets of 8 entries,
+ * chosen by the query's fingerprint; within a set a new entry takes an
+ * empty way, else the least recently used one.  Every entry stores the
+ * query vector, and a hit requires the whole vector to be equal: a
+ * fingerprint collision never returns another query's result.
+ *
+ * A batch runs: hs_cache_lookup over its merged queries -> retrieval of the
+ * misses (hs_retrieve_topk_n over miss_queries with count n_miss_dev) ->
+ * hs_cache_insert of those results.  After the insert, row u of scores_out /
+ * ids_out holds the top-k of query u, hit or miss.  Calls on one stream are
+ * ordered, so each batch sees the inserts of the batches before it; calls on
+ * different streams that share a cache race (a query that equals one still
+ * being retrieved elsewhere misses and is retrieved again; no kernel waits
+ * for another).
+ *
+ * Arguments common to the cache calls:
+ *   cache, cache_bytes   device memory, 256-byte aligned, at least
+ *                        hs_cache_bytes(capacity, dim, k) bytes;
+ *   capacity, dim, k     the values given to hs_cache_init (1 <= capacity
+ *                        <= 2^30, 8 <= dim <= 65536 with dim % 8 == 0,
+ *                        1 <= k <= HS_TOPK_MAX_K).  A cache whose header
+ *                        does not match them sets the device error word
+ *                        (HS_ERR_INVALID_ARG) and the call does nothing.
+ */
+size_t hs_cache_bytes(int64_t capacity, int32_t dim, int32_t k);  /* 0: invalid shape */
+hs_status hs_cache_init(void* cache, size_t cache_bytes, int64_t capacity, int32_t dim,
+                        int32_t k, hs_stream_t stream);
+
+/*
+ * hs_cache_lookup — look the merged queries of a batch up.
+ *
+ * queries        device bf16 bits [max_queries, dim], 16-byte aligned: the
+ *                merged (unique) queries; the first count are looked up,
+ *                count = min(*n_queries_dev, max_queries), or max_queries.
+ * fp, fp_rows    query u's key is fp[fp_rows[u]] (fp_rows NULL: fp[u]);
+ *                device uint64 / int32 (with hs_merge_queries: its fp_out
+ *                and unique_idx_out).
+ * scores_out     device float [max_queries, k], ids_out int32 [max_queries,
+ *                k]: rows of hits are written here.
+ * miss_list      device int32 [max_queries]: the ordinals u of the misses,
+ *                in no particular order; *n_miss_dev their number (reset by
+ *                this call); miss_queries device bf16 bits [max_queries,
+ *                dim]: row i = queries[miss_list[i]].
+ */
+hs_status hs_cache_lookup(void* cache, size_t cache_bytes, int64_t capacity, int32_t dim,
+                          int32_t k, const uint16_t* queries, const uint64_t* fp,
+                          const int32_t* fp_rows, int64_t max_queries,
+                          const int32_t* n_queries_dev, float* scores_out, int32_t* ids_out,
+                          int32_t* miss_list, int32_t* n_miss_dev, uint16_t* miss_queries,
+                          hs_stream_t stream);
+
+/*
+ * hs_cache_insert — store the retrieved results of a batch's misses.
+ *
+ * miss_list, n_miss_dev, miss_queries   as written by hs_cache_lookup.
+ * max_queries    the max_queries of that lookup.
+ * fp, fp_rows    as given to that lookup.
+ * miss_scores, miss_ids   device float / int32 [max_queries, k]: row i is
+ *                the top-k of miss_queries[i] (hs_retrieve_topk_n's output).
+ * scores_out, ids_out     the lookup's outputs: row miss_list[i] receives
+ *                row i of the results.  Entries are added to the cache; when
+ *                every way of a set is being written by this batch the
+ *                result is returned but not cached.
+ */
+hs_status hs_cache_insert(void* cache, size_t cache_bytes, int64_t capacity, int32_t dim,
+                          int32_t k, const int32_t* miss_list, const int32_t* n_miss_dev,
+                          int64_t max_queries, const uint16_t* miss_queries, const uint64_t* fp,
+                          const int32_t* fp_rows, const float* miss_scores,
+                          const int32_t* miss_ids, float* scores_out, int32_t* ids_out,
+                          hs_stream_t stream);
+
+/*
+ * hs_cache_stats — hits and misses counted since hs_cache_init.
+ * Synchronises `stream`; host pointers for the two counts.
+ */
+hs_status hs_cache_stats(const void* cache, uint64_t* hits, uint64_t* misses, hs_stream_t stream);
 
 /*
  * hs_segment_sum — priority contribution of each fused node: the sum of the

@@ -7,7 +7,8 @@ from ._lib import (HS_ERR_CUDA, HS_ERR_INVALID_ARG, HS_ERR_TIMEOUT, HS_ERR_UNSUP
                    HS_TOPK_MAX_K, HsError, hs_fingerprint, hs_get_device_error,
                    hs_launch_count, hs_merge_queries, hs_retrieve_topk, hs_retrieve_topk_fanout,
                    hs_retrieve_topk_n, hs_retrieve_topk_workspace, hs_scatter_results,
-                   hs_rerank_topk, hs_segment_sum,
+                   hs_rerank_topk, hs_segment_sum, ResultCache, hs_cache_bytes, hs_cache_init, hs_cache_insert,
+                   hs_cache_lookup, hs_cache_stats,
                    hs_unique_inverse, hs_unique_inverse_noalloc, hs_unique_inverse_workspace,
                    hs_version, library_path, load)
 from .pipeline import EmbedRetrieveStage, HostFeed, RetrieveGraph, StepGraph
@@ -18,6 +19,7 @@ __all__ = [
     "HsError", "hs_fingerprint", "hs_unique_inverse", "hs_unique_inverse_noalloc",
     "hs_unique_inverse_workspace", "hs_retrieve_topk", "hs_retrieve_topk_n",
     "hs_retrieve_topk_fanout", "hs_merge_queries", "hs_retrieve_topk_workspace",
-    "hs_scatter_results", "hs_rerank_topk", "hs_segment_sum", "hs_get_device_error", "hs_launch_count", "hs_version",
+    "hs_scatter_results", "hs_rerank_topk", "hs_segment_sum", "ResultCache",
+    "hs_cache_bytes", "hs_cache_init", "hs_cache_lookup", "hs_cache_insert", "hs_cache_stats", "hs_get_device_error", "hs_launch_count", "hs_version",
     "library_path", "load", "EmbedRetrieveStage", "HostFeed", "RetrieveGraph", "StepGraph",
 ]

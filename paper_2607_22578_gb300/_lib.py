@@ -80,6 +80,16 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
             lib.hs_merge_queries.restype = st
             lib.hs_rerank_topk.argtypes = [P, i64, P, P, i64, i32, P, i32, i32, P, i64, P, P, P]
             lib.hs_rerank_topk.restype = st
+            lib.hs_cache_bytes.argtypes = [i64, i32, i32]
+            lib.hs_cache_bytes.restype = sz
+            lib.hs_cache_init.argtypes = [P, sz, i64, i32, i32, P]
+            lib.hs_cache_init.restype = st
+            lib.hs_cache_lookup.argtypes = [P, sz, i64, i32, i32, P, P, P, i64, P, P, P, P, P, P, P]
+            lib.hs_cache_lookup.restype = st
+            lib.hs_cache_insert.argtypes = [P, sz, i64, i32, i32, P, P, i64, P, P, P, P, P, P, P, P]
+            lib.hs_cache_insert.restype = st
+            lib.hs_cache_stats.argtypes = [P, P, P, P]
+            lib.hs_cache_stats.restype = st
             lib.hs_segment_sum.argtypes = [P, P, i64, P, i64, P, P]
             lib.hs_segment_sum.restype = st
             lib.hs_scatter_results.argtypes = [P, i64, i64, P, i64, P, P]
@@ -373,6 +383,80 @@ def hs_rerank_topk(rerank_queries: torch.Tensor, rerank_corpus: torch.Tensor,
                                  _ptr(inverse), rows if inverse is not None else 0, _ptr(scores),
                                  _ptr(ids), _stream(stream)))
     return scores, ids
+
+
+class ResultCache:
+    """Device-resident fingerprint -> retrieval result table that persists
+    across batches (asynchronous cache reuse, Section 3.3 (II)): ``capacity``
+    entries of a dim-wide query vector and its k scores and ids, in one
+    uint8 tensor allocated here (the library itself allocates nothing)."""
+
+    def __init__(self, capacity: int, dim: int, k: int, device=None, stream=None):
+        self.capacity, self.dim, self.k = int(capacity), int(dim), int(k)
+        nbytes = int(load().hs_cache_bytes(self.capacity, self.dim, self.k))
+        if nbytes == 0:
+            raise ValueError("invalid cache shape")
+        self.mem = torch.empty(nbytes, dtype=torch.uint8, device=device or "cuda")
+        hs_cache_init(self, stream)
+
+    def _args(self):
+        return (_ptr(self.mem), self.mem.numel(), self.capacity, self.dim, self.k)
+
+
+def hs_cache_init(cache: ResultCache, stream=None) -> None:
+    """Empty the cache (every entry free, counters zero)."""
+    _check(load().hs_cache_init(*cache._args(), _stream(stream)))
+
+
+def hs_cache_bytes(capacity: int, dim: int, k: int) -> int:
+    return int(load().hs_cache_bytes(capacity, dim, k))
+
+
+def hs_cache_lookup(cache: ResultCache, queries: torch.Tensor, fp: torch.Tensor,
+                    fp_rows: torch.Tensor | None = None, n_queries_dev: torch.Tensor | None = None,
+                    out: tuple | None = None, miss: tuple | None = None, stream=None):
+    """Look the merged queries up in the cache.  Hits get their cached
+    (scores, ids) rows in ``out``; misses are listed in ``miss`` =
+    (miss_list [Q] int32, n_miss_dev [1] int32, miss_queries [Q, dim]) with
+    their vectors gathered for retrieval.  Query u's key is fp[fp_rows[u]]
+    (fp[u] if fp_rows is None).  Returns (out, miss)."""
+    for t, name in ((queries, "queries"), (fp, "fp")):
+        _cuda(t, name)
+    Q, d = queries.shape
+    dev = queries.device
+    if out is None:
+        out = (torch.empty((Q, cache.k), dtype=torch.float32, device=dev),
+               torch.empty((Q, cache.k), dtype=torch.int32, device=dev))
+    if miss is None:
+        miss = (torch.empty(max(Q, 1), dtype=torch.int32, device=dev),
+                torch.empty(1, dtype=torch.int32, device=dev),
+                torch.empty((max(Q, 1), d), dtype=queries.dtype, device=dev))
+    _check(load().hs_cache_lookup(*cache._args(), _ptr(queries), _ptr(fp), _ptr(fp_rows), Q,
+                                  _ptr(n_queries_dev), _ptr(out[0]), _ptr(out[1]), _ptr(miss[0]),
+                                  _ptr(miss[1]), _ptr(miss[2]), _stream(stream)))
+    return out, miss
+
+
+def hs_cache_insert(cache: ResultCache, miss: tuple, fp: torch.Tensor, miss_scores: torch.Tensor,
+                    miss_ids: torch.Tensor, out: tuple, fp_rows: torch.Tensor | None = None,
+                    stream=None):
+    """Insert the retrieved results of the misses of ``hs_cache_lookup``
+    (rows of miss_scores / miss_ids follow the miss list) into the cache and
+    write them to the queries' rows of ``out``."""
+    miss_list, n_miss, miss_q = miss
+    _check(load().hs_cache_insert(*cache._args(), _ptr(miss_list), _ptr(n_miss),
+                                  miss_list.numel(), _ptr(miss_q), _ptr(fp), _ptr(fp_rows),
+                                  _ptr(miss_scores), _ptr(miss_ids), _ptr(out[0]), _ptr(out[1]),
+                                  _stream(stream)))
+    return out
+
+
+def hs_cache_stats(cache: ResultCache, stream=None):
+    """(hits, misses) counted since the cache was initialised (synchronises)."""
+    h, m = ctypes.c_uint64(0), ctypes.c_uint64(0)
+    _check(load().hs_cache_stats(_ptr(cache.mem), ctypes.addressof(h), ctypes.addressof(m),
+                                 _stream(stream)))
+    return int(h.value), int(m.value)
 
 
 def hs_segment_sum(phi: torch.Tensor, inverse: torch.Tensor, max_groups: int,

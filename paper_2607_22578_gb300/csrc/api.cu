@@ -25,6 +25,15 @@ hs_status launch_segment_sum(const double*, const int32_t*, int64_t, const int32
 hs_status launch_rerank(const uint16_t*, int64_t, const int32_t*, const uint16_t*, int64_t, int32_t,
                         const int32_t*, int32_t, int32_t, const int32_t*, int64_t, float*,
                         int32_t*, cudaStream_t);
+size_t cache_bytes(int64_t, int32_t, int32_t);
+hs_status launch_cache_init(void*, int64_t, int32_t, int32_t, cudaStream_t);
+hs_status launch_cache_lookup(void*, int64_t, int32_t, int32_t, const uint16_t*, const uint64_t*,
+                              const int32_t*, int64_t, const int32_t*, float*, int32_t*, int32_t*,
+                              int32_t*, uint16_t*, cudaStream_t);
+hs_status launch_cache_insert(void*, int64_t, int32_t, int32_t, const int32_t*, const int32_t*,
+                              int64_t, const uint16_t*, const uint64_t*, const int32_t*,
+                              const float*, const int32_t*, float*, int32_t*, cudaStream_t);
+hs_status cache_stats(const void*, unsigned long long*, unsigned long long*, cudaStream_t);
 hs_status launch_merge_queries(const uint16_t*, int64_t, int32_t, uint64_t, const uint64_t*,
                                uint64_t*, int32_t*, int32_t*, int32_t*, uint16_t*, cudaStream_t);
 hs_status launch_scatter(const void*, int64_t, int64_t, const int32_t*, int64_t, void*,
@@ -296,6 +305,95 @@ hs_status hs_rerank_topk(const uint16_t* rerank_queries, int64_t max_queries,
   return launch_rerank(rerank_queries, max_queries, n_queries_dev, rerank_corpus, n_corpus, dim,
                        candidates, k1, k2, inverse, n_out, scores_out, ids_out,
                        reinterpret_cast<cudaStream_t>(stream));
+}
+
+size_t hs_cache_bytes(int64_t capacity, int32_t dim, int32_t k) {
+  if (capacity < 1 || capacity > (1LL << 30) || dim < 8 || dim % 8 != 0 || dim > 65536 || k < 1 ||
+      k > HS_TOPK_MAX_K)
+    return 0;
+  return cache_bytes(capacity, dim, k);
+}
+
+static hs_status cache_check(const void* cache, size_t bytes, int64_t capacity, int32_t dim,
+                             int32_t k) {
+  const size_t need = hs_cache_bytes(capacity, dim, k);
+  if (need == 0)
+    return fail(HS_ERR_INVALID_ARG, "cache shape: capacity in [1, 2^30], dim %% 8 == 0 in "
+                                    "[8, 65536], k in [1, %d]", HS_TOPK_MAX_K);
+  if (!cache || !aligned(cache, 256))
+    return fail(HS_ERR_WORKSPACE, "cache NULL or not 256-byte aligned");
+  if (bytes < need) return fail(HS_ERR_WORKSPACE, "cache too small: %zu < %zu", bytes, need);
+  return HS_OK;
+}
+
+hs_status hs_cache_init(void* cache, size_t cache_bytes_, int64_t capacity, int32_t dim, int32_t k,
+                        hs_stream_t stream) {
+  clear_msg();
+  const hs_status st = cache_check(cache, cache_bytes_, capacity, dim, k);
+  if (st != HS_OK) return st;
+  return launch_cache_init(cache, capacity, dim, k, reinterpret_cast<cudaStream_t>(stream));
+}
+
+hs_status hs_cache_lookup(void* cache, size_t cache_bytes_, int64_t capacity, int32_t dim,
+                          int32_t k, const uint16_t* queries, const uint64_t* fp,
+                          const int32_t* fp_rows, int64_t max_queries,
+                          const int32_t* n_queries_dev, float* scores_out, int32_t* ids_out,
+                          int32_t* miss_list, int32_t* n_miss_dev, uint16_t* miss_queries,
+                          hs_stream_t stream) {
+  clear_msg();
+  const hs_status st = cache_check(cache, cache_bytes_, capacity, dim, k);
+  if (st != HS_OK) return st;
+  if (max_queries < 0 || max_queries > 0x7fffffffLL)
+    return fail(HS_ERR_INVALID_ARG, "max_queries outside [0, 2^31 - 1]");
+  if (!n_miss_dev || !aligned(n_miss_dev, 4))
+    return fail(HS_ERR_INVALID_ARG, "n_miss_dev NULL or misaligned");
+  if (max_queries > 0) {
+    if (!queries || !fp || !scores_out || !ids_out || !miss_list || !miss_queries)
+      return fail(HS_ERR_INVALID_ARG, "NULL input or output pointer");
+    if (!aligned(queries, 16) || !aligned(miss_queries, 16) || !aligned(fp, 8) ||
+        !aligned(scores_out, 4) || !aligned(ids_out, 4) || !aligned(miss_list, 4) ||
+        (fp_rows && !aligned(fp_rows, 4)) || (n_queries_dev && !aligned(n_queries_dev, 4)))
+      return fail(HS_ERR_INVALID_ARG, "misaligned pointer");
+  }
+  return launch_cache_lookup(cache, capacity, dim, k, queries, fp, fp_rows, max_queries,
+                             n_queries_dev, scores_out, ids_out, miss_list, n_miss_dev,
+                             miss_queries, reinterpret_cast<cudaStream_t>(stream));
+}
+
+hs_status hs_cache_insert(void* cache, size_t cache_bytes_, int64_t capacity, int32_t dim,
+                          int32_t k, const int32_t* miss_list, const int32_t* n_miss_dev,
+                          int64_t max_queries, const uint16_t* miss_queries, const uint64_t* fp,
+                          const int32_t* fp_rows, const float* miss_scores,
+                          const int32_t* miss_ids, float* scores_out, int32_t* ids_out,
+                          hs_stream_t stream) {
+  clear_msg();
+  const hs_status st = cache_check(cache, cache_bytes_, capacity, dim, k);
+  if (st != HS_OK) return st;
+  if (max_queries < 0 || max_queries > 0x7fffffffLL)
+    return fail(HS_ERR_INVALID_ARG, "max_queries outside [0, 2^31 - 1]");
+  if (max_queries == 0) return HS_OK;
+  if (!miss_list || !n_miss_dev || !miss_queries || !fp || !miss_scores || !miss_ids ||
+      !scores_out || !ids_out)
+    return fail(HS_ERR_INVALID_ARG, "NULL input or output pointer");
+  if (!aligned(miss_queries, 16) || !aligned(fp, 8) || !aligned(miss_list, 4) ||
+      !aligned(n_miss_dev, 4) || !aligned(miss_scores, 4) || !aligned(miss_ids, 4) ||
+      !aligned(scores_out, 4) || !aligned(ids_out, 4) || (fp_rows && !aligned(fp_rows, 4)))
+    return fail(HS_ERR_INVALID_ARG, "misaligned pointer");
+  return launch_cache_insert(cache, capacity, dim, k, miss_list, n_miss_dev, max_queries,
+                             miss_queries, fp, fp_rows, miss_scores, miss_ids, scores_out,
+                             ids_out, reinterpret_cast<cudaStream_t>(stream));
+}
+
+hs_status hs_cache_stats(const void* cache, uint64_t* hits, uint64_t* misses,
+                         hs_stream_t stream) {
+  clear_msg();
+  if (!cache || !hits || !misses) return fail(HS_ERR_INVALID_ARG, "NULL pointer");
+  unsigned long long h = 0, m = 0;
+  const hs_status st = cache_stats(cache, &h, &m, reinterpret_cast<cudaStream_t>(stream));
+  if (st != HS_OK) return st;
+  *hits = h;
+  *misses = m;
+  return HS_OK;
 }
 
 hs_status hs_segment_sum(const double* phi, const int32_t* inverse, int64_t n_rows,

@@ -10,6 +10,8 @@ Composition of the C-ABI calls only (no arithmetic here):
            -> hs_retrieve_topk_fanout               (one retrieval per merged node,
                                                      results written to every
                                                      originating query)
+  cached:  hs_cache_lookup -> hs_retrieve_topk_n of the misses -> hs_cache_insert
+           -> hs_scatter_results (results reused across batches, Section 3.3 (II))
   rerank:  hs_retrieve_topk_n -> hs_scatter_results (rerank vectors of the
            merged queries) -> hs_rerank_topk        (top-k rescored, best kept,
                                                      fanned out; Section 4.1)
@@ -30,7 +32,7 @@ class EmbedRetrieveStage:
 
     def __init__(self, corpus: torch.Tensor, k: int, max_queries: int,
                  max_chunk_rows: int = 0, rerank_corpus: torch.Tensor | None = None,
-                 rerank_k: int = 0):
+                 rerank_k: int = 0, cache_capacity: int = 0):
         if not corpus.is_cuda:
             raise TypeError("corpus must be resident on the GPU")
         self.corpus = corpus
@@ -52,6 +54,17 @@ class EmbedRetrieveStage:
         self.uq = torch.empty((mq, self.d), dtype=corpus.dtype, device=dev)
         self.scores = torch.empty((mq, self.k), dtype=torch.float32, device=dev)
         self.ids = torch.empty((mq, self.k), **i32)
+        # results reused across batches (Section 3.3 (II)): merged queries
+        # found in the cache skip retrieval
+        self.cache = None
+        if cache_capacity > 0:
+            self.cache = _lib.ResultCache(cache_capacity, self.d, self.k, device=dev)
+            self.miss = (torch.empty(mq, **i32), torch.empty(1, **i32),
+                         torch.empty((mq, self.d), dtype=corpus.dtype, device=dev))
+            self.m_s = torch.empty((mq, self.k), dtype=torch.float32, device=dev)
+            self.m_i = torch.empty((mq, self.k), **i32)
+            self.c_s = torch.empty((mq, self.k), dtype=torch.float32, device=dev)
+            self.c_i = torch.empty((mq, self.k), **i32)
         # second stage (RAG with rerank): k candidates rescored, rerank_k kept
         self.rerank_corpus, self.rerank_k = rerank_corpus, int(rerank_k)
         if rerank_corpus is not None:
@@ -92,6 +105,31 @@ class EmbedRetrieveStage:
         nu, inv, uq = self._merge_queries(queries)
         return self._retrieve_merged(uq, nu, inv, events) + (nu,)
 
+    def _retrieve_cached(self, uq, nu, inv, events):
+        """Lookup of the merged queries, retrieval of the misses only, insert
+        of their results, fan-out to every query."""
+        Q = inv.shape[0]
+        fp, uidx = self.q_fp[:Q], self.q_out[1][:Q]
+        out = (self.c_s[:Q], self.c_i[:Q])
+        miss = (self.miss[0][:Q], self.miss[1], self.miss[2][:Q])
+        _lib.hs_cache_lookup(self.cache, uq, fp, fp_rows=uidx, n_queries_dev=nu, out=out,
+                             miss=miss)
+        if events is not None:
+            events[0].record()
+        _lib.hs_retrieve_topk_n(miss[2], miss[1], self.corpus, self.k, workspace=self.ws_r,
+                                out=(self.m_s[:Q], self.m_i[:Q]))
+        if events is not None:
+            events[1].record()
+        _lib.hs_cache_insert(self.cache, miss, fp, self.m_s[:Q], self.m_i[:Q], out,
+                             fp_rows=uidx)
+        scores = _lib.hs_scatter_results(out[0], inv, dst=self.scores[:Q])
+        ids = _lib.hs_scatter_results(out[1], inv, dst=self.ids[:Q])
+        return scores, ids
+
+    def cache_stats(self):
+        """(hits, misses) of the result cache since the stage was built."""
+        return _lib.hs_cache_stats(self.cache)
+
     def retrieve_rerank(self, queries: torch.Tensor, rerank_queries: torch.Tensor):
         """RAG with rerank (Section 4.1): merged retrieval of the top-k, then
         the k candidates of each merged query rescored with its rerank
@@ -130,6 +168,8 @@ class EmbedRetrieveStage:
 
     def _retrieve_merged(self, uq, nu, inv, events):
         Q = inv.shape[0]
+        if self.cache is not None:
+            return self._retrieve_cached(uq, nu, inv, events)
         if events is not None:
             events[0].record()
         scores, ids = _lib.hs_retrieve_topk_fanout(uq, nu, inv, self.corpus, self.k,
