@@ -671,6 +671,56 @@ def row_rerank(args, dev, peaks) -> dict:
                           "candidate ids + map entry + k2 results"}
 
 
+def row_cache(args, dev, peaks) -> dict:
+    """Cross-batch reuse (Section 3.3 (II)): a stream of RAG-mix-sized
+    batches whose queries repeat across batches (Zipf(1.1) over a pool of
+    distinct queries), retrieved against the 1,048,576 x 768 corpus with and
+    without the result cache."""
+    import numpy as np
+    import torch
+
+    import paper_2607_22578_gb300 as hs
+    import synth
+    from synth import configs
+    cfg = configs.RAG_MIX
+    corpus = _dev_array(configs.build_retrieval_mix(cfg, seed=args.seed)["corpus"], dev)
+    N, d = corpus.shape
+    B, pool_n, n_batches, k = 2048, 50_000, 24, cfg["k"]
+    pool = synth.unit_rows(pool_n, d, args.seed + 31)
+    rng = np.random.default_rng(args.seed + 32)
+    p = np.arange(1, pool_n + 1, dtype=np.float64) ** -1.1
+    p /= p.sum()
+    batches = [_dev_array(pool[rng.choice(pool_n, B, p=p)], dev) for _ in range(n_batches)]
+    out = {"workload": "cache: %d batches x %d queries drawn Zipf(1.1) from %d distinct, "
+                       "corpus %d x %d, k=%d" % (n_batches, B, pool_n, N, d, k),
+           "metric": "queries/s over the batch stream", "arms": {}}
+    for name, cap in (("no_cache", 0), ("cache_65536", 65536)):
+        stage = hs.EmbedRetrieveStage(corpus, k, max_queries=B, cache_capacity=cap)
+        stage.retrieve(batches[0])                      # builds the kernels' state once
+        torch.cuda.synchronize()
+        if cap:
+            stage.cache.mem.zero_()
+            hs.hs_cache_init(stage.cache)
+        e0, e1 = _ev(), _ev()
+        e0.record()
+        for qb in batches:
+            stage.retrieve(qb)
+        e1.record()
+        torch.cuda.synchronize()
+        hs.hs_get_device_error()
+        ms = e0.elapsed_time(e1)
+        arm = {"ms_total": ms, "queries_per_s": B * n_batches / (ms / 1e3)}
+        if cap:
+            h, m = stage.cache_stats()
+            arm.update(hits=h, misses=m, hit_rate=h / max(h + m, 1))
+        out["arms"][name] = arm
+        del stage
+    out["value"] = out["arms"]["cache_65536"]["queries_per_s"]
+    out["speedup_vs_no_cache"] = (out["arms"]["cache_65536"]["queries_per_s"] /
+                                  out["arms"]["no_cache"]["queries_per_s"])
+    return out
+
+
 def rag_mix_breakdown(stage, tokens, queries, K: int) -> dict:
     """Per-phase device time of the RAG-mix step (the same calls as the
     pipeline, with events between them)."""
@@ -712,7 +762,8 @@ def rows_arm(args) -> int:
     dev = torch.device("cuda", 0)
     peaks, kind = load_peaks()
     fn = {"dedup_heavy": row_dedup_heavy, "batch_sweep": row_batch_sweep,
-          "large_corpus": row_large_corpus, "rerank": row_rerank}[args.workload]
+          "large_corpus": row_large_corpus, "rerank": row_rerank,
+          "cache": row_cache}[args.workload]
     line = fn(args, dev, peaks)
     line["peaks"] = {"hbm_gbs": peaks["hbm_gbs"], "bf16_tflops": peaks["bf16_tflops"],
                      "source": kind}
@@ -731,7 +782,8 @@ def main() -> int:
                     help="seconds of host time for the oracle baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--workload", default="rag_mix",
-                    choices=["rag_mix", "dedup_heavy", "batch_sweep", "large_corpus", "rerank"],
+                    choices=["rag_mix", "dedup_heavy", "batch_sweep", "large_corpus", "rerank",
+                             "cache"],
                     help="rag_mix is the headline step; the others measure the other "
                          "rows of the hot-path table (one GPU)")
     ap.add_argument("--k", type=int, default=0, help="override k (large_corpus only)")
