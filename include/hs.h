@@ -49,7 +49,7 @@ typedef struct CUstream_st* hs_stream_t;
 typedef enum {
   HS_OK = 0,
   HS_ERR_INVALID_ARG = 1, /* bad size, pointer, alignment or (device) data  */
-  HS_ERR_UNSUPPORTED = 2, /* valid request this build does not handle       */
+  HS_ERR_UNSUPPORTED = 2, /* valid request the library does not handle      */
   HS_ERR_CUDA = 3,        /* a CUDA runtime/driver call failed              */
   HS_ERR_WORKSPACE = 4,   /* workspace pointer NULL/misaligned or too small */
   HS_ERR_TIMEOUT = 5      /* a bounded device-side wait ran out             */
