@@ -284,15 +284,18 @@ __global__ void __launch_bounds__(256) fingerprint_words_kernel(
 template <int VB, int K, int NB>
 hs_status launch_chunks(const int32_t* tokens, int64_t n, int32_t stride, const int32_t* lens,
                         uint64_t seed, uint64_t* fp_out, int64_t sms, cudaStream_t stream) {
-  // Resident warps per SM at this kernel's register count (one query per
-  // process; the kernel uses no shared memory).
-  static int warps_per_sm = 0;
+  // Resident warps per SM at this kernel's register count (queried once per
+  // device; the kernel uses no shared memory).
+  static std::atomic<int> per_device[kMaxDeviceOrdinals];
+  const int dev = device_ordinal();
+  int warps_per_sm = dev >= 0 ? per_device[dev].load() : 0;
   if (warps_per_sm == 0) {
     int blocks = 0;
     const cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
         &blocks, fingerprint_chunks_kernel<VB, K, NB>, 256, 0);
     if (e != cudaSuccess) return cuda_fail(e, "fingerprint occupancy");
     warps_per_sm = blocks > 0 ? blocks * 8 : 8;
+    if (dev >= 0) per_device[dev].store(warps_per_sm);
   }
   const int64_t warps_target = sms * warps_per_sm;
   int64_t rpw = (n + warps_target - 1) / warps_target;

@@ -3,6 +3,8 @@
 // the fifth-generation tensor cores (tcgen05) of sm_103a.
 #pragma once
 
+#include <atomic>
+
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -329,4 +331,27 @@ unsigned* device_error_word();  // device address of the current device's error 
 int num_sms();
 void clear_last_error();
 void count_launches(unsigned n);  // diagnostics: kernels launched by this library
+
+constexpr int kMaxDeviceOrdinals = 64;
+
+// Ordinal of the current device, or -1 (none, or >= kMaxDeviceOrdinals).
+inline int device_ordinal() {
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDeviceOrdinals) return -1;
+  return dev;
+}
+
+// Runs `setup` once per device for one call site (`done` holds a bit per
+// device ordinal): kernel attributes such as the dynamic shared memory
+// limit belong to a device, so each device a process uses needs its own.
+template <class F>
+hs_status once_per_device(std::atomic<uint64_t>& done, F&& setup) {
+  const int dev = device_ordinal();
+  if (dev < 0) return setup();
+  const uint64_t bit = 1ull << dev;
+  if (done.load(std::memory_order_acquire) & bit) return HS_OK;
+  const hs_status st = setup();
+  if (st == HS_OK) done.fetch_or(bit, std::memory_order_release);
+  return st;
+}
 }  // namespace hs

@@ -1130,22 +1130,22 @@ int p2_for(int64_t nsplit, int32_t k) {
 
 template <int KREG, int CL>
 hs_status configure_kernel() {
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(retrieve_kernel<KREG, CL>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)Ring<CL>::smem);
-    if (e != cudaSuccess) return cuda_fail(e, "retrieve smem attribute");
-    configured = true;
-  }
-  return HS_OK;
+  static std::atomic<uint64_t> done{0};
+  return once_per_device(done, [] {
+    return cuda_fail(cudaFuncSetAttribute(retrieve_kernel<KREG, CL>,
+                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                          (int)Ring<CL>::smem),
+                     "retrieve smem attribute");
+  });
 }
 
 // Clusters of two that can be resident at once (one CTA per SM; pairs must
 // share a GPC), cached per kernel variant.
 template <int KREG>
 int64_t max_pairs() {
-  static int64_t cached = -1;
+  static std::atomic<int64_t> per_device[kMaxDeviceOrdinals];   // 0: not yet queried
+  const int dev = device_ordinal();
+  int64_t cached = dev >= 0 ? per_device[dev].load() - 1 : -1;
   if (cached < 0) {
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr[1];
@@ -1161,6 +1161,7 @@ int64_t max_pairs() {
     int n = 0;
     if (cudaOccupancyMaxActiveClusters(&n, retrieve_kernel<KREG, 2>, &cfg) != cudaSuccess) n = 0;
     cached = n;
+    if (dev >= 0) per_device[dev].store(cached + 1);
   }
   return cached;
 }
@@ -1295,12 +1296,13 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
     }
     const int64_t mgrid = nr < sms * 8 ? nr : sms * 8;
     const size_t msmem = (size_t)p2_for(max_splits(sms, pm.tiles, pm.k), pm.k) * 8;
-    static size_t merge_configured = 0;
-    if (msmem > 48 * 1024 && msmem > merge_configured) {
+    static std::atomic<size_t> merge_configured[kMaxDeviceOrdinals];   // per device
+    const int dev = device_ordinal();
+    if (msmem > 48 * 1024 && (dev < 0 || msmem > merge_configured[dev].load())) {
       cudaError_t e = cudaFuncSetAttribute(merge_kernel,
                                            cudaFuncAttributeMaxDynamicSharedMemorySize, (int)msmem);
       if (e != cudaSuccess) return cuda_fail(e, "merge smem attribute");
-      merge_configured = msmem;
+      if (dev >= 0) merge_configured[dev].store(msmem);
     }
     merge_kernel<<<(unsigned)mgrid, 256, msmem, stream>>>(pm, os, oi, kout, orows);
     return cuda_fail(cudaGetLastError(), "merge launch");
@@ -1311,13 +1313,14 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
     CUtensorMap mq16, mc128;
     if (!make_map(&mq16, queries, Qmax, d, SQ_N) || !make_map(&mc128, corpus, N, d, SQ_BM))
       return fail(HS_ERR_CUDA, "cuTensorMapEncodeTiled failed (driver entry point or arguments)");
-    static bool sq_configured = false;
-    if (!sq_configured) {
-      const cudaError_t e = cudaFuncSetAttribute(
-          retrieve_small_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SQ_SMEM);
-      if (e != cudaSuccess) return cuda_fail(e, "retrieve smem attribute");
-      sq_configured = true;
-    }
+    static std::atomic<uint64_t> sq_configured{0};
+    const hs_status cst = once_per_device(sq_configured, [] {
+      return cuda_fail(cudaFuncSetAttribute(retrieve_small_kernel,
+                                            cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                            (int)SQ_SMEM),
+                       "retrieve smem attribute");
+    });
+    if (cst != HS_OK) return cst;
     // Lists per query = 2 * nsplit of the plan the merge kernel recomputes
     // (one query block, one group: nsplit = min(slots, tiles, 8192 / k)).
     prm.slots = (int32_t)std::max<int64_t>(1, sms / 2);

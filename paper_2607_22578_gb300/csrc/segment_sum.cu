@@ -180,13 +180,14 @@ hs_status launch_segment_sum(const double* phi, const int32_t* inverse, int64_t 
     if (e != cudaSuccess) return cuda_fail(e, "output clear");
   }
   if (n == 0) return HS_OK;
-  static bool configured = false;
-  if (!configured) {
-    const cudaError_t e = cudaFuncSetAttribute(
-        segment_sum_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSsSmem);
-    if (e != cudaSuccess) return cuda_fail(e, "segment sum smem attribute");
-    configured = true;
-  }
+  static std::atomic<uint64_t> configured{0};
+  const hs_status cst = once_per_device(configured, [] {
+    return cuda_fail(cudaFuncSetAttribute(segment_sum_kernel,
+                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                          (int)kSsSmem),
+                     "segment sum smem attribute");
+  });
+  if (cst != HS_OK) return cst;
   const int64_t blocks = (n + kSsCtaRows - 1) / kSsCtaRows;
   const int64_t cap = (int64_t)num_sms() * 4;
   const unsigned grid = (unsigned)(blocks < cap ? blocks : cap);

@@ -524,13 +524,15 @@ hs_status launch_small(const uint64_t* fp, const int32_t* tokens, int64_t n, int
                        int32_t* inverse, uint32_t* ctr, int32_t* coll_list, unsigned* err,
                        cudaStream_t stream) {
   const size_t smem = small_smem(n);
-  static size_t configured = 0;
-  if (smem > 48 * 1024 && smem > configured) {
-    const cudaError_t e = cudaFuncSetAttribute(unique_small_kernel<VEC>,
-                                               cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                               (int)small_smem(kSmallRows));
-    if (e != cudaSuccess) return cuda_fail(e, "unique smem attribute");
-    configured = small_smem(kSmallRows);
+  static std::atomic<uint64_t> configured{0};
+  if (smem > 48 * 1024) {
+    const hs_status cst = once_per_device(configured, [] {
+      return cuda_fail(cudaFuncSetAttribute(unique_small_kernel<VEC>,
+                                            cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                            (int)small_smem(kSmallRows)),
+                       "unique smem attribute");
+    });
+    if (cst != HS_OK) return cst;
   }
   // One CTA per 2 warp-rounds of rows (they wait on memory), at most one per SM.
   const unsigned grid = grid_for((n + 31) / 32, 2, num_sms());
