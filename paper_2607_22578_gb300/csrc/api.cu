@@ -109,7 +109,7 @@ extern "C" {
 
 const char* hs_last_error(void) { return g_msg; }
 
-const char* hs_version(void) { return "hs 0.1 (sm_103a)"; }
+const char* hs_version(void) { return "hs 0.2 (sm_103a)"; }
 
 uint64_t hs_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
 
