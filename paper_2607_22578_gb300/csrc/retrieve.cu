@@ -98,6 +98,9 @@ struct Params {
   // 0 = none), raised with atomicMax and read once per tile by every list of
   // the query.  Zeroed before each launch.
   uint32_t* qfloor;
+  // Optional, one word per query block: a unit whose query blocks are all 0
+  // here is skipped (the exact large-k pass re-runs only the flagged blocks).
+  const uint32_t* only;
 };
 
 // Rows the merge writes: with inv NULL one per query (row q = query q);
@@ -168,6 +171,19 @@ __device__ __forceinline__ void unit_coords(const SplitPlan& sp, int64_t tiles, 
   split = (int)(u / sp.groups);
   t0 = (int64_t)split * tiles / sp.nsplit;
   t1 = (int64_t)(split + 1) * tiles / sp.nsplit;
+}
+
+// True when `only` is set and no query block of unit u's group is flagged.
+// Every role of a CTA pair evaluates it for the same units, so all skip alike.
+__device__ __forceinline__ bool unit_skipped(const Params& p, const SplitPlan& sp, int64_t u,
+                                             int cl) {
+  if (!p.only) return false;
+  const int g = (int)(u % sp.groups);
+  for (int r = 0; r < cl; ++r) {
+    const int qb = g * cl + r;
+    if (qb < sp.qblocks && p.only[qb] != 0u) return false;
+  }
+  return true;
 }
 
 __device__ __forceinline__ float max3f(float a, float b, float c) {
@@ -360,6 +376,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint64_t pol_q = policy_evict_last();
       uint32_t stage = 0, phase = 0;
       for (int64_t u = u0; u < units; u += ustep) {
+        if (unit_skipped(p, sp, u, CL)) continue;
         int qb, split;
         int64_t t0, t1;
         unit_coords(sp, p.tiles, u, rank, CL, qb, split, t0, t1);
@@ -401,6 +418,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       constexpr uint32_t idesc = idesc_bf16_f32(BM * CL, BN);
       uint32_t stage = 0, phase = 0, tile_i = 0;
       for (int64_t u = u0; u < units; u += ustep) {
+        if (unit_skipped(p, sp, u, CL)) continue;
         int qb, split;
         int64_t t0, t1;
         unit_coords(sp, p.tiles, u, rank, CL, qb, split, t0, t1);
@@ -456,6 +474,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     float* Ls = p.list_s + ((size_t)blockIdx.x * kEpi + et) * 2 * (size_t)k;
     int32_t* Li = p.list_i + ((size_t)blockIdx.x * kEpi + et) * 2 * (size_t)k;
     for (int64_t u = u0; u < units; u += ustep) {
+      if (unit_skipped(p, sp, u, CL)) continue;
       int qb, split;
       int64_t t0, t1;
       unit_coords(sp, p.tiles, u, rank, CL, qb, split, t0, t1);
@@ -782,10 +801,17 @@ __global__ void __launch_bounds__(256) merge_warp_kernel(const Params p, float* 
 
 // Lists of p.k entries per (query, split, half) -> the kout best per query.
 // With out_i NULL only the kout-th best score of each query is written, to
-// out_s[q] (the floor of the second large-k pass).
+// out_s[q] (the floor of the second large-k pass).  With `only` set, rows
+// whose query block is not flagged there are skipped.  With `flag_out` set,
+// a query's block is flagged when one of its lists may have cut off a member
+// of the top kout: a full list whose last (k-th) entry is not below the
+// union's kout-th best.  A list whose last entry is below that score holds
+// every row of its range that can be in the top kout, so with no list
+// flagged the union's first kout entries are exact.
 __global__ void __launch_bounds__(256) merge_kernel(const Params p, float* __restrict__ out_s,
                                                     int32_t* __restrict__ out_i, int32_t kout,
-                                                    OutRows rows) {
+                                                    OutRows rows, uint32_t* flag_out,
+                                                    const uint32_t* only) {
   extern __shared__ uint64_t keys[];
   const int64_t Q = query_count(p);
   const SplitPlan sp = split_plan(Q, p.tiles, p.k, p.slots, p.cl);
@@ -803,6 +829,7 @@ __global__ void __launch_bounds__(256) merge_kernel(const Params p, float* __res
       if (threadIdx.x == 0) set_error(p.err, kErrInvalidArg);
       continue;
     }
+    if (only && only[q / BM] == 0u) continue;      // block-uniform
     const float* ps = part_s + (size_t)q * m;
     const int32_t* pi = part_i + (size_t)q * m;
     for (int e = threadIdx.x; e < p2; e += blockDim.x) keys[e] = e < m ? pack_key(ps[e], pi[e]) : 0ull;
@@ -822,6 +849,13 @@ __global__ void __launch_bounds__(256) merge_kernel(const Params p, float* __res
         }
         __syncthreads();
       }
+    }
+    if (flag_out) {
+      const uint64_t kth = kout - 1 < m ? keys[kout - 1] : 0ull;
+      bool cut = false;
+      for (int l = threadIdx.x; l < lists; l += blockDim.x)
+        cut |= pack_key(ps[(size_t)l * k + k - 1], pi[(size_t)l * k + k - 1]) >= kth;
+      if (__syncthreads_or(cut) && threadIdx.x == 0) atomicOr(flag_out + q / BM, 1u);
     }
     if (!out_i) {
       if (threadIdx.x == 0) {
@@ -1236,7 +1270,9 @@ size_t retrieve_topk_workspace(int64_t Q, int64_t N, int32_t d, int32_t k) {
   const size_t part = (((size_t)Q * 2 * ns * k * 4) + 255) & ~(size_t)255;
   const size_t list = k <= 32 ? 0 : ((((size_t)sms * kEpi * 2 * k * 4) + 255) & ~(size_t)255);
   const size_t qfloor = (((size_t)Q * 4) + 255) & ~(size_t)255;
-  return 2 * part + 2 * list + 2 * qfloor + 256;   // shared floors + large-k floors
+  const size_t flags = ((((size_t)(Q + BM - 1) / BM) * 4) + 255) & ~(size_t)255;
+  // lists, large-k lists, shared floors, large-k floors, block flags
+  return 2 * part + 2 * list + 2 * qfloor + flags + 256;
 }
 
 // Qmax rows of `queries` are addressable; the kernels process the first
@@ -1275,6 +1311,8 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
   const size_t qfloor_bytes = (((size_t)Qmax * 4) + 255) & ~(size_t)255;
   prm.qfloor = reinterpret_cast<uint32_t*>(w + 2 * part + 2 * list);
   float* kth = reinterpret_cast<float*>(w + 2 * part + 2 * list + qfloor_bytes);
+  uint32_t* block_flags =
+      reinterpret_cast<uint32_t*>(w + 2 * part + 2 * list + 2 * qfloor_bytes);
   prm.err = err;
   const bool small = Qmax <= SQ_N && k <= 32 && prm.kb_count <= SQ_MAXKB;
   if (!small) {
@@ -1284,11 +1322,12 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
   }
   const OutRows rows{inv, n_out};
   const int64_t R = inv ? n_out : Qmax;             // rows the final merge writes
-  auto merge = [&](const Params& pm, int32_t kout, float* os, int32_t* oi,
-                   OutRows orows) -> hs_status {
+  auto merge = [&](const Params& pm, int32_t kout, float* os, int32_t* oi, OutRows orows,
+                   uint32_t* flag_out = nullptr, const uint32_t* only = nullptr) -> hs_status {
     const int64_t nr = orows.inv ? orows.n_out : Qmax;
     if (nr == 0) return HS_OK;
-    if (oi && kout <= 32 && 2 * (int64_t)pm.slots <= 32 * kMaxListsPerLane) {
+    if (oi && kout <= 32 && !flag_out && !only &&
+        2 * (int64_t)pm.slots <= 32 * kMaxListsPerLane) {
       const int64_t blocks = (nr + 7) / 8;          // one warp per row
       merge_warp_kernel<<<(unsigned)(blocks < sms * 16 ? blocks : sms * 16), 256, 0, stream>>>(
           pm, os, oi, kout, orows);
@@ -1304,7 +1343,7 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
       if (e != cudaSuccess) return cuda_fail(e, "merge smem attribute");
       if (dev >= 0) merge_configured[dev].store(msmem);
     }
-    merge_kernel<<<(unsigned)mgrid, 256, msmem, stream>>>(pm, os, oi, kout, orows);
+    merge_kernel<<<(unsigned)mgrid, 256, msmem, stream>>>(pm, os, oi, kout, orows, flag_out, only);
     return cuda_fail(cudaGetLastError(), "merge launch");
   };
   hs_status st;
@@ -1339,35 +1378,55 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
   } else if (k <= 32) {
     st = launch_variant<32>(corpus, N, d, mq, prm, stream);
   } else {
-    // Large k, two passes.  Pass 1 runs the register-list kernel (32 per
-    // list) over the first eighth of the corpus; the k-th best of the union
-    // of its lists is a score that k distinct corpus rows reach, hence at
-    // most the query's final k-th best: a floor.  Pass 2 runs the large-k
-    // kernel over the whole corpus keeping only scores >= the floor, which
-    // leaves few candidates per list.  Both passes' lists go through the
-    // same workspace; the floors (one score per query) are staged in it.
+    // Large k.  With at least 64 corpus tiles an optimistic pass runs first:
+    // the register-list kernel (32 per list, no shared floor: a floor that
+    // bounds 32nd-best scores would cut rows of the top k) over the whole
+    // corpus, merged to the first k of the union of its lists.  A list whose
+    // last entry is below the union's k-th best holds every row of its range
+    // that can be in the top k, so where no list of a query is cut that way
+    // the union's first k are exact.  The merge flags the query blocks where
+    // some list may have been cut; only those take the exact two-pass path
+    // (pass 1: register lists over the first eighth of the corpus, whose
+    // union's k-th best is a score k distinct rows reach, hence a floor;
+    // pass 2: the large-k kernel over the whole corpus keeping scores >= the
+    // floor), and every kernel of it skips the other blocks.  Both passes'
+    // lists go through the same workspace; the floors are staged in it.
     if (tiles >= 64) {
+      const int64_t nb = (Qmax + BM - 1) / BM;
+      cudaError_t ze = cudaMemsetAsync(block_flags, 0, (size_t)nb * 4, stream);
+      if (ze != cudaSuccess) return cuda_fail(ze, "flag clear");
+      Params pa = prm;
+      pa.k = 32;
+      pa.qfloor = nullptr;
+      pa.floor = nullptr;
+      st = launch_variant<32>(corpus, N, d, mq, pa, stream);
+      if (st != HS_OK) return st;
+      st = merge(pa, k, scores_out, ids_out, rows, block_flags, nullptr);
+      if (st != HS_OK) return st;
+      count_launches(2);
       Params p1 = prm;
       p1.tiles = tiles / 8;
       p1.N = p1.tiles * BN;
       p1.k = 32;
       p1.floor = nullptr;
+      p1.only = block_flags;
       st = launch_variant<32>(corpus, N, d, mq, p1, stream);
       if (st != HS_OK) return st;
-      st = merge(p1, k, kth, nullptr, OutRows{nullptr, 0});
+      st = merge(p1, k, kth, nullptr, OutRows{nullptr, 0}, nullptr, block_flags);
       if (st != HS_OK) return st;
       count_launches(2);
       prm.floor = kth;
       prm.floor_stride = 1;
       prm.floor_index = 0;
+      prm.only = block_flags;
       // Pass 1's shared floors bound 32nd-best scores, not k-th best: clear.
-      const cudaError_t ze2 = cudaMemsetAsync(prm.qfloor, 0, (size_t)Qmax * 4, stream);
-      if (ze2 != cudaSuccess) return cuda_fail(ze2, "floor clear");
+      ze = cudaMemsetAsync(prm.qfloor, 0, (size_t)Qmax * 4, stream);
+      if (ze != cudaSuccess) return cuda_fail(ze, "floor clear");
     }
     st = launch_variant<0>(corpus, N, d, mq, prm, stream);
   }
   if (st != HS_OK) return st;
-  st = merge(prm, k, scores_out, ids_out, rows);
+  st = merge(prm, k, scores_out, ids_out, rows, nullptr, prm.only);
   if (st != HS_OK) return st;
   count_launches(R > 0 ? 2 : 1);  // retrieve_kernel + merge_kernel
   return HS_OK;

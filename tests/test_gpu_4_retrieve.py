@@ -306,3 +306,33 @@ def test_tiny_corpus_edges(nq, N, d, k):
     Q, C = unit_pair(nq, N, d, nq + 3 * N)
     gs, gi = gpu_topk(to_dev(Q), to_dev(C), k)
     parity(Q, C, k, gs, gi, range(nq))
+
+
+@pytest.mark.parametrize("hot", [0, 150])
+def test_large_k_optimistic_pass_and_exact_fallback(hot):
+    """k > 32 over >= 64 tiles: the optimistic register-list pass is exact
+    when no list is cut; queries whose top-k crowds into one list's corpus
+    range (here 200 contiguous near-copies of their direction) are flagged
+    and recomputed by the exact two-pass path."""
+    N, d, k, Q = 64 * 256 * 2, 128, 100, 300
+    rng = np.random.default_rng(7 + hot)
+    corpus = synth.unit_rows(N, d, 31)
+    q = synth.unit_rows(Q, d, 32)
+    if hot:
+        base = (q[0].astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+        noise = rng.standard_normal((200, d)) * 0.02
+        rows = base / np.linalg.norm(base) + noise
+        rows /= np.linalg.norm(rows, axis=1, keepdims=True)
+        corpus[1000:1200] = (rows.astype(np.float32).view(np.uint32) >> 16).astype(np.uint16)
+        q[1:hot] = q[0]
+    s, i = hs.hs_retrieve_topk(to_dev(q), to_dev(corpus), k)
+    hs.hs_get_device_error()
+    s, i = s.cpu().numpy(), i.cpu().numpy()
+    sample = np.unique(np.concatenate([np.arange(0, Q, 37), [0, 1, hot]]))
+    sample = sample[sample < Q]
+    os_, oi = oracle.topk(q[sample], corpus, k + 1)
+    for r, qq in enumerate(sample):
+        exact = oracle.pair_scores(q, corpus, np.full(k, qq), i[qq])
+        check_topk(s[qq], i[qq], os_[r], oi[r], exact, N, k)
+    if hot:
+        assert set(range(1000, 1100)) & set(i[0].tolist())   # the crowded rows are found
