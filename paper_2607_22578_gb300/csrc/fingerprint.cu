@@ -56,6 +56,8 @@ __global__ void __launch_bounds__(256) fingerprint_chunks_kernel(
     const int32_t* __restrict__ tokens, int64_t n, int32_t stride,
     const int32_t* __restrict__ lens, uint64_t seed, uint64_t* __restrict__ fp_out,
     int64_t rows_per_warp) {
+  pdl_wait();
+  pdl_trigger();
   constexpr int W = VB / 4;  // tokens per vector load
   constexpr int T = W * K;   // tokens per chunk
   static_assert(T == kTailChunk, "chunk size shared with the tail kernel");
@@ -175,6 +177,8 @@ __global__ void __launch_bounds__(256) fingerprint_tails_kernel(
     const int32_t* __restrict__ tokens, int64_t n, int32_t stride,
     const int32_t* __restrict__ lens, uint64_t seed, uint64_t* __restrict__ fp_out,
     unsigned* err) {
+  pdl_wait();
+  pdl_trigger();
   constexpr int T = kTailChunk;
   for (int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; r < n;
        r += (int64_t)gridDim.x * blockDim.x) {
@@ -213,6 +217,8 @@ __global__ void __launch_bounds__(256) fingerprint_words_kernel(
     const int32_t* __restrict__ tokens, int64_t n, int32_t stride,
     const int32_t* __restrict__ lens, uint64_t seed, uint64_t* __restrict__ fp_out,
     int64_t rows_per_warp, unsigned* err) {
+  pdl_wait();
+  pdl_trigger();
   const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int64_t r_begin = warp * rows_per_warp;
   if (r_begin >= n) return;
@@ -304,8 +310,8 @@ hs_status launch_chunks(const int32_t* tokens, int64_t n, int32_t stride, const 
   // Few warps: one-warp blocks, so they spread over all SMs.
   const int threads = warps >= sms * 8 ? 256 : 32;
   const int64_t blocks = (warps * 32 + threads - 1) / threads;
-  fingerprint_chunks_kernel<VB, K, NB><<<(unsigned)blocks, threads, 0, stream>>>(
-      tokens, n, stride, lens, seed, fp_out, rpw);
+  launch_pdl(fingerprint_chunks_kernel<VB, K, NB>, dim3((unsigned)blocks), dim3(threads), 0, stream,
+             tokens, n, stride, lens, seed, fp_out, rpw);
   count_launches(1);
   return HS_OK;
 }
@@ -331,8 +337,8 @@ hs_status launch_fingerprint(const int32_t* tokens, int64_t n, int32_t stride,
     if (lens || stride % kTailChunk != 0 || stride == 0) {
       int64_t blocks = (n + 255) / 256;
       if (blocks > sms * 64) blocks = sms * 64;
-      fingerprint_tails_kernel<<<(unsigned)blocks, 256, 0, stream>>>(tokens, n, stride, lens,
-                                                                     seed, fp_out, err);
+      launch_pdl(fingerprint_tails_kernel, dim3((unsigned)blocks), dim3(256), 0, stream, tokens, n,
+                 stride, lens, seed, fp_out, err);
       count_launches(1);
     }
   } else {
@@ -341,8 +347,8 @@ hs_status launch_fingerprint(const int32_t* tokens, int64_t n, int32_t stride,
     if (rpw < 32) rpw = 32;
     const int64_t warps = (n + rpw - 1) / rpw;
     const int64_t blocks = (warps + 7) / 8;
-    fingerprint_words_kernel<<<(unsigned)blocks, 256, 0, stream>>>(tokens, n, stride, lens, seed,
-                                                                   fp_out, rpw, err);
+    launch_pdl(fingerprint_words_kernel, dim3((unsigned)blocks), dim3(256), 0, stream, tokens, n,
+               stride, lens, seed, fp_out, rpw, err);
     count_launches(1);
   }
   return cuda_fail(cudaGetLastError(), "fingerprint launch");

@@ -323,6 +323,18 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
 
 }  // namespace hs
 
+// ---- programmatic dependent launch ---------------------------------------------------
+// Kernels launched with launch_pdl may be scheduled while the kernel before
+// them on the stream is still running; each such kernel calls pdl_wait()
+// before it touches global memory (the wait returns once the previous grid
+// has completed and its writes are visible), then pdl_trigger() so that the
+// kernel after it may be scheduled in turn.  Only launch latency and the
+// prologue overlap the previous kernel; no data is read early.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // ---- host-side internals (api.cu) -------------------------------------------------------
 namespace hs {
 hs_status fail(hs_status s, const char* fmt, ...);
@@ -333,6 +345,23 @@ void clear_last_error();
 void count_launches(unsigned n);  // diagnostics: kernels launched by this library
 
 constexpr int kMaxDeviceOrdinals = 64;
+
+// Launch with programmatic stream serialization (see pdl_wait).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t stream, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
 
 // Ordinal of the current device, or -1 (none, or >= kMaxDeviceOrdinals).
 inline int device_ordinal() {

@@ -48,6 +48,8 @@ __global__ void __launch_bounds__(kQmThreads) merge_queries_kernel(
     const uint4* __restrict__ q, int n, int nv, uint64_t seed, const uint64_t* __restrict__ fp_in,
     uint64_t* __restrict__ fp_out, int32_t* __restrict__ n_unique,
     int32_t* __restrict__ unique_idx, int32_t* __restrict__ inverse, uint4* __restrict__ uq) {
+  pdl_wait();
+  pdl_trigger();
   __shared__ uint64_t s_fp[kQmMaxRows];
   __shared__ uint64_t s_keys[kQmSlots];
   __shared__ uint32_t s_idx[kQmSlots];
@@ -228,9 +230,9 @@ hs_status launch_merge_queries(const uint16_t* queries, int64_t n, int32_t dim, 
   const int64_t work = n * (int64_t)nv;
   int64_t grid = (work + kQmThreads * kQmUnroll - 1) / (kQmThreads * kQmUnroll);
   grid = grid < 1 ? 1 : (grid > kQmMaxCtas ? kQmMaxCtas : grid);
-  merge_queries_kernel<<<(unsigned)grid, kQmThreads, 0, stream>>>(
-      reinterpret_cast<const uint4*>(queries), (int)n, nv, seed, fp_in, fp_out, n_unique,
-      unique_idx, inverse, reinterpret_cast<uint4*>(uq));
+  launch_pdl(merge_queries_kernel, dim3((unsigned)grid), dim3(kQmThreads), 0, stream,
+             reinterpret_cast<const uint4*>(queries), (int)n, nv, seed, fp_in, fp_out, n_unique,
+             unique_idx, inverse, reinterpret_cast<uint4*>(uq));
   count_launches(1);
   return cuda_fail(cudaGetLastError(), "merge_queries launch");
 }

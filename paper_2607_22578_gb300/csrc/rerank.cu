@@ -44,6 +44,8 @@ __global__ void __launch_bounds__(kRrThreads) rerank_kernel(
     const uint4* __restrict__ rc, int64_t n_rc, int nv, const int32_t* __restrict__ cand, int k1,
     int k2, const int32_t* __restrict__ inv, int64_t n_out, float* __restrict__ out_s,
     int32_t* __restrict__ out_i, unsigned* err) {
+  pdl_wait();
+  pdl_trigger();
   const int lane = threadIdx.x & 31;
   int64_t Q = Qmax;
   if (count_dev) {
@@ -122,9 +124,10 @@ hs_status launch_rerank(const uint16_t* rq, int64_t Qmax, const int32_t* count_d
   int64_t grid = (rows + warps_per_cta - 1) / warps_per_cta;
   const int64_t cap = (int64_t)num_sms() * 16;
   if (grid > cap) grid = cap;
-  rerank_kernel<<<(unsigned)grid, kRrThreads, 0, stream>>>(
-      reinterpret_cast<const uint4*>(rq), Qmax, count_dev, reinterpret_cast<const uint4*>(rc),
-      n_rc, d / 8, cand, k1, k2, inv, n_out, out_s, out_i, err);
+  launch_pdl(rerank_kernel, dim3((unsigned)grid), dim3(kRrThreads), 0, stream,
+             reinterpret_cast<const uint4*>(rq), Qmax, count_dev,
+             reinterpret_cast<const uint4*>(rc), n_rc, d / 8, cand, k1, k2, inv, n_out, out_s,
+             out_i, err);
   count_launches(1);
   return cuda_fail(cudaGetLastError(), "rerank launch");
 }

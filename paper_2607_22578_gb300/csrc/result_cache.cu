@@ -99,6 +99,8 @@ __device__ __forceinline__ bool rows_equal(const uint4* a, const uint4* b, int n
 }
 
 __global__ void cache_init_kernel(CacheView c) {
+  pdl_wait();
+  pdl_trigger();
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t s = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; s < c.slots; s += stride) {
     c.state[s] = kEmptyState;
@@ -129,6 +131,8 @@ __global__ void __launch_bounds__(256) cache_lookup_kernel(
     const int32_t* __restrict__ rows, int64_t Qmax, const int32_t* __restrict__ count_dev,
     float* __restrict__ out_s, int32_t* __restrict__ out_i, int32_t* __restrict__ miss_list,
     int32_t* __restrict__ n_miss, uint4* __restrict__ miss_q, unsigned* err) {
+  pdl_wait();
+  pdl_trigger();
   if (!header_ok(c, err)) return;
   const int lane = threadIdx.x & 31;
   const int nv = c.dim / 8, k = c.k;
@@ -188,6 +192,8 @@ __global__ void __launch_bounds__(256) cache_insert_kernel(
     const int32_t* __restrict__ rows, const float* __restrict__ miss_s,
     const int32_t* __restrict__ miss_i, float* __restrict__ out_s, int32_t* __restrict__ out_i,
     unsigned* err) {
+  pdl_wait();
+  pdl_trigger();
   if (!header_ok(c, err)) return;
   const int lane = threadIdx.x & 31;
   const int nv = c.dim / 8, k = c.k;
@@ -259,7 +265,8 @@ hs_status launch_cache_init(void* cache, int64_t capacity, int32_t dim, int32_t 
                             cudaStream_t stream) {
   const CacheView c = view_of(cache, slots_for(capacity), dim, k);
   const int64_t blocks = ((int64_t)c.slots + 255) / 256;
-  cache_init_kernel<<<(unsigned)(blocks < 4096 ? blocks : 4096), 256, 0, stream>>>(c);
+  launch_pdl(cache_init_kernel, dim3((unsigned)(blocks < 4096 ? blocks : 4096)), dim3(256), 0,
+             stream, c);
   count_launches(1);
   return cuda_fail(cudaGetLastError(), "cache init launch");
 }
@@ -278,9 +285,9 @@ hs_status launch_cache_lookup(void* cache, int64_t capacity, int32_t dim, int32_
   int64_t grid = (Qmax + 7) / 8;
   const int64_t cap = (int64_t)num_sms() * 8;
   if (grid > cap) grid = cap;
-  cache_lookup_kernel<<<(unsigned)grid, 256, 0, stream>>>(
-      c, reinterpret_cast<const uint4*>(queries), fp, rows, Qmax, count_dev, out_s, out_i,
-      miss_list, n_miss, reinterpret_cast<uint4*>(miss_q), err);
+  launch_pdl(cache_lookup_kernel, dim3((unsigned)grid), dim3(256), 0, stream, c,
+             reinterpret_cast<const uint4*>(queries), fp, rows, Qmax, count_dev, out_s, out_i,
+             miss_list, n_miss, reinterpret_cast<uint4*>(miss_q), err);
   count_launches(1);
   return cuda_fail(cudaGetLastError(), "cache lookup launch");
 }
@@ -297,9 +304,9 @@ hs_status launch_cache_insert(void* cache, int64_t capacity, int32_t dim, int32_
   const int64_t cap = (int64_t)num_sms() * 8;
   if (grid > cap) grid = cap;
   if (grid < 1) grid = 1;
-  cache_insert_kernel<<<(unsigned)grid, 256, 0, stream>>>(
-      c, miss_list, n_miss, Qmax, reinterpret_cast<const uint4*>(miss_q), fp, rows, miss_s,
-      miss_i, out_s, out_i, err);
+  launch_pdl(cache_insert_kernel, dim3((unsigned)grid), dim3(256), 0, stream, c, miss_list, n_miss,
+             Qmax, reinterpret_cast<const uint4*>(miss_q), fp, rows, miss_s, miss_i, out_s, out_i,
+             err);
   count_launches(1);
   return cuda_fail(cudaGetLastError(), "cache insert launch");
 }

@@ -734,6 +734,8 @@ constexpr int kMaxListsPerLane = 10;
 __global__ void __launch_bounds__(256) merge_warp_kernel(const Params p, float* __restrict__ out_s,
                                                          int32_t* __restrict__ out_i,
                                                          int32_t kout, OutRows rows) {
+  pdl_wait();
+  pdl_trigger();
   const int64_t Q = query_count(p);
   const SplitPlan sp = split_plan(Q, p.tiles, p.k, p.slots, p.cl);
   const int k = p.k;
@@ -812,6 +814,8 @@ __global__ void __launch_bounds__(256) merge_kernel(const Params p, float* __res
                                                     int32_t* __restrict__ out_i, int32_t kout,
                                                     OutRows rows, uint32_t* flag_out,
                                                     const uint32_t* only) {
+  pdl_wait();
+  pdl_trigger();
   extern __shared__ uint64_t keys[];
   const int64_t Q = query_count(p);
   const SplitPlan sp = split_plan(Q, p.tiles, p.k, p.slots, p.cl);
@@ -1329,8 +1333,8 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
     if (oi && kout <= 32 && !flag_out && !only &&
         2 * (int64_t)pm.slots <= 32 * kMaxListsPerLane) {
       const int64_t blocks = (nr + 7) / 8;          // one warp per row
-      merge_warp_kernel<<<(unsigned)(blocks < sms * 16 ? blocks : sms * 16), 256, 0, stream>>>(
-          pm, os, oi, kout, orows);
+      launch_pdl(merge_warp_kernel, dim3((unsigned)(blocks < sms * 16 ? blocks : sms * 16)),
+                 dim3(256), 0, stream, pm, os, oi, kout, orows);
       return cuda_fail(cudaGetLastError(), "merge launch");
     }
     const int64_t mgrid = nr < sms * 8 ? nr : sms * 8;
@@ -1343,7 +1347,8 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
       if (e != cudaSuccess) return cuda_fail(e, "merge smem attribute");
       if (dev >= 0) merge_configured[dev].store(msmem);
     }
-    merge_kernel<<<(unsigned)mgrid, 256, msmem, stream>>>(pm, os, oi, kout, orows, flag_out, only);
+    launch_pdl(merge_kernel, dim3((unsigned)mgrid), dim3(256), msmem, stream, pm, os, oi, kout,
+               orows, flag_out, only);
     return cuda_fail(cudaGetLastError(), "merge launch");
   };
   hs_status st;

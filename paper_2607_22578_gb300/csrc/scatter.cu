@@ -34,6 +34,8 @@ __global__ void __launch_bounds__(256) scatter_kernel(const T* __restrict__ src,
                                                       int64_t n_rows, uint32_t cpr,
                                                       uint64_t magic, T* __restrict__ dst,
                                                       unsigned* err) {
+  pdl_wait();
+  pdl_trigger();
   const int64_t total = n_rows * (int64_t)cpr;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t g0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g0 < total; g0 += stride * U) {
@@ -77,9 +79,9 @@ hs_status launch_typed(const void* src, int64_t n_src, int64_t row_bytes, const 
   uint64_t magic = 0;
   const unsigned __int128 span = (unsigned __int128)(uint64_t)(total > 0 ? total - 1 : 0) * (uint64_t)cpr;
   if (cpr > 0 && (span >> 64) == 0) magic = ~0ull / (uint64_t)cpr + 1ull;
-  scatter_kernel<T, U><<<(unsigned)blocks, 256, 0, stream>>>(
-      static_cast<const T*>(src), n_src, map, n_rows, (uint32_t)cpr, magic, static_cast<T*>(dst),
-      err);
+  launch_pdl(scatter_kernel<T, U>, dim3((unsigned)blocks), dim3(256), 0, stream,
+             static_cast<const T*>(src), n_src, map, n_rows, (uint32_t)cpr, magic,
+             static_cast<T*>(dst), err);
   count_launches(1);
   return cuda_fail(cudaGetLastError(), "scatter launch");
 }

@@ -87,6 +87,8 @@ __global__ void __launch_bounds__(kSsThreads) segment_sum_kernel(
     const double* __restrict__ phi, const int32_t* __restrict__ inverse, int64_t n,
     const int32_t* __restrict__ count_dev, int64_t max_groups, double* __restrict__ out,
     unsigned* err) {
+  pdl_wait();
+  pdl_trigger();
   extern __shared__ __align__(16) uint8_t sm[];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   double* cta_sums = reinterpret_cast<double*>(sm);
@@ -191,8 +193,8 @@ hs_status launch_segment_sum(const double* phi, const int32_t* inverse, int64_t 
   const int64_t blocks = (n + kSsCtaRows - 1) / kSsCtaRows;
   const int64_t cap = (int64_t)num_sms() * 4;
   const unsigned grid = (unsigned)(blocks < cap ? blocks : cap);
-  segment_sum_kernel<<<grid, kSsThreads, kSsSmem, stream>>>(phi, inverse, n, count_dev,
-                                                            max_groups, out, err);
+  launch_pdl(segment_sum_kernel, dim3(grid), dim3(kSsThreads), kSsSmem, stream, phi, inverse, n,
+             count_dev, max_groups, out, err);
   count_launches(1);
   return cuda_fail(cudaGetLastError(), "segment sum launch");
 }

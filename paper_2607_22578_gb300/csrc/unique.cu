@@ -232,6 +232,8 @@ __device__ void peel_block(const uint64_t* __restrict__ fp, const int32_t* __res
 // ---- multi-kernel path ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) insert_kernel(const uint64_t* __restrict__ fp, int64_t n,
                                                      uint64_t* keys, uint32_t* idx, int log2T) {
+  pdl_wait();
+  pdl_trigger();
   for (int64_t base = (int64_t)blockIdx.x * blockDim.x; base < n;
        base += (int64_t)gridDim.x * blockDim.x) {
     const int64_t i = base + threadIdx.x;
@@ -246,6 +248,8 @@ __global__ void __launch_bounds__(256) verify_kernel(
     const uint32_t* __restrict__ idx, int log2T, const int32_t* __restrict__ tokens,
     int32_t stride, const int32_t* __restrict__ lens, int32_t* __restrict__ rep,
     int32_t* coll_list, uint32_t* ctr, unsigned* err) {
+  pdl_wait();
+  pdl_trigger();
   const int lane = threadIdx.x & 31;
   const int64_t warps = ((int64_t)gridDim.x * blockDim.x) >> 5;
   const int64_t w = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
@@ -273,6 +277,8 @@ __global__ void __launch_bounds__(1024) resolve_kernel(const uint64_t* __restric
                                                        const int32_t* __restrict__ lens,
                                                        int32_t* rep, const int32_t* coll_list,
                                                        const uint32_t* ctr, unsigned* err) {
+  pdl_wait();
+  pdl_trigger();
   const uint32_t m = ctr[kCtrColl];
   if (m == 0) return;
   peel_block<VEC>(fp, tokens, stride, lens, rep, coll_list, m, err);
@@ -303,6 +309,8 @@ __global__ void __launch_bounds__(kScanThreads) scan_kernel(const int32_t* __res
                                                             unsigned long long* status,
                                                             uint32_t* ctr, int32_t* total_out,
                                                             unsigned* err) {
+  pdl_wait();
+  pdl_trigger();
   __shared__ uint32_t s_tile;
   __shared__ int32_t s_warp[kScanThreads / 32];
   __shared__ int32_t s_prefix;
@@ -399,6 +407,8 @@ __global__ void __launch_bounds__(256) finalize_kernel(const int32_t* __restrict
                                                        const int32_t* __restrict__ n_unique,
                                                        int32_t* __restrict__ unique_idx,
                                                        int32_t* __restrict__ inverse) {
+  pdl_wait();
+  pdl_trigger();
   const int64_t nu = *n_unique;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
        i += (int64_t)gridDim.x * blockDim.x) {
@@ -422,6 +432,8 @@ __global__ void __launch_bounds__(kSmallThreads) unique_small_kernel(
     int32_t stride, const int32_t* __restrict__ lens, int32_t* __restrict__ n_unique,
     int32_t* __restrict__ unique_idx, int32_t* __restrict__ inverse, uint32_t* ctr,
     int32_t* coll_list, unsigned* err) {
+  pdl_wait();
+  pdl_trigger();
   extern __shared__ __align__(16) uint8_t sm[];
   __shared__ bool s_last;
   __shared__ int32_t s_warp[kSmallThreads / 32];
@@ -536,8 +548,8 @@ hs_status launch_small(const uint64_t* fp, const int32_t* tokens, int64_t n, int
   }
   // One CTA per 2 warp-rounds of rows (they wait on memory), at most one per SM.
   const unsigned grid = grid_for((n + 31) / 32, 2, num_sms());
-  unique_small_kernel<VEC><<<grid, kSmallThreads, smem, stream>>>(
-      fp, n, tokens, stride, lens, n_unique, unique_idx, inverse, ctr, coll_list, err);
+  launch_pdl(unique_small_kernel<VEC>, dim3(grid), dim3(kSmallThreads), smem, stream, fp, n, tokens,
+             stride, lens, n_unique, unique_idx, inverse, ctr, coll_list, err);
   return HS_OK;
 }
 
@@ -577,25 +589,26 @@ hs_status launch_unique_inverse(const uint64_t* fp, const int32_t* tokens, int64
   }
   e = cudaMemsetAsync(w + L.zero_end, 0xff, L.ones_end - L.zero_end, stream);
   if (e != cudaSuccess) return cuda_fail(e, "hash table clear");
-  insert_kernel<<<grid_for(n, 256, sms * 8), 256, 0, stream>>>(fp, n, keys, idx, L.log2T);
+  launch_pdl(insert_kernel, dim3(grid_for(n, 256, sms * 8)), dim3(256), 0, stream, fp, n, keys, idx,
+             L.log2T);
   const unsigned vgrid = grid_for(n, 256, sms * 8);   // one warp per 32 rows
   if (vec)
-    verify_kernel<true><<<vgrid, 256, 0, stream>>>(fp, n, keys, idx, L.log2T, tokens, stride,
-                                                   lens, rep, coll_list, ctr, err);
+    launch_pdl(verify_kernel<true>, dim3(vgrid), dim3(256), 0, stream, fp, n, keys, idx, L.log2T,
+               tokens, stride, lens, rep, coll_list, ctr, err);
   else
-    verify_kernel<false><<<vgrid, 256, 0, stream>>>(fp, n, keys, idx, L.log2T, tokens, stride,
-                                                    lens, rep, coll_list, ctr, err);
+    launch_pdl(verify_kernel<false>, dim3(vgrid), dim3(256), 0, stream, fp, n, keys, idx, L.log2T,
+               tokens, stride, lens, rep, coll_list, ctr, err);
   if (vec)
-    resolve_kernel<true><<<1, 1024, 0, stream>>>(fp, tokens, stride, lens, rep, coll_list, ctr,
-                                                 err);
+    launch_pdl(resolve_kernel<true>, dim3(1), dim3(1024), 0, stream, fp, tokens, stride, lens, rep,
+               coll_list, ctr, err);
   else
-    resolve_kernel<false><<<1, 1024, 0, stream>>>(fp, tokens, stride, lens, rep, coll_list, ctr,
-                                                  err);
+    launch_pdl(resolve_kernel<false>, dim3(1), dim3(1024), 0, stream, fp, tokens, stride, lens, rep,
+               coll_list, ctr, err);
   const int64_t tiles = (n + kScanTile - 1) / kScanTile;
-  scan_kernel<<<(unsigned)tiles, kScanThreads, 0, stream>>>(rep, n, uid, status, ctr,
-                                                           n_unique_dev, err);
-  finalize_kernel<<<grid_for(n, 256, sms * 8), 256, 0, stream>>>(rep, uid, n, n_unique_dev,
-                                                                 unique_idx, inverse);
+  launch_pdl(scan_kernel, dim3((unsigned)tiles), dim3(kScanThreads), 0, stream, rep, n, uid, status,
+             ctr, n_unique_dev, err);
+  launch_pdl(finalize_kernel, dim3(grid_for(n, 256, sms * 8)), dim3(256), 0, stream, rep, uid, n,
+             n_unique_dev, unique_idx, inverse);
   count_launches(5);  // insert, verify, resolve, scan, finalize
   return cuda_fail(cudaGetLastError(), "unique_inverse launch");
 }
