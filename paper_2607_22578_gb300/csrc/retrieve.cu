@@ -364,6 +364,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (CL > 1) cluster_sync();            // the pair's barriers exist before any remote signal
   const uint32_t tmem_base = *tmem_slot;
   const int rank = CL > 1 ? (int)cluster_ctarank() : 0;
+  // Everything above touched only shared memory, TMEM and the kernel
+  // parameters; global memory (the query count, queries, corpus) waits for
+  // the previous kernel on the stream.
+  pdl_wait();
+  pdl_trigger();
   const int64_t Q = query_count(p);
   const SplitPlan sp = split_plan(Q, p.tiles, p.k, p.slots, CL);
   const int64_t units = Q > 0 ? (int64_t)sp.groups * sp.nsplit : 0;
@@ -966,6 +971,8 @@ __global__ void __launch_bounds__(SQ_THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  pdl_wait();                            // global memory only after the previous kernel
+  pdl_trigger();
   const int64_t Q = query_count(p);
   const int k = p.k;
   const int64_t t0 = (int64_t)blockIdx.x * tiles128 / gridDim.x;
@@ -1208,17 +1215,19 @@ template <int KREG, int CL>
 hs_status launch_kernel(const CUtensorMap& mq, const CUtensorMap& mc, const Params& prm,
                         int64_t grid, cudaStream_t stream) {
   cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = CL;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = CL;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
   cfg.gridDim = dim3((unsigned)grid, 1, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = Ring<CL>::smem;
   cfg.stream = stream;
   cfg.attrs = attr;
-  cfg.numAttrs = CL > 1 ? 1 : 0;
+  cfg.numAttrs = CL > 1 ? 2 : 1;
   return cuda_fail(cudaLaunchKernelEx(&cfg, retrieve_kernel<KREG, CL>, mq, mc, prm),
                    "retrieve launch");
 }
@@ -1371,8 +1380,8 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
     prm.cl = 1;
     const SplitPlan sp = split_plan(1, tiles, k, prm.slots, 1);
     const int64_t grid = 2 * (int64_t)sp.nsplit;
-    retrieve_small_kernel<<<(unsigned)grid, SQ_THREADS, SQ_SMEM, stream>>>(
-        mq16, mc128, prm, (N + SQ_BM - 1) / SQ_BM);
+    launch_pdl(retrieve_small_kernel, dim3((unsigned)grid), dim3(SQ_THREADS), SQ_SMEM, stream,
+               mq16, mc128, prm, (N + SQ_BM - 1) / SQ_BM);
     st = cuda_fail(cudaGetLastError(), "retrieve launch");
   } else if (k <= 8) {
     st = launch_variant<8>(corpus, N, d, mq, prm, stream);
