@@ -159,7 +159,7 @@ def fanout_case(Q_max, n_real, n_out, N, d, k, seed):
     (1, 1, 3, 300, 64, 5),
     (300, 250, 400, 20000, 768, 10),   # CTA-pair kernel, register lists
     (64, 64, 70, 9000, 256, 32),
-    (40, 33, 50, 70000, 128, 100),     # two-pass large k: floors staged in the workspace
+    (40, 33, 50, 70000, 128, 100),     # large k over >= 64 tiles: the optimistic pass
     (20, 20, 21, 3000, 128, 300),      # large k, one pass
 ])
 def test_fanout_matches_scatter_and_oracle(Q_max, n_real, n_out, N, d, k):
@@ -181,3 +181,30 @@ def test_fanout_rejects_bad_map_entries():
     # n_out = 0 enqueues nothing
     hs.hs_retrieve_topk_fanout(queries, None, inv[:0], corpus, 7)
     hs.hs_get_device_error()
+
+
+def test_fanout_large_k_flagged_blocks_with_device_count():
+    """k > 32 with the exact fallback taken (a query whose top-k crowds into
+    one list's rows), a device-side query count and a fan-out map."""
+    N, d, k, Qmax, n_real = 64 * 256 * 2, 64, 100, 200, 150
+    corpus = synth.unit_rows(N, d, 61)
+    q = synth.unit_rows(Qmax, d, 62)
+    rng = np.random.default_rng(63)
+    base = (q[3].astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    rows = base / np.linalg.norm(base) + rng.standard_normal((180, d)) * 0.02
+    rows /= np.linalg.norm(rows, axis=1, keepdims=True)
+    corpus[5000:5180] = (rows.astype(np.float32).view(np.uint32) >> 16).astype(np.uint16)
+    inv = rng.integers(0, n_real, size=260).astype(np.int32)
+    inv[:4] = 3
+    cnt = to_dev(np.array([n_real], np.int32))
+    s, i = hs.hs_retrieve_topk_fanout(to_dev(q), cnt, to_dev(inv), to_dev(corpus), k)
+    hs.hs_get_device_error()
+    s, i = s.cpu().numpy(), i.cpu().numpy()
+    used = np.unique(np.concatenate([[3], inv[::29]]))
+    os_, oi = oracle.topk(q[used], corpus, k + 1)
+    for r, qi in enumerate(used):
+        o = int(np.nonzero(inv == qi)[0][0])
+        exact = oracle.pair_scores(q, corpus, np.full(k, qi), i[o])
+        check_topk(s[o], i[o], os_[r], oi[r], exact, N, k)
+        rows_o = np.nonzero(inv == qi)[0]
+        assert (s[rows_o] == s[o]).all() and (i[rows_o] == i[o]).all()
