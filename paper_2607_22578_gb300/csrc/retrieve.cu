@@ -728,7 +728,7 @@ __device__ __forceinline__ void unpack_key(uint64_t key, float& s, int32_t& idx)
   idx = (int32_t)(0xffffffffu - (uint32_t)key);
 }
 
-// Small kout: one warp per query runs a tournament over the sorted lists.
+// One warp per query runs a tournament over the sorted lists.
 // Lane l owns lists l, l+32, ...; it keeps each list's head and the entry
 // after it (prefetched) in registers.  Each round the warp takes the largest
 // head (keys are unique: a corpus row lives in exactly one list; padding
@@ -736,9 +736,14 @@ __device__ __forceinline__ void unpack_key(uint64_t key, float& s, int32_t& idx)
 // best in order.
 constexpr int kMaxListsPerLane = 10;
 
+// Any kout: picks 0..31 are kept one per lane and written together when
+// kout <= 32; for larger kout each pick is written as it is made.  With
+// out_i NULL only the kout-th pick's score is written, to out_s[o].  `only`
+// and `flag_out` are as for merge_kernel.
 __global__ void __launch_bounds__(256) merge_warp_kernel(const Params p, float* __restrict__ out_s,
                                                          int32_t* __restrict__ out_i,
-                                                         int32_t kout, OutRows rows) {
+                                                         int32_t kout, OutRows rows,
+                                                         uint32_t* flag_out, const uint32_t* only) {
   pdl_wait();
   pdl_trigger();
   const int64_t Q = query_count(p);
@@ -754,6 +759,7 @@ __global__ void __launch_bounds__(256) merge_warp_kernel(const Params p, float* 
       if (lane == 0) set_error(p.err, kErrInvalidArg);
       continue;
     }
+    if (only && only[q / BM] == 0u) continue;      // warp-uniform
     const float* __restrict__ ps = p.part_s + (size_t)q * lists * k;
     const int32_t* __restrict__ pi = p.part_i + (size_t)q * lists * k;
     uint64_t head[kMaxListsPerLane], next[kMaxListsPerLane];
@@ -767,6 +773,7 @@ __global__ void __launch_bounds__(256) merge_warp_kernel(const Params p, float* 
     }
     float my_s = -FLT_MAX;
     int32_t my_i = -1;
+    uint64_t last = 0ull;                          // key of the latest pick
     for (int r = 0; r < kout; ++r) {
       uint64_t best = 0ull;
       int bj = 0;
@@ -778,13 +785,20 @@ __global__ void __launch_bounds__(256) merge_warp_kernel(const Params p, float* 
         }
       uint64_t mx = best;
 #pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        const uint64_t y = __shfl_xor_sync(0xffffffffu, mx, o);
+      for (int sh = 16; sh > 0; sh >>= 1) {
+        const uint64_t y = __shfl_xor_sync(0xffffffffu, mx, sh);
         mx = y > mx ? y : mx;
       }
       const unsigned win = __ballot_sync(0xffffffffu, best == mx && mx != 0ull);
-      if (lane == r) {
-        if (mx != 0ull) unpack_key(mx, my_s, my_i);
+      last = mx;
+      if (kout <= 32) {
+        if (lane == r && mx != 0ull) unpack_key(mx, my_s, my_i);
+      } else if (out_i && lane == 0) {
+        float sc = -FLT_MAX;
+        int32_t id = -1;
+        if (mx != 0ull) unpack_key(mx, sc, id);
+        out_s[(size_t)o * kout + r] = sc;
+        out_i[(size_t)o * kout + r] = id;
       }
       if (win != 0u && lane == __ffs(win) - 1) {
 #pragma unroll
@@ -799,9 +813,25 @@ __global__ void __launch_bounds__(256) merge_warp_kernel(const Params p, float* 
           }
       }
     }
-    if (lane < kout) {
+    if (out_i && kout <= 32 && lane < kout) {
       out_s[(size_t)o * kout + lane] = my_s;
       out_i[(size_t)o * kout + lane] = my_i;
+    }
+    if (!out_i && lane == 0) {
+      float sc = -FLT_MAX;
+      int32_t id = -1;
+      if (last != 0ull) unpack_key(last, sc, id);
+      out_s[o] = sc;
+    }
+    if (flag_out) {
+      bool cut = false;
+#pragma unroll
+      for (int j = 0; j < kMaxListsPerLane; ++j) {
+        const int l = j * 32 + lane;
+        if (l < lists)
+          cut |= pack_key(ps[(size_t)l * k + k - 1], pi[(size_t)l * k + k - 1]) >= last;
+      }
+      if (__any_sync(0xffffffffu, cut) && lane == 0) atomicOr(flag_out + q / BM, 1u);
     }
   }
 }
@@ -1339,11 +1369,10 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
                    uint32_t* flag_out = nullptr, const uint32_t* only = nullptr) -> hs_status {
     const int64_t nr = orows.inv ? orows.n_out : Qmax;
     if (nr == 0) return HS_OK;
-    if (oi && kout <= 32 && !flag_out && !only &&
-        2 * (int64_t)pm.slots <= 32 * kMaxListsPerLane) {
+    if (2 * (int64_t)pm.slots <= 32 * kMaxListsPerLane) {
       const int64_t blocks = (nr + 7) / 8;          // one warp per row
       launch_pdl(merge_warp_kernel, dim3((unsigned)(blocks < sms * 16 ? blocks : sms * 16)),
-                 dim3(256), 0, stream, pm, os, oi, kout, orows);
+                 dim3(256), 0, stream, pm, os, oi, kout, orows, flag_out, only);
       return cuda_fail(cudaGetLastError(), "merge launch");
     }
     const int64_t mgrid = nr < sms * 8 ? nr : sms * 8;
