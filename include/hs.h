@@ -354,10 +354,12 @@ hs_status hs_rerank_topk(const uint16_t* rerank_queries, int64_t max_queries,
  * misses (hs_retrieve_topk_n over miss_queries with count n_miss_dev) ->
  * hs_cache_insert of those results.  After the insert, row u of scores_out /
  * ids_out holds the top-k of query u, hit or miss.  Calls on one stream are
- * ordered, so each batch sees the inserts of the batches before it; calls on
- * different streams that share a cache race (a query that equals one still
- * being retrieved elsewhere misses and is retrieved again; no kernel waits
- * for another).
+ * ordered, so each batch sees the inserts of the batches before it.  Streams
+ * may share a cache: a query that equals one still being retrieved on
+ * another stream misses and is retrieved again (no kernel waits for
+ * another), and a lookup that overlaps an insert evicting the entry it reads
+ * sees the slot's generation change and takes the miss path, so a hit never
+ * returns a half-written or replaced entry.
  *
  * Arguments common to the cache calls:
  *   cache, cache_bytes   device memory, 256-byte aligned, at least

@@ -67,6 +67,7 @@ __global__ void __launch_bounds__(kRrThreads) rerank_kernel(
         set_error(err, kErrInvalidArg);
         id = -1;
       }
+      if (id < 0) id = -1;                                  // absent: written as -1
     }
     const uint4* qrow = rq + q * nv;
     float score = 0.0f;

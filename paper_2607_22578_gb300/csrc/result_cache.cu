@@ -25,13 +25,22 @@
 // batches before it.  A query that equals one still being retrieved by a
 // concurrent stream is not waited for: it misses and is retrieved again (a
 // kernel never waits for another kernel here).
+//
+// Concurrent streams.  A slot's state word carries, above its two state
+// bits, a generation count that every claim advances.  A lookup reads the
+// state, then the slot's key, vector and result (from L2, never from a
+// stale L1 line), then the state again: a hit needs both reads to show the
+// same ready generation.  An insert that claimed the slot in between (to
+// evict it) changes the word, and the lookup takes the miss path, so a hit
+// never returns a half-written or replaced entry.
 #include "hs_internal.cuh"
 
 namespace hs {
 namespace {
 
 constexpr int kWays = 8;
-constexpr uint32_t kEmptyState = 0, kBusy = 1, kReady = 2;
+constexpr uint32_t kEmptyState = 0, kBusy = 1, kReady = 2;   // state word: generation << 2 | state
+constexpr uint32_t kStateMask = 3u;
 constexpr uint32_t kMagic = 0x48534331u;   // "HSC1"
 
 struct CacheHeader {
@@ -92,7 +101,7 @@ __device__ __forceinline__ bool rows_equal(const uint4* a, const uint4* b, int n
   bool eq = true;
 #pragma unroll 1
   for (int v = lane; v < nv; v += 32) {
-    const uint4 x = __ldg(a + v), y = b[v];
+    const uint4 x = __ldg(a + v), y = __ldcg(b + v);
     eq &= x.x == y.x && x.y == y.y && x.z == y.z && x.w == y.w;
   }
   return __all_sync(0xffffffffu, eq);
@@ -148,26 +157,36 @@ __global__ void __launch_bounds__(256) cache_lookup_kernel(
     const uint32_t base = set_of(f, c.slots) * kWays;
     const uint4* qrow = queries + u * nv;
     bool match = false;
+    uint32_t st = 0;
     if (lane < kWays) {
-      const uint32_t st = *reinterpret_cast<volatile uint32_t*>(c.state + base + lane);
-      match = st == kReady && c.keys[base + lane] == f;
+      st = *reinterpret_cast<volatile uint32_t*>(c.state + base + lane);
+      __threadfence();   // order the state read before the key
+      match = (st & kStateMask) == kReady && __ldcg(c.keys + base + lane) == f;
     }
     unsigned cand = __ballot_sync(0xffffffffu, match);
     int hit = -1;
     while (cand && hit < 0) {
       const int w = __ffs(cand) - 1;
       cand &= cand - 1;
+      const uint32_t seen = __shfl_sync(0xffffffffu, st, w);
+      const uint32_t s = base + w;
       __threadfence();   // order the state read before the slot contents
-      if (rows_equal(qrow, reinterpret_cast<const uint4*>(c.vec) + (int64_t)(base + w) * nv, nv,
-                     lane))
-        hit = w;
+      if (!rows_equal(qrow, reinterpret_cast<const uint4*>(c.vec) + (int64_t)s * nv, nv, lane))
+        continue;
+      // copy the result, then confirm that no insert claimed the slot meanwhile;
+      // a row copied from a changed slot is overwritten by the miss path
+      for (int j = lane; j < k; j += 32) {
+        out_s[u * k + j] = __ldcg(c.scores + (int64_t)s * k + j);
+        out_i[u * k + j] = __ldcg(c.ids + (int64_t)s * k + j);
+      }
+      __syncwarp();
+      __threadfence();
+      uint32_t again = 0;
+      if (lane == 0) again = *reinterpret_cast<volatile uint32_t*>(c.state + s);
+      if (__shfl_sync(0xffffffffu, again, 0) == seen) hit = w;
     }
     if (hit >= 0) {
       const uint32_t s = base + hit;
-      for (int j = lane; j < k; j += 32) {
-        out_s[u * k + j] = c.scores[(int64_t)s * k + j];
-        out_i[u * k + j] = c.ids[(int64_t)s * k + j];
-      }
       if (lane == 0) {
         c.used[s] = epoch;
         atomicAdd(&c.hdr->hits, 1ull);
@@ -212,10 +231,11 @@ __global__ void __launch_bounds__(256) cache_insert_kernel(
     // claim a way: empty first, then least recently used; a way another
     // miss of this batch claimed first is skipped
     int claimed = -1;
+    uint32_t gen_busy = 0;
     for (int attempt = 0; attempt < kWays && claimed < 0; ++attempt) {
       uint32_t st = kBusy, age = 0xffffffffu;
       if (lane < kWays) {
-        st = *reinterpret_cast<volatile uint32_t*>(c.state + base + lane);
+        st = *reinterpret_cast<volatile uint32_t*>(c.state + base + lane) & kStateMask;
         age = st == kEmptyState ? 0u : (st == kReady ? c.used[base + lane] + 1u : 0xffffffffu);
       }
       // lowest (age, way) over the ways that are not busy
@@ -231,9 +251,16 @@ __global__ void __launch_bounds__(256) cache_insert_kernel(
       uint32_t ok = 0;
       if (lane == w) {
         const uint32_t seen = *reinterpret_cast<volatile uint32_t*>(c.state + base + w);
-        ok = seen != kBusy && atomicCAS(c.state + base + w, seen, kBusy) == seen;
+        const uint32_t busy = (((seen >> 2) + 1u) << 2) | kBusy;   // next generation
+        ok = (seen & kStateMask) != kBusy && atomicCAS(c.state + base + w, seen, busy) == seen
+                 ? busy : 0u;
+        __threadfence();   // the claim is visible before any write to the slot
       }
-      if (__shfl_sync(0xffffffffu, ok, w)) claimed = w;
+      ok = __shfl_sync(0xffffffffu, ok, w);
+      if (ok) {
+        claimed = w;
+        gen_busy = ok;
+      }
     }
     if (claimed < 0) continue;
     const uint32_t s = base + claimed;
@@ -249,7 +276,7 @@ __global__ void __launch_bounds__(256) cache_insert_kernel(
     }
     __threadfence();
     __syncwarp();
-    if (lane == 0) atomicExch(c.state + s, kReady);        // publish
+    if (lane == 0) atomicExch(c.state + s, (gen_busy & ~kStateMask) | kReady);   // publish
   }
   if (blockIdx.x == 0 && threadIdx.x == 0) atomicAdd(&c.hdr->epoch, 1u);
 }

@@ -69,9 +69,9 @@ def test_rerank_of_retrieval_candidates():
 def test_absent_duplicate_and_bad_candidates():
     rc = synth.unit_rows(100, 32, 7)
     rq = synth.unit_rows(3, 32, 8)
-    cand = np.array([[5, -1, 7, -1, 9],      # three present, k2 = 4
+    cand = np.array([[5, -1, 7, -7, 9],      # three present, k2 = 4
                      [4, 4, 8, 12, 16],      # a duplicated id is scored twice
-                     [-1, -1, -1, -1, -1]], np.int32)
+                     [-1, -2, -2147483648, -1, -1]], np.int32)   # any negative is absent
     s, i = run(rq, rc, cand, 4)
     os_, oi = oracle.rerank(rq, rc, cand, 4)
     assert (i == oi).all()

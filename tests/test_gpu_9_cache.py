@@ -103,3 +103,44 @@ def test_uninitialised_cache_is_rejected():
     hs.hs_cache_lookup(cache, q, torch.zeros(3, dtype=torch.int64, device="cuda"))
     with pytest.raises(hs.HsError):
         hs.hs_get_device_error()
+
+
+def test_two_streams_share_a_cache_without_torn_results():
+    """Two streams look up and insert into one small cache at the same time,
+    so inserts on one stream evict entries that lookups on the other may be
+    reading.  Every row, hit or miss, must be exactly its own query's top-k."""
+    d, k, pool_n, B = 256, 10, 48, 12
+    corpus = to_dev(synth.unit_rows(400000, d, 21))
+    pd = to_dev(synth.unit_rows(pool_n, d, 22))
+    fp_all = hs.hs_fingerprint(pd.view(torch.int32))
+    want_s = torch.empty((pool_n, k), dtype=torch.float32, device="cuda")
+    want_i = torch.empty((pool_n, k), dtype=torch.int32, device="cuda")
+    for c0 in range(0, pool_n, B):                   # the kernel the misses take (<= 16 rows)
+        s, i = hs.hs_retrieve_topk(pd[c0:c0 + B], corpus, k)
+        want_s[c0:c0 + B], want_i[c0:c0 + B] = s, i
+    rng = np.random.default_rng(23)
+    sels = torch.from_numpy(np.stack([rng.choice(pool_n, B, replace=False)
+                                      for _ in range(120)])).to("cuda")
+    torch.cuda.synchronize()
+    cache = hs.ResultCache(16, d, k)                 # two sets of eight ways: steady eviction
+    streams = [torch.cuda.Stream(), torch.cuda.Stream()]
+    for st in streams:
+        st.wait_stream(torch.cuda.current_stream())
+    outs = []
+    for it in range(sels.shape[0]):
+        st = streams[it % 2]
+        with torch.cuda.stream(st):
+            sel = sels[it]
+            q, f = pd[sel], fp_all[sel]
+            out, miss = hs.hs_cache_lookup(cache, q, f)
+            ms, mi = hs.hs_retrieve_topk_n(miss[2], miss[1], corpus, k)
+            hs.hs_cache_insert(cache, miss, f, ms, mi, out)
+            outs.append((it, out))
+    torch.cuda.synchronize()
+    hs.hs_get_device_error()
+    for it, (s, i) in outs:
+        sel = sels[it]
+        assert torch.equal(i, want_i[sel]), "batch %d returned another query's ids" % it
+        assert torch.equal(s, want_s[sel]), "batch %d returned another query's scores" % it
+    hits, misses = hs.hs_cache_stats(cache)
+    assert hits + misses == sels.numel() and hits > 0 and misses > 0
