@@ -12,8 +12,12 @@
 //      round, 16 lanes each).  A mismatch — rows with equal fingerprints but
 //      different contents — sends the row to a collision list;
 //   3. collision list (empty unless fingerprints collide): exact regrouping
-//      by peeling — the smallest unassigned row becomes a representative and
-//      every listed row equal to it joins it;
+//      in linear work — the listed rows are grouped again by a second key
+//      (a different hash of the row, mixed with its fingerprint) in the now
+//      free table, and each is compared with the smallest listed row of its
+//      group; rows that collide in both keys (practically never) are peeled:
+//      the smallest unassigned one becomes a representative and every one
+//      equal to it joins it;
 //   4. exclusive sum-scan of "row is its own representative" gives each
 //      group its ordinal in first-occurrence order (single pass, decoupled
 //      look-back with bounded spins); the final kernel writes unique_idx and
@@ -39,6 +43,7 @@ static_assert(kScanThreads % 32 == 0 && kScanThreads <= 1024, "scan block: whole
 constexpr int kLookBatch = 8;           // predecessor statuses read per round trip
 constexpr int64_t kSmallRows = 4096;    // single-launch path
 constexpr int kSmallThreads = 512;
+constexpr int kResolveThreads = 512;    // one block for the collision list
 
 constexpr size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
@@ -155,7 +160,7 @@ __device__ __forceinline__ bool warp_pairs_differ(const int32_t* __restrict__ to
 
 // Whole warp: are rows a and b equal (same length, same tokens below it)?
 template <bool VEC>
-__device__ bool rows_equal_warp(const int32_t* __restrict__ tokens, int32_t stride,
+__device__ __forceinline__ bool rows_equal_warp(const int32_t* __restrict__ tokens, int32_t stride,
                                 const int32_t* __restrict__ lens, int64_t a, int64_t b,
                                 unsigned* err) {
   const int lane = threadIdx.x & 31;
@@ -195,12 +200,108 @@ __device__ __forceinline__ bool verify_warp(const int32_t* __restrict__ tokens, 
   return self || (need && !differ);
 }
 
+// Second grouping key of row a for the collision list: a multiply-xorshift
+// hash over its length and tokens (structurally unlike FNV-1a, so rows whose
+// fingerprints collide almost never collide here too), mixed with the row's
+// fingerprint.  Rows with equal contents get equal keys, because their
+// fingerprints are equal.  The key only groups rows for the comparison that
+// follows, so exactness does not depend on it.
+template <bool VEC>
+__device__ __forceinline__ uint64_t regroup_key(const uint64_t* __restrict__ fp, const int32_t* __restrict__ tokens,
+                                int32_t stride, const int32_t* __restrict__ lens, int64_t a,
+                                unsigned* err) {
+  constexpr uint64_t kMul = 0x9E3779B97F4A7C15ull, kFin = 0xD6E8FEB86659FD93ull;
+  const int32_t len = clamp_len(lens, a, stride, err);
+  const int32_t* row = tokens + a * (int64_t)stride;
+  uint64_t h = 0x243F6A8885A308D3ull ^ (uint64_t)(uint32_t)len;
+  int32_t t = 0;
+  if (VEC) {
+    const int4* p = reinterpret_cast<const int4*>(row);
+#pragma unroll 1
+    for (; t + 4 <= len; t += 4) {
+      const int4 v = __ldg(p + (t >> 2));
+      h = (h ^ (uint32_t)v.x) * kMul;
+      h ^= h >> 29;
+      h = (h ^ (uint32_t)v.y) * kMul;
+      h ^= h >> 29;
+      h = (h ^ (uint32_t)v.z) * kMul;
+      h ^= h >> 29;
+      h = (h ^ (uint32_t)v.w) * kMul;
+      h ^= h >> 29;
+    }
+  }
+#pragma unroll 1
+  for (; t < len; ++t) {
+    h = (h ^ (uint32_t)__ldg(row + t)) * kMul;
+    h ^= h >> 29;
+  }
+  h ^= __ldg(fp + a) * kFin;
+  h ^= h >> 32;
+  h *= kFin;
+  return h ^ (h >> 29);
+}
+
+// Exact regrouping of the m listed rows (rep == -1: each differs from the
+// smallest row with its fingerprint, so it can only equal other listed
+// rows) in linear work; one block.  The listed rows are grouped by
+// regroup_key in the table keys/idx (any contents; it needs
+// 2^table_log2(m) + 1 slots), each row is compared in full with the
+// smallest listed row of its group and joins it if equal (the smallest row
+// of a group is its own representative: every row equal to it is listed and
+// in its group).  A row that differs from its group's smallest row as well
+// goes to list2; returns their number, the same in every thread.
+template <bool VEC>
+__device__ __forceinline__ uint32_t regroup_block(const uint64_t* __restrict__ fp,
+                                  const int32_t* __restrict__ tokens, int32_t stride,
+                                  const int32_t* __restrict__ lens, int32_t* rep,
+                                  const int32_t* list, uint32_t m, uint64_t* keys, uint32_t* idx,
+                                  int32_t* list2, unsigned* err) {
+  __shared__ uint32_t s_m2;
+  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5, nw = blockDim.x >> 5;
+  const int log2M = table_log2(m);
+  const uint32_t T1 = (1u << log2M) + 1u;
+  for (uint32_t s = tid; s < T1; s += blockDim.x) {
+    keys[s] = kEmpty;
+    idx[s] = kNoRow;
+  }
+  if (tid == 0) s_m2 = 0;
+  __syncthreads();
+  for (uint32_t b = 0; b < m; b += blockDim.x) {
+    const uint32_t c = b + tid;
+    const bool valid = c < m;
+    const int32_t a = valid ? list[c] : 0;
+    const uint64_t k2 = valid ? regroup_key<VEC>(fp, tokens, stride, lens, a, err) : 0ull;
+    insert_row(keys, idx, log2M, valid, k2, (uint32_t)a);
+  }
+  __syncthreads();
+  for (uint32_t b = (uint32_t)w * 32u; b < m; b += (uint32_t)nw * 32u) {
+    const uint32_t c = b + lane;
+    const bool valid = c < m;
+    const int64_t a = valid ? list[c] : 0;
+    int64_t r = a;
+    if (valid) {
+      const uint64_t k2 = regroup_key<VEC>(fp, tokens, stride, lens, a, err);
+      const uint32_t v = idx[find_key(keys, k2, log2M)];
+      if (v != kNoRow) r = v;
+    }
+    const bool merged = verify_warp<VEC>(tokens, stride, lens, valid, a, r, err);
+    if (valid) {
+      if (merged)
+        rep[a] = (int32_t)r;
+      else
+        list2[atomicAdd(&s_m2, 1u)] = (int32_t)a;
+    }
+  }
+  __syncthreads();
+  return s_m2;
+}
+
 // Exact regrouping of the listed rows (rep == -1) by peeling; one block.
 // Listed rows differ from the representative of their fingerprint, so they
 // can only equal each other; the smallest unassigned row of each content
 // becomes its representative.  rep may be in shared or global memory.
 template <bool VEC>
-__device__ void peel_block(const uint64_t* __restrict__ fp, const int32_t* __restrict__ tokens,
+__device__ __forceinline__ void peel_block(const uint64_t* __restrict__ fp, const int32_t* __restrict__ tokens,
                            int32_t stride, const int32_t* __restrict__ lens, int32_t* rep,
                            const int32_t* coll_list, uint32_t m, unsigned* err) {
   __shared__ int32_t s_first;
@@ -270,18 +371,20 @@ __global__ void __launch_bounds__(256) verify_kernel(
   }
 }
 
+// The collision list, after verify: the table is free again (verify was its
+// last reader) and so is uid (the scan writes it next), which holds list2.
 template <bool VEC>
-__global__ void __launch_bounds__(1024) resolve_kernel(const uint64_t* __restrict__ fp,
-                                                       const int32_t* __restrict__ tokens,
-                                                       int32_t stride,
-                                                       const int32_t* __restrict__ lens,
-                                                       int32_t* rep, const int32_t* coll_list,
-                                                       const uint32_t* ctr, unsigned* err) {
+__global__ void __launch_bounds__(kResolveThreads) resolve_kernel(
+    const uint64_t* __restrict__ fp, const int32_t* __restrict__ tokens, int32_t stride,
+    const int32_t* __restrict__ lens, int32_t* rep, const int32_t* coll_list,
+    const uint32_t* ctr, uint64_t* keys, uint32_t* idx, int32_t* list2, unsigned* err) {
   pdl_wait();
   pdl_trigger();
   const uint32_t m = ctr[kCtrColl];
   if (m == 0) return;
-  peel_block<VEC>(fp, tokens, stride, lens, rep, coll_list, m, err);
+  const uint32_t m2 = regroup_block<VEC>(fp, tokens, stride, lens, rep, coll_list, m, keys, idx,
+                                         list2, err);
+  if (m2 > 0) peel_block<VEC>(fp, tokens, stride, lens, rep, list2, m2, err);
 }
 
 // Single-pass exclusive sum-scan of "rep[i] == i" with decoupled look-back;
@@ -427,7 +530,7 @@ constexpr size_t small_smem(int64_t n) {
 }
 
 template <bool VEC>
-__global__ void __launch_bounds__(kSmallThreads) unique_small_kernel(
+__global__ void __launch_bounds__(kSmallThreads, 1) unique_small_kernel(
     const uint64_t* __restrict__ fp, int64_t n, const int32_t* __restrict__ tokens,
     int32_t stride, const int32_t* __restrict__ lens, int32_t* __restrict__ n_unique,
     int32_t* __restrict__ unique_idx, int32_t* __restrict__ inverse, uint32_t* ctr,
@@ -488,7 +591,11 @@ __global__ void __launch_bounds__(kSmallThreads) unique_small_kernel(
   const uint32_t m = *reinterpret_cast<volatile uint32_t*>(ctr + kCtrColl);
   for (uint32_t c = tid; c < m; c += kSmallThreads) rep[coll_list[c]] = -1;
   __syncthreads();
-  if (m) peel_block<VEC>(fp, tokens, stride, lens, rep, coll_list, m, err);
+  if (m) {   // the table and uid are free here: uid holds the rows left for peeling
+    const uint32_t m2 =
+        regroup_block<VEC>(fp, tokens, stride, lens, rep, coll_list, m, keys, idx, uid, err);
+    if (m2) peel_block<VEC>(fp, tokens, stride, lens, rep, uid, m2, err);
+  }
   __syncthreads();
   // exclusive scan of rep[i] == i: contiguous items per thread
   const int64_t per = (n + kSmallThreads - 1) / kSmallThreads;
@@ -599,11 +706,11 @@ hs_status launch_unique_inverse(const uint64_t* fp, const int32_t* tokens, int64
     launch_pdl(verify_kernel<false>, dim3(vgrid), dim3(256), 0, stream, fp, n, keys, idx, L.log2T,
                tokens, stride, lens, rep, coll_list, ctr, err);
   if (vec)
-    launch_pdl(resolve_kernel<true>, dim3(1), dim3(1024), 0, stream, fp, tokens, stride, lens, rep,
-               coll_list, ctr, err);
+    launch_pdl(resolve_kernel<true>, dim3(1), dim3(kResolveThreads), 0, stream, fp, tokens, stride,
+               lens, rep, coll_list, ctr, keys, idx, uid, err);
   else
-    launch_pdl(resolve_kernel<false>, dim3(1), dim3(1024), 0, stream, fp, tokens, stride, lens, rep,
-               coll_list, ctr, err);
+    launch_pdl(resolve_kernel<false>, dim3(1), dim3(kResolveThreads), 0, stream, fp, tokens,
+               stride, lens, rep, coll_list, ctr, keys, idx, uid, err);
   const int64_t tiles = (n + kScanTile - 1) / kScanTile;
   launch_pdl(scan_kernel, dim3((unsigned)tiles), dim3(kScanThreads), 0, stream, rep, n, uid, status,
              ctr, n_unique_dev, err);

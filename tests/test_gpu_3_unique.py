@@ -144,3 +144,17 @@ def test_unique_idx_tail_is_a_valid_map():
     hs.hs_get_device_error()
     n = int(nu.item())
     assert n == 128 and (uidx[n:] == 0).all()
+
+
+@pytest.mark.parametrize("n,distinct", [(4096, 4096), (200_000, 50_000)])
+def test_constant_fingerprints_regroup_in_linear_work(n, distinct):
+    """Every row given the same fingerprint (a caller's weak hash): each row
+    that differs from row 0 is a collision.  The collision list is regrouped
+    by a second key and compared in full — on the one-launch path (n <= 4096)
+    and on the multi-kernel path — and the result is still exact."""
+    rng = np.random.default_rng(n)
+    base = rng.integers(-(1 << 30), 1 << 30, size=(distinct, 6)).astype(np.int32)
+    tok = base[rng.integers(0, distinct, size=n)]
+    same_as_oracle(tok, None, np.zeros(n, np.uint64))
+    lens = rng.integers(0, 7, size=n).astype(np.int32)   # lengths in the key too
+    same_as_oracle(tok, lens, np.full(n, 12345, np.uint64))
