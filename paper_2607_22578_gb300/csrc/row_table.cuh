@@ -56,18 +56,17 @@ __device__ __forceinline__ uint32_t find_key(const uint64_t* keys, uint64_t f, i
   return mask + 1u;
 }
 
-// One warp-round of inserts: lane l offers (f, i) if valid.  Lanes with equal
-// fingerprints are combined: the lowest of them inserts the smallest of their
-// row indices (lanes need not hold rows in ascending order).
+// One warp-round of inserts: lane l offers (f, i) if valid, with rows in
+// ascending lane order.  Lanes with equal fingerprints are combined; the
+// lowest such lane (smallest index) inserts.
 __device__ __forceinline__ void insert_row(uint64_t* keys, uint32_t* idx, int log2T, bool valid,
                                            uint64_t f, uint32_t i) {
   const unsigned act = __ballot_sync(0xffffffffu, valid);
   if (!valid) return;
   const unsigned peers = __match_any_sync(act, f);
-  const uint32_t least = __reduce_min_sync(peers, i);
   if ((int)(__ffs(peers) - 1) != (int)(threadIdx.x & 31)) return;
   const uint32_t s = insert_key(keys, f, log2T);
-  if (*reinterpret_cast<volatile uint32_t*>(idx + s) > least) atomicMin(idx + s, least);
+  if (*reinterpret_cast<volatile uint32_t*>(idx + s) > i) atomicMin(idx + s, i);
 }
 
 }  // namespace table

@@ -266,12 +266,10 @@ __device__ __forceinline__ uint32_t regroup_block(const uint64_t* __restrict__ f
   }
   if (tid == 0) s_m2 = 0;
   __syncthreads();
-  for (uint32_t b = 0; b < m; b += blockDim.x) {
-    const uint32_t c = b + tid;
-    const bool valid = c < m;
-    const int32_t a = valid ? list[c] : 0;
-    const uint64_t k2 = valid ? regroup_key<VEC>(fp, tokens, stride, lens, a, err) : 0ull;
-    insert_row(keys, idx, log2M, valid, k2, (uint32_t)a);
+  for (uint32_t c = tid; c < m; c += blockDim.x) {   // list order is arbitrary: no combining
+    const int32_t a = list[c];
+    const uint32_t s = insert_key(keys, regroup_key<VEC>(fp, tokens, stride, lens, a, err), log2M);
+    atomicMin(idx + s, (uint32_t)a);
   }
   __syncthreads();
   for (uint32_t b = (uint32_t)w * 32u; b < m; b += (uint32_t)nw * 32u) {
