@@ -120,9 +120,12 @@ hs_status hs_fingerprint(const int32_t* tokens, int64_t n_rows, int32_t row_stri
  * one seed); different rows may share a fingerprint (a collision): they are
  * told apart by a full row comparison, never merged.  Cost is linear in the
  * row bytes of rows that have an equal-fingerprint predecessor, plus one hash
- * table insert and lookup per row; rows whose fingerprint equals an earlier
- * row's but whose contents differ (a collision) are regrouped by an extra
- * pass that is quadratic in the number of such rows.
+ * table insert and lookup per row.  Rows whose fingerprint equals an earlier
+ * row's but whose contents differ (a collision) are regrouped by a second
+ * hash of their contents and compared once more, in one thread block: linear
+ * in their row bytes, so even a constant fp is exact at linear cost (slower
+ * than distinct fingerprints, which spread the work over the whole GPU).
+ * Only rows that collide in both hashes are compared pairwise.
  *
  * fp              device uint64 [n_rows], 8-byte aligned.
  * tokens, n_rows, row_stride, lens   as for hs_fingerprint;
