@@ -129,3 +129,24 @@ def test_bad_k_is_rejected():
     with pytest.raises(ValueError):
         oracle.topk(Q, C, 0)
 
+
+
+def test_corpus_permutation_maps_ids():
+    """Reordering the corpus rows maps each returned id through the
+    permutation and leaves the scores unchanged (distinct scores, so no
+    tie-break depends on the order)."""
+    rng = np.random.default_rng(11)
+    Q = rng.integers(-8, 9, size=(5, 16)).astype(np.float32)
+    C = rng.integers(-8, 9, size=(300, 16)).astype(np.float32)
+    # every score distinct: column 0 takes 300 distinct bf16-exact values
+    # (8 significant bits) spaced 1024 or more apart, beyond what the other
+    # columns can add (|sum| <= 15 * 64 = 960), and q[0] >= 1
+    k = np.arange(300)
+    C[:, 0] = (128 + k % 128) * 2.0 ** (10 + k // 128)
+    Q[:, 0] = rng.integers(1, 9, size=5)
+    q_bits, c_bits = to_bf16_bits(Q), to_bf16_bits(C)
+    perm = rng.permutation(300)
+    s1, i1 = oracle.topk(q_bits, c_bits, 12)
+    s2, i2 = oracle.topk(q_bits, c_bits[perm], 12)
+    assert (s1 == s2).all()
+    assert (perm[i2] == i1).all()

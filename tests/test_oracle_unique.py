@@ -139,3 +139,26 @@ def test_generator_ground_truth_dedup_heavy_scaled():
 def test_out_of_range_len_is_rejected():
     with pytest.raises(ValueError):
         oracle.unique_inverse(np.zeros((2, 3), np.int32), np.array([4, 0], np.int32))
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_partition_is_invariant_under_row_permutation(seed):
+    """Reordering the rows reorders the groups but never changes which rows
+    share a group (only the choice of representative follows the order)."""
+    rng = np.random.default_rng(700 + seed)
+    n, stride = 3000, 7
+    base = rng.integers(0, 3, size=(400, stride)).astype(np.int32)
+    pick = rng.integers(0, 400, size=n)
+    tokens = base[pick]
+    lens = rng.integers(4, stride + 1, size=400).astype(np.int32)[pick]
+    perm = rng.permutation(n)
+    _, inv = oracle.unique_inverse(tokens, lens)
+    _, inv_p = oracle.unique_inverse(tokens[perm], lens[perm])
+    # rows i and j share a group iff their permuted images share one
+    pairs = rng.integers(0, n, size=(20000, 2))
+    where = np.empty(n, dtype=np.int64)
+    where[perm] = np.arange(n)
+    same = inv[pairs[:, 0]] == inv[pairs[:, 1]]
+    same_p = inv_p[where[pairs[:, 0]]] == inv_p[where[pairs[:, 1]]]
+    assert (same == same_p).all()
+    assert inv.max() == inv_p.max()
