@@ -76,3 +76,17 @@ def test_oracle_is_not_imported_by_the_library():
                 src = open(os.path.join(dirpath, f)).read()
                 assert "import oracle" not in src and "from oracle" not in src
                 assert "hs_oracle" not in src and "liboracle" not in src
+
+
+def test_binding_constants_match_header():
+    """The status codes and the #define limits the binding restates are the
+    header's values."""
+    import paper_2607_22578_gb300._lib as lib
+    text = open(HEADER).read()
+    for name, val in re.findall(r"#define (HS_[A-Z0-9_]+) (0x[0-9a-fA-F]+|\d+)", text):
+        assert getattr(lib, name) == int(val, 0), name
+    enum = dict(re.findall(r"\b(HS_(?:OK|ERR_[A-Z_]+)) = (\d+)", text))
+    assert enum["HS_OK"] == "0"
+    for name, val in enum.items():
+        if name != "HS_OK":
+            assert getattr(lib, name) == int(val), name
