@@ -84,3 +84,21 @@ def test_bad_inverse():
         oracle.segment_sum(np.ones(3), np.array([0, 3, 1]), 3)
     with pytest.raises(IndexError):
         oracle.segment_sum(np.ones(2), np.array([-1, 0]), 3)
+
+
+def test_row_order_does_not_change_integer_sums():
+    """Permuting the rows (with their group ordinals) leaves every group's
+    sum unchanged; with integer contributions below 2^53 every partial sum
+    is exact, so the sums must agree bit for bit."""
+    rng = np.random.default_rng(31)
+    n, groups = 50_000, 700
+    phi = rng.integers(-(1 << 20), 1 << 20, size=n).astype(np.float64)
+    inv = rng.integers(0, groups, size=n).astype(np.int32)
+    perm = rng.permutation(n)
+    a = oracle.segment_sum(phi, inv, groups)
+    b = oracle.segment_sum(phi[perm], inv[perm], groups)
+    assert (a == b).all()
+    # and a relabelling of the groups permutes the sums the same way
+    relabel = rng.permutation(groups).astype(np.int32)
+    c = oracle.segment_sum(phi, relabel[inv], groups)
+    assert (c[relabel] == a).all()
