@@ -44,6 +44,7 @@ constexpr size_t kSsSmem = (size_t)(kSsWarps * kSsSlots + kSsCtaSlots) *
                            (size_t)kSsWarps * kSsSlots * sizeof(int32_t);
 static_assert(kSsSlots >= 2 * kSsTile && kSsCtaSlots >= 2 * kSsCtaRows,
               "tables at least twice the rows they hold");
+static_assert(kSsSmem <= 232448, "the warp and CTA tables fit one CTA's shared memory");
 
 __device__ __forceinline__ uint32_t ss_slot(int32_t g, int log2_slots) {
   return ((uint32_t)g * 0x9E3779B1u) >> (32 - log2_slots);

@@ -526,6 +526,8 @@ constexpr size_t small_smem(int64_t n) {
   const size_t T1 = (size_t(1) << table_log2(n)) + 1;
   return T1 * 8 + T1 * 4 + (size_t)n * 8 + 16;
 }
+static_assert(small_smem(kSmallRows) + kSmallThreads / 32 * 4 + 16 <= 232448,
+              "one-launch path: the table, rep and uid fit one CTA's shared memory");
 
 template <bool VEC>
 __global__ void __launch_bounds__(kSmallThreads, 1) unique_small_kernel(
