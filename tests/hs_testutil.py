@@ -62,3 +62,40 @@ def check_topk(gs, gi, os_, oi, exact_g, N, k, tol=TOL, strict=STRICT):
         assert set(must) <= set(gi.tolist()), "a clearly-better oracle id is missing"
         assert (exact_g >= s_k - tol).all(), "a returned id is clearly worse than the k-th"
     return err
+
+
+_TOPK_MEMO: dict = {}
+
+
+def oracle_topk_memo(tag: str, Q: np.ndarray, C: np.ndarray, k: int):
+    """oracle.topk(Q, C, k), remembered for the rest of the test session.
+
+    The full-size parity tests of several modules need the oracle's top-k of
+    the same merged queries against the same corpus (minutes of fp64 work
+    on the host); the key is the caller's name for the corpus, the corpus
+    shape, k and a digest of the query rows."""
+    import hashlib
+
+    import oracle
+    key = (tag, C.shape, int(k), hashlib.sha1(np.ascontiguousarray(Q).tobytes()).hexdigest())
+    if key not in _TOPK_MEMO:
+        _TOPK_MEMO[key] = oracle.topk(Q, C, k)
+    return _TOPK_MEMO[key]
+
+
+def check_rows(Q, C, k, gs, gi, rows, tag=None):
+    """check_topk on each listed query row of a GPU result (gs, gi indexed
+    like Q); the oracle's first k + 1 entries come from oracle.topk (through
+    oracle_topk_memo when a corpus tag is given).  Returns the max score
+    error."""
+    import oracle
+    rows = np.asarray(rows, dtype=np.int64)
+    N = C.shape[0]
+    kk = min(k + 1, N)
+    Qs = np.ascontiguousarray(Q[rows])
+    os_, oi = oracle_topk_memo(tag, Qs, C, kk) if tag else oracle.topk(Qs, C, kk)
+    exact = oracle.pair_scores(Q, C, np.repeat(rows, k), gi[rows].reshape(-1)).reshape(-1, k)
+    worst = 0.0
+    for r, q in enumerate(rows):
+        worst = max(worst, check_topk(gs[q], gi[q], os_[r], oi[r], exact[r], N, k))
+    return worst

@@ -11,7 +11,7 @@ import torch
 import oracle
 import paper_2607_22578_gb300 as hs
 import synth
-from hs_testutil import to_dev
+from hs_testutil import check_rows, to_dev
 
 pytestmark = pytest.mark.gpu
 
@@ -35,7 +35,8 @@ def miss_flags(stage, Q):
 def test_hits_follow_the_reuse_model_and_results_match(B):
     """B = 40 takes the fused query path; B = 700 the separate calls."""
     pool = synth.unit_rows(300, 256, 1)
-    corpus = to_dev(synth.unit_rows(20000, 256, 2))
+    corpus_h = synth.unit_rows(20000, 256, 2)
+    corpus = to_dev(corpus_h)
     batches = zipf_batches(pool, 6, B, seed=B)
     cached = hs.EmbedRetrieveStage(corpus, 10, max_queries=B, cache_capacity=4096)
     plain = hs.EmbedRetrieveStage(corpus, 10, max_queries=B)
@@ -48,6 +49,9 @@ def test_hits_follow_the_reuse_model_and_results_match(B):
         hs.hs_get_device_error()
         assert torch.equal(s.cpu(), s2.cpu()) and torch.equal(i.cpu(), i2.cpu())
         uidx, _ = oracle.unique_inverse(qb.view(np.int32))
+        # hit rows (from the cache) and miss rows (retrieved now) alike
+        # against the oracle
+        check_rows(qb, corpus_h, 10, s.cpu().numpy(), i.cpu().numpy(), uidx)
         uniq_rows.append((qb[uidx], ~flags))
     model = oracle.cache_reuse([u for u, _ in uniq_rows])
     for (_, hit), want in zip(uniq_rows, model):
@@ -59,7 +63,8 @@ def test_hits_follow_the_reuse_model_and_results_match(B):
 
 def test_small_cache_evicts_but_stays_correct():
     pool = synth.unit_rows(400, 128, 3)
-    corpus = to_dev(synth.unit_rows(5000, 128, 4))
+    corpus_h = synth.unit_rows(5000, 128, 4)
+    corpus = to_dev(corpus_h)
     batches = zipf_batches(pool, 8, 200, seed=5)
     cached = hs.EmbedRetrieveStage(corpus, 8, max_queries=200, cache_capacity=16)
     plain = hs.EmbedRetrieveStage(corpus, 8, max_queries=200)
@@ -69,6 +74,8 @@ def test_small_cache_evicts_but_stays_correct():
         s2, i2, _ = plain.retrieve(to_dev(qb))
         hs.hs_get_device_error()
         assert torch.equal(s.cpu(), s2.cpu()) and torch.equal(i.cpu(), i2.cpu())
+        check_rows(qb, corpus_h, 8, s.cpu().numpy(), i.cpu().numpy(),
+                   oracle.unique_inverse(qb.view(np.int32))[0])
         total_unique += int(nu.item())
     hits, misses = cached.cache_stats()
     assert hits + misses == total_unique
@@ -81,12 +88,14 @@ def test_fingerprint_collisions_never_share_results():
     """All queries given the same key: every distinct vector is its own
     entry (up to the set's 8 ways), and each lookup returns its own top-k."""
     d, k = 64, 5
-    corpus = to_dev(synth.unit_rows(2000, d, 6))
+    corpus_h = synth.unit_rows(2000, d, 6)
+    corpus = to_dev(corpus_h)
     q = synth.unit_rows(6, d, 7)
     cache = hs.ResultCache(64, d, k)
     fp = torch.zeros(6, dtype=torch.int64, device="cuda")
     qd = to_dev(q)
     want_s, want_i = hs.hs_retrieve_topk(qd, corpus, k)
+    check_rows(q, corpus_h, k, want_s.cpu().numpy(), want_i.cpu().numpy(), np.arange(6))
     for _ in range(2):
         out, miss = hs.hs_cache_lookup(cache, qd, fp)
         ms, mi = hs.hs_retrieve_topk_n(miss[2], miss[1], corpus, k)
@@ -110,14 +119,18 @@ def test_two_streams_share_a_cache_without_torn_results():
     so inserts on one stream evict entries that lookups on the other may be
     reading.  Every row, hit or miss, must be exactly its own query's top-k."""
     d, k, pool_n, B = 256, 10, 48, 12
-    corpus = to_dev(synth.unit_rows(400000, d, 21))
-    pd = to_dev(synth.unit_rows(pool_n, d, 22))
+    corpus_h = synth.unit_rows(400000, d, 21)
+    pool_h = synth.unit_rows(pool_n, d, 22)
+    corpus = to_dev(corpus_h)
+    pd = to_dev(pool_h)
     fp_all = hs.hs_fingerprint(pd.view(torch.int32))
     want_s = torch.empty((pool_n, k), dtype=torch.float32, device="cuda")
     want_i = torch.empty((pool_n, k), dtype=torch.int32, device="cuda")
     for c0 in range(0, pool_n, B):                   # the kernel the misses take (<= 16 rows)
         s, i = hs.hs_retrieve_topk(pd[c0:c0 + B], corpus, k)
         want_s[c0:c0 + B], want_i[c0:c0 + B] = s, i
+    check_rows(pool_h, corpus_h, k, want_s.cpu().numpy(), want_i.cpu().numpy(),
+               np.arange(pool_n))
     rng = np.random.default_rng(23)
     sels = torch.from_numpy(np.stack([rng.choice(pool_n, B, replace=False)
                                       for _ in range(120)])).to("cuda")

@@ -10,7 +10,7 @@ import torch
 import oracle
 import paper_2607_22578_gb300 as hs
 import synth
-from hs_testutil import check_topk, to_dev
+from hs_testutil import check_rows, check_topk, to_dev
 from synth import configs
 
 pytestmark = pytest.mark.gpu
@@ -34,12 +34,8 @@ def test_fused_query_path_batch_sweep_sizes():
         assert int(nu.item()) == len(ou)
         s, i = s.cpu().numpy(), i.cpu().numpy()
         assert (s == s[ou][oi]).all() and (i == i[ou][oi]).all()   # merged rows share results
-        sample = ou[:: max(1, len(ou) // 4)][:4]
-        k = configs.BATCH_SWEEP["k"]
-        os_, oid = oracle.topk(q[sample], C, k + 1)
-        for r, qq in enumerate(sample):
-            exact = oracle.pair_scores(q, C, np.full(k, qq), i[qq])
-            check_topk(s[qq], i[qq], os_[r], oid[r], exact, C.shape[0], k)
+        # every merged query of the batch against the oracle
+        check_rows(q, C, configs.BATCH_SWEEP["k"], s, i, ou)
 
 
 def test_cache_on_rag_mix_stream(rag):
@@ -50,14 +46,29 @@ def test_cache_on_rag_mix_stream(rag):
     p /= p.sum()
     cached = hs.EmbedRetrieveStage(corpus, w["k"], max_queries=2048, cache_capacity=65536)
     plain = hs.EmbedRetrieveStage(corpus, w["k"], max_queries=2048)
+    checked = 0
     for b in range(3):
-        qb = to_dev(pool[rng.choice(3000, 2048, p=p)])
-        s, i, _ = cached.retrieve(qb)
+        qh = pool[rng.choice(3000, 2048, p=p)]
+        qb = to_dev(qh)
+        s, i, nu = cached.retrieve(qb)
+        n_u = int(nu.item())
+        n_miss = int(cached.miss[1].item())
+        hit = np.ones(n_u, bool)
+        hit[cached.miss[0][:n_miss].cpu().numpy()] = False
         s2, i2, _ = plain.retrieve(qb)
         hs.hs_get_device_error()
         assert torch.equal(s.cpu(), s2.cpu()) and torch.equal(i.cpu(), i2.cpu())
+        # rows served from the cache against the oracle (a seeded sample)
+        uidx, _ = oracle.unique_inverse(qh.view(np.int32))
+        hit_rows = uidx[hit]
+        if len(hit_rows):
+            pick = np.random.default_rng(b).choice(len(hit_rows), min(96, len(hit_rows)),
+                                                   replace=False)
+            check_rows(qh, w["corpus"], w["k"], s.cpu().numpy(), i.cpu().numpy(),
+                       hit_rows[pick])
+            checked += len(pick)
     hits, misses = cached.cache_stats()
-    assert hits > 0 and misses > 0
+    assert hits > 0 and misses > 0 and checked > 0
 
 
 def test_rerank_full_size_sampled(rag):

@@ -5,8 +5,11 @@ budget, or request paths that must not stall in an allocator).  Its scratch
 is a fixed array inside the library, so it takes no workspace.
 
 Called through the C ABI; each of two calls in a row must give exactly the
-same outputs as hs_unique_inverse on the same input (unique sets and inverse
-maps are compared bit-exactly, as everywhere in these tests).  This file is
+same outputs as hs_unique_inverse on the same input and as the oracle's
+unique/inverse (unique sets and inverse maps are compared bit-exactly, as
+everywhere in these tests).  Both of the variant's paths are covered: the
+one-launch path of at most 4096 rows (which uses the scratch's counters and
+collision list) and the multi-kernel path up to the 65,536-row limit.  This file is
 collected last, so a run that stops at its first failure has already run every
 other test."""
 import ctypes
@@ -15,6 +18,7 @@ import numpy as np
 import pytest
 import torch
 
+import oracle
 import paper_2607_22578_gb300 as hs
 from hs_testutil import to_dev
 from synth import configs
@@ -46,6 +50,25 @@ def _noalloc(lib, fp, tokens, lens):
     return nu, uidx, inv
 
 
+def _check(lib, tokens_np, lens_np, mask=None):
+    t = to_dev(tokens_np)
+    L = None if lens_np is None else to_dev(lens_np)
+    fp = hs.hs_fingerprint(t, L)
+    if mask is not None:                     # forced fingerprint collisions
+        fp = fp & mask
+    nu_a, uidx_a, inv_a = _noalloc(lib, fp, t, L)
+    nu_b, uidx_b, inv_b = hs.hs_unique_inverse(fp, t, L)
+    hs.hs_get_device_error()
+    n = int(nu_b.item())
+    assert int(nu_a.item()) == n
+    assert torch.equal(uidx_a[:n], uidx_b[:n])
+    assert torch.equal(inv_a, inv_b)
+    ou, oi = oracle.unique_inverse(tokens_np, lens_np)
+    assert n == len(ou)
+    assert (uidx_a[:n].cpu().numpy() == ou).all()
+    assert (inv_a.cpu().numpy() == oi).all()
+
+
 def test_noalloc_matches_workspace_entry_point_twice_in_a_row():
     lib = _lib()
     full = configs.build_retrieval_mix(configs.RAG_MIX, corpus=False)
@@ -55,16 +78,21 @@ def test_noalloc_matches_workspace_entry_point_twice_in_a_row():
     cases = [(full["tokens"], None), (heavy["tokens"][:50000], heavy["lens"][:50000])]
     assert full["tokens"].shape[0] == LIMIT
     for tokens_np, lens_np in cases:
-        t = to_dev(tokens_np)
-        L = None if lens_np is None else to_dev(lens_np)
-        fp = hs.hs_fingerprint(t, L)
-        nu_a, uidx_a, inv_a = _noalloc(lib, fp, t, L)
-        nu_b, uidx_b, inv_b = hs.hs_unique_inverse(fp, t, L)
-        hs.hs_get_device_error()
-        n = int(nu_b.item())
-        assert int(nu_a.item()) == n
-        assert torch.equal(uidx_a[:n], uidx_b[:n])
-        assert torch.equal(inv_a, inv_b)
+        _check(lib, tokens_np, lens_np)
+
+
+def test_noalloc_one_launch_path_with_collisions_twice_in_a_row():
+    """At most 4096 rows take the one-launch path; keeping 4 bits of each
+    fingerprint forces collisions, so the collision list in the scratch is
+    used and must be cleared between the two calls."""
+    lib = _lib()
+    heavy = configs.build_dedup_heavy(scale=0.01)
+    tok, ln = heavy["tokens"][:4096], heavy["lens"][:4096]
+    for mask in (0xF, 0xF, None):
+        _check(lib, tok, ln, mask)
+    tiny = configs.build_retrieval_mix(configs.TINY, corpus=False)["tokens"]
+    _check(lib, tiny, None, 0x1)
+    _check(lib, tiny[:37], None)
 
 
 def test_noalloc_rejects_rows_beyond_its_limit():
