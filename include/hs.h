@@ -152,8 +152,8 @@ hs_status hs_unique_inverse(const uint64_t* fp, const int32_t* tokens, int64_t n
  * that are given a fixed memory budget and no allocator, and latency-critical
  * request paths where an allocator call is an unbounded stall.  This entry
  * point takes no workspace: its scratch is a fixed array inside the
- * library's device memory (about 2.5 MB, present on every GPU that loads the
- * library until the process exits), so it calls no allocator at all.
+ * library's device memory (2,360,320 bytes, about 2.36 MB, present on every GPU
+ * that loads the library until the process exits), so it calls no allocator at all.
  *
  * Same arguments, outputs and error behaviour as hs_unique_inverse, except:
  *   - n_rows must not exceed 65536 (larger n_rows returns
@@ -471,6 +471,51 @@ hs_status hs_get_device_error(hs_stream_t stream);
  * part in the method; callers use it to count device work per call.
  */
 uint64_t hs_launch_count(void);
+
+/*
+ * hs_debug_scan_wait — test hook of the bounded device waits (failure
+ * detection); takes no part in the method.
+ *
+ * Every device-side wait of the library gives up after a limit (2 s by
+ * default) and then sets HS_ERR_TIMEOUT in the device error word instead of
+ * spinning on.  hs_unique_inverse's scan waits for the status each earlier
+ * tile of 16,384 rows publishes (decoupled look-back).  This hook, for tests
+ * only, lowers that wait's limit and can stop one tile from publishing, so
+ * that a test can make the wait run out and check that the call returns,
+ * that hs_get_device_error reports HS_ERR_TIMEOUT, and that the next call
+ * is correct again.  While a tile is withheld, the outputs of
+ * hs_unique_inverse calls with more than withhold_tile + 1 tiles are
+ * unspecified (every write stays inside the outputs and the workspace).
+ *
+ * limit_ns       wait limit in ns, 1 <= limit_ns <= 2e9; 0 restores 2 s.
+ * withhold_tile  index of the scan tile that does not publish; -1: none.
+ * Settings are process-wide and take effect at the next launch.
+ * Returns HS_ERR_INVALID_ARG for a limit above 2 s or withhold_tile < -1.
+ */
+hs_status hs_debug_scan_wait(uint64_t limit_ns, int64_t withhold_tile);
+
+/*
+ * hs_debug_stream_rows — diagnostics: stream the rows' valid prefixes with
+ * no hashing, to measure what the row layout itself costs to read; takes no
+ * part in the method.
+ *
+ * Reads tokens[i, 0:len_i] of every row (the bytes hs_fingerprint hashes)
+ * with access pattern `pattern`, folds them into *checksum_dev (xor; the
+ * caller zeroes it first), and enqueues one kernel on num_SMs *
+ * blocks_per_sm blocks of 256 threads:
+ *   0  a warp per row, 16 bytes per lane (coalesced 512-byte reads);
+ *   1  a lane per row, 32-byte loads (hs_fingerprint's chunk pattern);
+ *   2  a warp per row over the whole padded row (row_stride tokens).
+ * tokens        device int32 [n_rows, row_stride], 32-byte aligned,
+ *               row_stride % 8 == 0.
+ * lens          device int32 [n_rows] or NULL; lengths are clamped to
+ *               [0, row_stride] (no error is recorded).
+ * checksum_dev  device uint32 scalar.
+ * blocks_per_sm 1 ... 8.
+ */
+hs_status hs_debug_stream_rows(const int32_t* tokens, int64_t n_rows, int32_t row_stride,
+                               const int32_t* lens, int32_t pattern, uint32_t* checksum_dev,
+                               int32_t blocks_per_sm, hs_stream_t stream);
 
 #ifdef __cplusplus
 }

@@ -97,6 +97,10 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
             lib.hs_get_device_error.argtypes = [P]
             lib.hs_get_device_error.restype = st
             lib.hs_launch_count.restype = ctypes.c_uint64
+            lib.hs_debug_scan_wait.argtypes = [u64, i64]
+            lib.hs_debug_scan_wait.restype = st
+            lib.hs_debug_stream_rows.argtypes = [P, i64, i32, P, i32, P, i32, P]
+            lib.hs_debug_stream_rows.restype = st
             _lib = lib
     return _lib
 
@@ -490,3 +494,23 @@ def hs_launch_count() -> int:
 def hs_get_device_error(stream=None) -> None:
     """Synchronise the stream; raise HsError if a kernel reported a problem."""
     _check(load().hs_get_device_error(_stream(stream)))
+
+
+def hs_debug_scan_wait(limit_ns: int = 0, withhold_tile: int = -1) -> None:
+    """Test hook of hs_unique_inverse's bounded look-back wait (see hs.h);
+    hs_debug_scan_wait() restores the defaults."""
+    _check(load().hs_debug_scan_wait(int(limit_ns), int(withhold_tile)))
+
+
+def hs_debug_stream_rows(tokens: torch.Tensor, lens: torch.Tensor | None = None, pattern: int = 0,
+                         checksum: torch.Tensor | None = None, blocks_per_sm: int = 4,
+                         stream=None) -> torch.Tensor:
+    """Read the rows' valid prefixes with one access pattern (diagnostics,
+    see hs.h); returns the xor checksum tensor it folded them into."""
+    n, stride = tokens.shape
+    if checksum is None:
+        checksum = torch.zeros(1, dtype=torch.int32, device=tokens.device)
+    _check(load().hs_debug_stream_rows(tokens.data_ptr(), n, stride,
+                                        None if lens is None else lens.data_ptr(), int(pattern),
+                                        checksum.data_ptr(), int(blocks_per_sm), _stream(stream)))
+    return checksum

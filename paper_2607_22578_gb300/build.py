@@ -18,7 +18,7 @@ BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libhs.so")
 SOURCES = ["api.cu", "fingerprint.cu", "unique.cu", "scatter.cu", "retrieve.cu",
            "query_merge.cu", "segment_sum.cu", "rerank.cu",
-           "result_cache.cu"]
+           "result_cache.cu", "diag.cu"]
 HEADERS = [os.path.join(CSRC, h) for h in ("hs_internal.cuh", "fnv.cuh", "row_table.cuh")] + \
     [os.path.join(ROOT, "include", "hs.h")]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]

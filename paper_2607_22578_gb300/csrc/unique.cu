@@ -386,9 +386,12 @@ __global__ void __launch_bounds__(kResolveThreads) resolve_kernel(
 }
 
 // Single-pass exclusive sum-scan of "rep[i] == i" with decoupled look-back;
-// the last tile writes the total (the group count).
+// the last tile writes the total (the group count).  A predecessor's status
+// is awaited for at most limit_ns of %globaltimer; then the wait gives up,
+// sets kErrTimeout and counts the predecessor as a zero prefix (the call's
+// outputs are then unspecified, but every write stays in bounds).
 __device__ __forceinline__ uint64_t wait_status(const volatile unsigned long long* p,
-                                                unsigned* err) {
+                                                unsigned* err, uint64_t limit_ns) {
   unsigned long long s = *p;
   if (s >> 32) return s;
   const uint64_t t0 = globaltimer_ns();
@@ -397,7 +400,7 @@ __device__ __forceinline__ uint64_t wait_status(const volatile unsigned long lon
     if (s >> 32) return s;
     if ((it & 31u) == 0) {
       __nanosleep(64);
-      if (globaltimer_ns() - t0 > kWaitLimitNs) {
+      if (globaltimer_ns() - t0 > limit_ns) {
         set_error(err, kErrTimeout);
         return 2ull << 32;  // give up: treat as a zero prefix
       }
@@ -409,7 +412,8 @@ __global__ void __launch_bounds__(kScanThreads) scan_kernel(const int32_t* __res
                                                             int64_t n, int32_t* __restrict__ uid,
                                                             unsigned long long* status,
                                                             uint32_t* ctr, int32_t* total_out,
-                                                            unsigned* err) {
+                                                            unsigned* err, uint64_t limit_ns,
+                                                            int64_t withhold_tile) {
   pdl_wait();
   pdl_trigger();
   __shared__ uint32_t s_tile;
@@ -459,10 +463,13 @@ __global__ void __launch_bounds__(kScanThreads) scan_kernel(const int32_t* __res
       const int32_t tile_total = iv;
       volatile unsigned long long* st = status;
       int32_t prefix = 0;
+      // A withheld tile (test hook, -1 in normal use) never publishes, so
+      // its successors' waits run out.
+      const bool publish = (int64_t)tile != withhold_tile;
       if (tile == 0) {
-        st[0] = (2ull << 32) | (uint32_t)tile_total;
+        if (publish) st[0] = (2ull << 32) | (uint32_t)tile_total;
       } else {
-        st[tile] = (1ull << 32) | (uint32_t)tile_total;
+        if (publish) st[tile] = (1ull << 32) | (uint32_t)tile_total;
         bool done = false;
         for (int64_t j0 = (int64_t)tile - 1; j0 >= 0 && !done; j0 -= kLookBatch) {
           unsigned long long sv[kLookBatch];
@@ -472,12 +479,12 @@ __global__ void __launch_bounds__(kScanThreads) scan_kernel(const int32_t* __res
           for (int b = 0; b < kLookBatch; ++b) {
             if (done) break;
             unsigned long long sb = sv[b];
-            if ((sb >> 32) == 0) sb = wait_status(st + (j0 - b), err);
+            if ((sb >> 32) == 0) sb = wait_status(st + (j0 - b), err, limit_ns);
             if (j0 - b >= 0) prefix += (int32_t)(uint32_t)sb;
             if ((sb >> 32) == 2ull) done = true;
           }
         }
-        st[tile] = (2ull << 32) | (uint32_t)(prefix + tile_total);
+        if (publish) st[tile] = (2ull << 32) | (uint32_t)(prefix + tile_total);
       }
       s_prefix = prefix;
       const int64_t tiles = (n + kScanTile - 1) / kScanTile;
@@ -630,6 +637,11 @@ __global__ void __launch_bounds__(kSmallThreads, 1) unique_small_kernel(
   if (tid == 0) *n_unique = total;
 }
 
+// Test hook of the look-back's bounded wait (hs_debug_scan_wait): the wait
+// limit and a tile that does not publish its status (-1: none).
+std::atomic<uint64_t> g_scan_wait_limit_ns{kWaitLimitNs};
+std::atomic<int64_t> g_scan_withhold_tile{-1};
+
 unsigned grid_for(int64_t items, int per_block, int max_blocks) {
   int64_t b = (items + per_block - 1) / per_block;
   if (b < 1) b = 1;
@@ -713,7 +725,7 @@ hs_status launch_unique_inverse(const uint64_t* fp, const int32_t* tokens, int64
                stride, lens, rep, coll_list, ctr, keys, idx, uid, err);
   const int64_t tiles = (n + kScanTile - 1) / kScanTile;
   launch_pdl(scan_kernel, dim3((unsigned)tiles), dim3(kScanThreads), 0, stream, rep, n, uid, status,
-             ctr, n_unique_dev, err);
+             ctr, n_unique_dev, err, g_scan_wait_limit_ns.load(), g_scan_withhold_tile.load());
   launch_pdl(finalize_kernel, dim3(grid_for(n, 256, sms * 8)), dim3(256), 0, stream, rep, uid, n,
              n_unique_dev, unique_idx, inverse);
   count_launches(5);  // insert, verify, resolve, scan, finalize
@@ -730,12 +742,13 @@ hs_status launch_unique_inverse(const uint64_t* fp, const int32_t* tokens, int64
 // latency-critical request paths where an allocator call (or a pool that has
 // to grow) is an unbounded stall.  hs_unique_inverse_noalloc serves them with
 // a scratch area that is part of the library's own module memory: a
-// file-scope device array sized for kNoAllocMaxRows rows (about 2.5 MB),
+// file-scope device array sized for kNoAllocMaxRows rows (2,360,320 bytes),
 // which every GPU that loads the library holds until the process exits.
 namespace hs {
 namespace {
 constexpr int64_t kNoAllocMaxRows = 65536;
 constexpr size_t kNoAllocBytes = layout(kNoAllocMaxRows).total;
+static_assert(kNoAllocBytes == 2360320, "the scratch size stated in hs.h");
 static __device__ __align__(256) unsigned char g_noalloc_ws[kNoAllocBytes];
 constexpr int kNoAllocDevices = 64;
 void* g_noalloc_addr[kNoAllocDevices] = {};
@@ -761,6 +774,18 @@ hs_status noalloc_scratch(void** out) {
 }
 }  // namespace
 }  // namespace hs
+
+extern "C" hs_status hs_debug_scan_wait(uint64_t limit_ns, int64_t withhold_tile) {
+  using namespace hs;
+  clear_last_error();
+  if (limit_ns > kWaitLimitNs)
+    return fail(HS_ERR_INVALID_ARG, "wait limit above the default of %llu ns",
+                (unsigned long long)kWaitLimitNs);
+  if (withhold_tile < -1) return fail(HS_ERR_INVALID_ARG, "withhold_tile < -1");
+  g_scan_wait_limit_ns.store(limit_ns == 0 ? kWaitLimitNs : limit_ns);
+  g_scan_withhold_tile.store(withhold_tile);
+  return HS_OK;
+}
 
 extern "C" hs_status hs_unique_inverse_noalloc(const uint64_t* fp, const int32_t* tokens,
                                                int64_t n_rows, int32_t row_stride,

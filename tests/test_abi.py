@@ -58,6 +58,10 @@ def test_host_only_calls_without_gpu():
     rc = lib.hs_retrieve_topk_fanout(None, 4, None, None, 4, None, 10, 64, 3, None, None, None,
                                      0, None)
     assert rc == _lib.HS_ERR_INVALID_ARG and b"inverse" in lib.hs_last_error()
+    # the wait-limit test hook never allows a wait longer than the default
+    assert lib.hs_debug_scan_wait(3_000_000_000, -1) == _lib.HS_ERR_INVALID_ARG
+    assert lib.hs_debug_scan_wait(0, -2) == _lib.HS_ERR_INVALID_ARG
+    assert lib.hs_debug_scan_wait(0, -1) == _lib.HS_OK
 
 
 def test_binding_names_match_header():

@@ -93,3 +93,19 @@ def test_warmup_floor():
     r = subprocess.run([sys.executable, os.path.join(bench.ROOT, "bench.py"), "--warmup", "1"],
                        capture_output=True, text=True)
     assert r.returncode != 0 and "warmup" in r.stderr
+
+
+def test_oracle_baseline_is_measured_on_a_bounded_sample():
+    """The CPU baseline and the reference arm time the oracle on a sample of
+    the step and divide the merged queries they processed by the time they
+    took (no extrapolation)."""
+    from synth import configs
+    w = configs.build_retrieval_mix(configs.TINY)
+    r = bench.oracle_step(w, 5, 2)
+    assert r["merged"] == 5 and r["merged_total"] == 24
+    assert r["chunk_rows"] == round(256 * 5 / 24) and r["step_s"] > 0
+    m = bench.oracle_measured(w, 0.2, 2, steps=2)
+    assert m["steps"] == 2 and 2 <= m["S"] <= 24
+    assert abs(m["value"] - m["S"] / (m["ms_per_step"] / 1e3)) < 1e-6 * m["value"]
+    assert "measured" in bench.oracle_sample_desc(m)
+    assert bench.cpu_model()

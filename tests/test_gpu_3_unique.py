@@ -158,3 +158,35 @@ def test_constant_fingerprints_regroup_in_linear_work(n, distinct):
     same_as_oracle(tok, None, np.zeros(n, np.uint64))
     lens = rng.integers(0, 7, size=n).astype(np.int32)   # lengths in the key too
     same_as_oracle(tok, lens, np.full(n, 12345, np.uint64))
+
+
+def test_lookback_wait_runs_out_and_reports_timeout():
+    """Failure detection without a fault: the scan's look-back wait gets a
+    1 ms limit and tile 1 withholds its status, so the later tiles wait for
+    a status nobody publishes.  The call returns within the limit (not the
+    default 2 s), hs_get_device_error reports HS_ERR_TIMEOUT and clears it,
+    and the next call on the same stream is exact again."""
+    import time
+    w = configs.build_dedup_heavy(scale=0.2)
+    tok, ln = w["tokens"][:70000], w["lens"][:70000]     # five scan tiles
+    t, L = to_dev(tok), to_dev(ln)
+    f = hs.hs_fingerprint(t, L)
+    hs.hs_get_device_error()
+    try:
+        hs.hs_debug_scan_wait(1_000_000, 1)
+        t0 = time.perf_counter()
+        hs.hs_unique_inverse(f, t, L)
+        with pytest.raises(hs.HsError) as e:
+            hs.hs_get_device_error()
+        elapsed = time.perf_counter() - t0
+        assert e.value.status == hs.HS_ERR_TIMEOUT
+        assert elapsed < 1.0, elapsed
+    finally:
+        hs.hs_debug_scan_wait()
+    hs.hs_get_device_error()                              # the word was cleared
+    nu, uidx, inv = hs.hs_unique_inverse(f, t, L)
+    hs.hs_get_device_error()
+    ou, oi = oracle.unique_inverse(tok, ln)
+    n = int(nu.item())
+    assert n == len(ou)
+    assert (uidx[:n].cpu().numpy() == ou).all() and (inv.cpu().numpy() == oi).all()
