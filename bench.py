@@ -558,7 +558,38 @@ def row_dedup_heavy(args, dev, peaks) -> dict:
     e1.record()
     torch.cuda.synchronize()
     hs.hs_get_device_error()
-    t_all = e0.elapsed_time(e1) / K
+    t_sep = e0.elapsed_time(e1) / K
+
+    t_all = t_sep
+
+    # The fused entry point (hs_merge_rows: fingerprint + unique/inverse in
+    # one pass over the rows), timed call by call with the scatter after it.
+    ws_m = torch.empty(hs.hs_merge_rows_workspace(n), dtype=torch.uint8, device=dev)
+    mr_out = (fp, outs[0], outs[1], outs[2])
+
+    def fused_step(e=None):
+        if e: e[0].record()
+        hs.hs_merge_rows(tokens, lens, workspace=ws_m, out=mr_out)
+        if e: e[1].record()
+        hs.hs_scatter_results(payload, outs[2], dst=dst)
+
+    for _ in range(args.warmup):
+        fused_step()
+    torch.cuda.synchronize()
+    hs.hs_get_device_error()
+    mevs = [[_ev(), _ev()] for _ in range(K)]
+    for i in range(K):
+        fused_step(mevs[i])
+    torch.cuda.synchronize()
+    t_mr = statistics.mean(e[0].elapsed_time(e[1]) for e in mevs)
+    e0.record()
+    for _ in range(K):
+        fused_step()
+    e1.record()
+    torch.cuda.synchronize()
+    hs.hs_get_device_error()
+    assert int(outs[0].item()) == n_u
+    t_fused = e0.elapsed_time(e1) / K
     L = w["lens"].astype(np.int64)
     sizes = np.bincount(gi, minlength=n_u)
     multi = sizes[gi] > 1
@@ -567,17 +598,29 @@ def row_dedup_heavy(args, dev, peaks) -> dict:
     un_bytes = 4 * int(L[multi].sum()) + 8 * n + 8 * n
     sc_bytes = n_u * W + n * W + 4 * n
     ss_bytes = 8 * n + 4 * n + 8 * n_u
+    one_pass = tok_bytes + 4 * n + 8 * n + 8 * n
+    merge = _roof(fp_bytes + un_bytes, None, t_mr, peaks)
+    merge["one_pass_bytes"] = one_pass
+    merge["frac_hbm_one_pass"] = one_pass / (t_mr / 1e3) / 1e9 / peaks["hbm_gbs"]
     return {
         "workload": "dedup_heavy: 400,000 rows x 512 int32 (lens U[64,512], Zipf(1.1) over "
                     "100,000 distinct) -> %d unique; scatter %d B per row" % (n_u, W),
         "metric": "dedup rows/s (fingerprint + unique/inverse + scatter)",
         "value": n / (t_all / 1e3), "ms_per_step": t_all, "steps": K,
+        "step": "hs_fingerprint + hs_unique_inverse + hs_scatter_results",
         "ms_per_step_with_events": statistics.mean(e[0].elapsed_time(e[3]) for e in evs),
+        "fused_ms_per_step": t_fused,
         "kernels": {
+            "hs_merge_rows": merge,
             "hs_fingerprint": _roof(fp_bytes, None, t_fp, peaks),
             "hs_unique_inverse": _roof(un_bytes, None, t_un, peaks),
             "hs_scatter_results": _roof(sc_bytes, None, t_sc, peaks),
             "hs_segment_sum": _roof(ss_bytes, None, t_ss, peaks)},
+        "merge_bytes_note": "hs_merge_rows: 'bytes' are the method bytes of the two calls it "
+                            "replaces (one pass over the valid tokens + the verify re-read of "
+                            "every row in a group of size >= 2, + lens, fp, outputs); "
+                            "'one_pass_bytes' count each valid token byte once (the verify "
+                            "re-read comes from L2 in the fused pass)",
         "segment_sum_note": "priority contribution per merged node (Eq. 3) over the same "
                             "inverse map, timed after the step and not part of its value; bytes: "
                             "phi (fp64) + inverse in, one fp64 per merged node out; the output "

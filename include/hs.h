@@ -5,6 +5,7 @@
  * The stage has four steps, each one call:
  *   hs_fingerprint      hash every input row (chunk tokens or query vectors)
  *   hs_unique_inverse   merge exactly-equal rows into unique nodes + inverse map
+ *   (hs_merge_rows      the two above in one pass over the rows)
  *   hs_retrieve_topk    score merged queries against a corpus, keep top-k
  *   hs_scatter_results  fan each kept result back out to every merged row
  * two fused forms for latency-bound batches:
@@ -141,6 +142,41 @@ hs_status hs_unique_inverse(const uint64_t* fp, const int32_t* tokens, int64_t n
                             int32_t row_stride, const int32_t* lens, int32_t* n_unique_dev,
                             int32_t* unique_idx_out, int32_t* inverse_out, void* workspace,
                             size_t workspace_bytes, hs_stream_t stream);
+
+/*
+ * hs_merge_rows — hs_fingerprint and hs_unique_inverse in one pass over the
+ * rows: node signatures and the exact merge of equal rows.
+ *
+ * Paper: Section 3.3, Eq. 2 (the signature of a node) and "Dynamic Fusion
+ * and Reuse Mechanism" (I) (a node equal to one already in the window is
+ * merged into it); Appendix A.2 (merge sets M(v*) executed once);
+ * Appendix B.3, Phase 1 (duplicate detection by signature lookup).
+ * The outputs are exactly those of
+ *   hs_fingerprint(tokens, n_rows, row_stride, lens, seed_state, fp_out)
+ *   hs_unique_inverse(fp_out, tokens, ..., n_unique_dev, unique_idx_out,
+ *                     inverse_out)
+ * (fingerprints, group count, first occurrences and inverse map, bit for
+ * bit).  Each row is read from memory once: it is hashed, its fingerprint
+ * is offered to the hash table, and the row is compared in full with the
+ * smallest row holding the same fingerprint while both are still in L2.
+ * Rows not 16-byte aligned (tokens or row_stride % 4 != 0) and batches of
+ * at most 4096 rows take the two calls instead.
+ *
+ * tokens, n_rows, row_stride, lens, seed_state   as for hs_fingerprint;
+ *                 0 <= n_rows <= 2^30 - 1 (0 writes *n_unique_dev = 0).
+ *                 A length outside [0, row_stride] sets the device error
+ *                 word, that row's fingerprint is 0 and it is compared with
+ *                 its length clamped to [0, row_stride].
+ * fp_out          device uint64 [n_rows], 8-byte aligned.
+ * n_unique_dev, unique_idx_out, inverse_out   as for hs_unique_inverse.
+ * workspace       device, >= hs_merge_rows_workspace(n_rows) bytes, 256-byte
+ *                 aligned; contents on entry are ignored.
+ */
+size_t hs_merge_rows_workspace(int64_t n_rows);
+hs_status hs_merge_rows(const int32_t* tokens, int64_t n_rows, int32_t row_stride,
+                        const int32_t* lens, uint64_t seed_state, uint64_t* fp_out,
+                        int32_t* n_unique_dev, int32_t* unique_idx_out, int32_t* inverse_out,
+                        void* workspace, size_t workspace_bytes, hs_stream_t stream);
 
 /*
  * hs_unique_inverse_noalloc — hs_unique_inverse for callers that cannot
@@ -493,6 +529,16 @@ uint64_t hs_launch_count(void);
  * Returns HS_ERR_INVALID_ARG for a limit above 2 s or withhold_tile < -1.
  */
 hs_status hs_debug_scan_wait(uint64_t limit_ns, int64_t withhold_tile);
+
+/*
+ * hs_debug_merge_key_mask — test hook of hs_merge_rows; takes no part in
+ * the method.  hs_merge_rows keys its hash table by fingerprint & mask
+ * (the fingerprints it writes are not masked), so a narrow mask forces
+ * fingerprint collisions and exercises the full-row comparison that keeps
+ * the merge exact.  mask 0 restores all ones.  Process-wide; takes effect
+ * at the next launch; affects only batches of more than 4096 aligned rows.
+ */
+hs_status hs_debug_merge_key_mask(uint64_t mask);
 
 /*
  * hs_debug_stream_rows — diagnostics: stream the rows' valid prefixes with

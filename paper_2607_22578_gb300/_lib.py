@@ -99,6 +99,12 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
             lib.hs_launch_count.restype = ctypes.c_uint64
             lib.hs_debug_scan_wait.argtypes = [u64, i64]
             lib.hs_debug_scan_wait.restype = st
+            lib.hs_merge_rows_workspace.argtypes = [i64]
+            lib.hs_merge_rows_workspace.restype = sz
+            lib.hs_merge_rows.argtypes = [P, i64, i32, P, u64, P, P, P, P, P, sz, P]
+            lib.hs_merge_rows.restype = st
+            lib.hs_debug_merge_key_mask.argtypes = [u64]
+            lib.hs_debug_merge_key_mask.restype = st
             lib.hs_debug_stream_rows.argtypes = [P, i64, i32, P, i32, P, i32, P]
             lib.hs_debug_stream_rows.restype = st
             _lib = lib
@@ -180,6 +186,40 @@ def hs_unique_inverse(fp: torch.Tensor, tokens: torch.Tensor, lens: torch.Tensor
                                     _ptr(uidx), _ptr(inv), _ptr(workspace), workspace.numel(),
                                     _stream(stream)))
     return nu, uidx[:n], inv[:n]
+
+
+def hs_merge_rows_workspace(n_rows: int) -> int:
+    return int(load().hs_merge_rows_workspace(int(n_rows)))
+
+
+def hs_merge_rows(tokens: torch.Tensor, lens: torch.Tensor | None = None,
+                  seed_state: int = HS_FNV64_OFFSET_BASIS, workspace: torch.Tensor | None = None,
+                  out: tuple | None = None, stream=None):
+    """Fingerprint and exact merge in one pass.  Returns (fp [n] int64 (uint64
+    bits), n_unique_dev [1] int32, unique_idx [n] int32, inverse [n] int32);
+    `out`, if given, is that tuple of preallocated tensors."""
+    _cuda(tokens, "tokens")
+    n, stride = tokens.shape
+    dev = tokens.device
+    if out is None:
+        out = (torch.empty(max(n, 1), dtype=torch.int64, device=dev),
+               torch.empty(1, dtype=torch.int32, device=dev),
+               torch.empty(max(n, 1), dtype=torch.int32, device=dev),
+               torch.empty(max(n, 1), dtype=torch.int32, device=dev))
+    fp, nu, uidx, inv = out
+    need = hs_merge_rows_workspace(n)
+    if workspace is None:
+        workspace = torch.empty(need, dtype=torch.uint8, device=dev)
+    _check(load().hs_merge_rows(_ptr(tokens), n, stride, _ptr(lens), int(seed_state), _ptr(fp),
+                                _ptr(nu), _ptr(uidx), _ptr(inv), _ptr(workspace),
+                                workspace.numel(), _stream(stream)))
+    return fp[:n], nu, uidx[:n], inv[:n]
+
+
+def hs_debug_merge_key_mask(mask: int = 0) -> None:
+    """Test hook of hs_merge_rows: key the table by fp & mask (0 restores
+    all ones; see hs.h)."""
+    _check(load().hs_debug_merge_key_mask(int(mask)))
 
 
 def hs_unique_inverse_noalloc(fp: torch.Tensor, tokens: torch.Tensor,

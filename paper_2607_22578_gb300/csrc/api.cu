@@ -16,6 +16,9 @@ size_t unique_inverse_workspace(int64_t);
 hs_status launch_unique_inverse(const uint64_t*, const int32_t*, int64_t, int32_t,
                                 const int32_t*, int32_t*, int32_t*, int32_t*, void*,
                                 cudaStream_t);
+size_t merge_rows_workspace(int64_t);
+hs_status launch_merge_rows(const int32_t*, int64_t, int32_t, const int32_t*, uint64_t, uint64_t*,
+                            int32_t*, int32_t*, int32_t*, void*, cudaStream_t);
 size_t retrieve_topk_workspace(int64_t, int64_t, int32_t, int32_t);
 hs_status launch_retrieve_topk(const uint16_t*, int64_t, const int32_t*, const int32_t*, int64_t,
                                const uint16_t*, int64_t, int32_t, int32_t, float*, int32_t*,
@@ -155,6 +158,35 @@ hs_status hs_unique_inverse(const uint64_t* fp, const int32_t* tokens, int64_t n
     return fail(HS_ERR_WORKSPACE, "unique workspace too small: %zu < %zu", workspace_bytes, need);
   return launch_unique_inverse(fp, tokens, n_rows, row_stride, lens, n_unique_dev,
                                unique_idx_out, inverse_out, workspace, s);
+}
+
+size_t hs_merge_rows_workspace(int64_t n_rows) { return merge_rows_workspace(n_rows); }
+
+hs_status hs_merge_rows(const int32_t* tokens, int64_t n_rows, int32_t row_stride,
+                        const int32_t* lens, uint64_t seed_state, uint64_t* fp_out,
+                        int32_t* n_unique_dev, int32_t* unique_idx_out, int32_t* inverse_out,
+                        void* workspace, size_t workspace_bytes, hs_stream_t stream) {
+  clear_msg();
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (n_rows < 0 || n_rows > (int64_t)((1u << 30) - 1))
+    return fail(HS_ERR_INVALID_ARG, "n_rows outside [0, 2^30 - 1]");
+  if (row_stride < 0) return fail(HS_ERR_INVALID_ARG, "row_stride < 0");
+  if (!n_unique_dev) return fail(HS_ERR_INVALID_ARG, "n_unique_dev is NULL");
+  if (!aligned(n_unique_dev, 4)) return fail(HS_ERR_INVALID_ARG, "n_unique_dev misaligned");
+  if (n_rows == 0) return cuda_fail(cudaMemsetAsync(n_unique_dev, 0, sizeof(int32_t), s),
+                                    "n_unique clear");
+  if (!fp_out || !unique_idx_out || !inverse_out || (!tokens && row_stride > 0))
+    return fail(HS_ERR_INVALID_ARG, "NULL input or output pointer");
+  if (!aligned(fp_out, 8) || !aligned(tokens, 4) || (lens && !aligned(lens, 4)) ||
+      !aligned(unique_idx_out, 4) || !aligned(inverse_out, 4))
+    return fail(HS_ERR_INVALID_ARG, "misaligned pointer");
+  const size_t need = merge_rows_workspace(n_rows);
+  if (!workspace || !aligned(workspace, 256))
+    return fail(HS_ERR_WORKSPACE, "workspace NULL or not 256-byte aligned");
+  if (workspace_bytes < need)
+    return fail(HS_ERR_WORKSPACE, "merge workspace too small: %zu < %zu", workspace_bytes, need);
+  return launch_merge_rows(tokens, n_rows, row_stride, lens, seed_state, fp_out, n_unique_dev,
+                           unique_idx_out, inverse_out, workspace, s);
 }
 
 size_t hs_retrieve_topk_workspace(int64_t n_queries, int64_t n_corpus, int32_t dim, int32_t k) {
