@@ -560,10 +560,9 @@ def row_dedup_heavy(args, dev, peaks) -> dict:
     hs.hs_get_device_error()
     t_sep = e0.elapsed_time(e1) / K
 
-    t_all = t_sep
-
-    # The fused entry point (hs_merge_rows: fingerprint + unique/inverse in
-    # one pass over the rows), timed call by call with the scatter after it.
+    # The step as the stage runs it: hs_merge_rows (the fingerprint and the
+    # merge in one call: chunk pass, tails fused with the table insert,
+    # verify, resolve, scan, finalize) and the scatter after it.
     ws_m = torch.empty(hs.hs_merge_rows_workspace(n), dtype=torch.uint8, device=dev)
     mr_out = (fp, outs[0], outs[1], outs[2])
 
@@ -589,7 +588,7 @@ def row_dedup_heavy(args, dev, peaks) -> dict:
     torch.cuda.synchronize()
     hs.hs_get_device_error()
     assert int(outs[0].item()) == n_u
-    t_fused = e0.elapsed_time(e1) / K
+    t_all = e0.elapsed_time(e1) / K
     L = w["lens"].astype(np.int64)
     sizes = np.bincount(gi, minlength=n_u)
     multi = sizes[gi] > 1
@@ -598,29 +597,25 @@ def row_dedup_heavy(args, dev, peaks) -> dict:
     un_bytes = 4 * int(L[multi].sum()) + 8 * n + 8 * n
     sc_bytes = n_u * W + n * W + 4 * n
     ss_bytes = 8 * n + 4 * n + 8 * n_u
-    one_pass = tok_bytes + 4 * n + 8 * n + 8 * n
     merge = _roof(fp_bytes + un_bytes, None, t_mr, peaks)
-    merge["one_pass_bytes"] = one_pass
-    merge["frac_hbm_one_pass"] = one_pass / (t_mr / 1e3) / 1e9 / peaks["hbm_gbs"]
     return {
         "workload": "dedup_heavy: 400,000 rows x 512 int32 (lens U[64,512], Zipf(1.1) over "
                     "100,000 distinct) -> %d unique; scatter %d B per row" % (n_u, W),
         "metric": "dedup rows/s (fingerprint + unique/inverse + scatter)",
         "value": n / (t_all / 1e3), "ms_per_step": t_all, "steps": K,
-        "step": "hs_fingerprint + hs_unique_inverse + hs_scatter_results",
-        "ms_per_step_with_events": statistics.mean(e[0].elapsed_time(e[3]) for e in evs),
-        "fused_ms_per_step": t_fused,
+        "step": "hs_merge_rows + hs_scatter_results",
+        "separate_calls_ms_per_step": t_sep,
+        "separate_calls_ms_per_step_with_events": statistics.mean(e[0].elapsed_time(e[3])
+                                                                  for e in evs),
         "kernels": {
             "hs_merge_rows": merge,
             "hs_fingerprint": _roof(fp_bytes, None, t_fp, peaks),
             "hs_unique_inverse": _roof(un_bytes, None, t_un, peaks),
             "hs_scatter_results": _roof(sc_bytes, None, t_sc, peaks),
             "hs_segment_sum": _roof(ss_bytes, None, t_ss, peaks)},
-        "merge_bytes_note": "hs_merge_rows: 'bytes' are the method bytes of the two calls it "
-                            "replaces (one pass over the valid tokens + the verify re-read of "
-                            "every row in a group of size >= 2, + lens, fp, outputs); "
-                            "'one_pass_bytes' count each valid token byte once (the verify "
-                            "re-read comes from L2 in the fused pass)",
+        "merge_bytes_note": "hs_merge_rows: the method bytes of the two calls it combines "
+                            "(one pass over the valid tokens + the verify re-read of every row "
+                            "in a group of size >= 2, + lens, fp, outputs)",
         "segment_sum_note": "priority contribution per merged node (Eq. 3) over the same "
                             "inverse map, timed after the step and not part of its value; bytes: "
                             "phi (fp64) + inverse in, one fp64 per merged node out; the output "
@@ -904,16 +899,15 @@ def rag_mix_breakdown(stage, tokens, queries, K: int) -> dict:
 
     import paper_2607_22578_gb300 as hs
     from paper_2607_22578_gb300 import _lib
-    names = ["chunk_fingerprint", "chunk_unique", "query_fingerprint", "query_unique",
+    names = ["chunk_merge", "chunk_merge_", "query_fingerprint", "query_unique",
              "gather_unique_queries", "retrieve_topk_fanout"]
     acc = {n: 0.0 for n in names}
     Q = queries.shape[0]
     for _ in range(K):
         ev = [_ev() for _ in range(len(names) + 1)]
         ev[0].record()
-        fp = _lib.hs_fingerprint(tokens, fp_out=stage.c_fp[:tokens.shape[0]])
+        stage.dedup_chunks(tokens)
         ev[1].record()
-        _lib.hs_unique_inverse(fp, tokens, workspace=stage.ws_c, out=stage.c_out)
         ev[2].record()
         qi32 = queries.view(torch.int32)
         qfp = _lib.hs_fingerprint(qi32, fp_out=stage.q_fp[:Q])
@@ -929,7 +923,9 @@ def rag_mix_breakdown(stage, tokens, queries, K: int) -> dict:
         for i, n in enumerate(names):
             acc[n] += ev[i].elapsed_time(ev[i + 1])
     hs.hs_get_device_error()
-    return {n: v / K for n, v in acc.items()}
+    out = {n: v / K for n, v in acc.items()}
+    out.pop("chunk_merge_")
+    return out
 
 
 def rows_arm(args) -> int:

@@ -318,6 +318,23 @@ hs_status launch_chunks(const int32_t* tokens, int64_t n, int32_t stride, const 
 
 }  // namespace
 
+// The full 32-token chunks only (the first pass of hs_merge_rows, whose
+// second pass finishes the tails): 16-byte aligned rows with stride % 4 == 0.
+// Sets *ran = false when no row can have a full chunk (stride < 32).
+hs_status launch_fingerprint_chunks(const int32_t* tokens, int64_t n, int32_t stride,
+                                    const int32_t* lens, uint64_t seed, uint64_t* fp_out,
+                                    bool* ran, cudaStream_t stream) {
+  *ran = false;
+  if (stride < kTailChunk) return HS_OK;
+  const bool vec32 = (reinterpret_cast<uintptr_t>(tokens) & 31u) == 0 && stride % 8 == 0;
+  const int64_t sms = num_sms();
+  const hs_status st =
+      vec32 ? launch_chunks<32, 4, 2>(tokens, n, stride, lens, seed, fp_out, sms, stream)
+            : launch_chunks<16, 8, 2>(tokens, n, stride, lens, seed, fp_out, sms, stream);
+  if (st == HS_OK) *ran = true;
+  return st;
+}
+
 hs_status launch_fingerprint(const int32_t* tokens, int64_t n, int32_t stride,
                              const int32_t* lens, uint64_t seed, uint64_t* fp_out,
                              cudaStream_t stream) {

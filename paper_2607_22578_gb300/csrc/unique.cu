@@ -80,40 +80,6 @@ constexpr Layout layout(int64_t n) {
   return L;
 }
 
-// Workspace of the fused merge (hs_merge_rows): the counters and scan status
-// (zeroed), the table and the parent links (all-ones bytes: free slots,
-// no row, and -1 = root), the scan's ordinals, and the lists and scratch of
-// the collision resolve.
-struct MergeLayout {
-  int log2T;
-  size_t ctr, scan_status, zero_end;
-  size_t keys, idx, parent, ones_end;
-  size_t uid, coll_list, list2, rep2, list3, total;
-};
-
-constexpr MergeLayout merge_layout(int64_t n) {
-  MergeLayout L{};
-  L.log2T = table_log2(n);
-  const size_t T1 = (size_t(1) << L.log2T) + 1;
-  const int64_t tiles = (n + kScanTile - 1) / kScanTile;
-  const size_t rows = align256(sizeof(int32_t) * (size_t)n);
-  size_t o = 0;
-  L.ctr = o;          o += align256(sizeof(uint32_t) * 16);
-  L.scan_status = o;  o += align256(sizeof(uint64_t) * (size_t)tiles);
-  L.zero_end = o;
-  L.keys = o;         o += align256(sizeof(uint64_t) * T1);
-  L.idx = o;          o += align256(sizeof(uint32_t) * T1);
-  L.parent = o;       o += rows;
-  L.ones_end = o;
-  L.uid = o;          o += rows;
-  L.coll_list = o;    o += rows;
-  L.list2 = o;        o += rows;
-  L.rep2 = o;         o += rows;
-  L.list3 = o;        o += rows;
-  L.total = o;
-  return L;
-}
-
 // ---- row comparison ---------------------------------------------------------------------------
 __device__ __forceinline__ int32_t clamp_len(const int32_t* lens, int64_t r, int32_t stride,
                                              unsigned* err) {
@@ -443,15 +409,6 @@ __device__ __forceinline__ uint64_t wait_status(const volatile unsigned long lon
   }
 }
 
-// A row starts its group (is counted by the scan) when its representative is
-// itself (rep array) or when it has no parent (parent array of the fused
-// merge: -1 for a root).
-template <bool kParent>
-__device__ __forceinline__ int32_t is_group_head(int32_t v, int64_t e) {
-  return kParent ? (v == -1) : (v == (int32_t)e);
-}
-
-template <bool kParent>
 __global__ void __launch_bounds__(kScanThreads) scan_kernel(const int32_t* __restrict__ rep,
                                                             int64_t n, int32_t* __restrict__ uid,
                                                             unsigned long long* status,
@@ -475,13 +432,13 @@ __global__ void __launch_bounds__(kScanThreads) scan_kernel(const int32_t* __res
     const int64_t e = base + i;
     if (e + 3 < n) {
       const int4 v = *reinterpret_cast<const int4*>(rep + e);
-      x[i] = is_group_head<kParent>(v.x, e);
-      x[i + 1] = is_group_head<kParent>(v.y, e + 1);
-      x[i + 2] = is_group_head<kParent>(v.z, e + 2);
-      x[i + 3] = is_group_head<kParent>(v.w, e + 3);
+      x[i] = v.x == (int32_t)e;
+      x[i + 1] = v.y == (int32_t)(e + 1);
+      x[i + 2] = v.z == (int32_t)(e + 2);
+      x[i + 3] = v.w == (int32_t)(e + 3);
     } else {
 #pragma unroll
-      for (int j = 0; j < 4; ++j) x[i + j] = (e + j < n) ? is_group_head<kParent>(rep[e + j], e + j) : 0;
+      for (int j = 0; j < 4; ++j) x[i + j] = (e + j < n) ? (rep[e + j] == (int32_t)(e + j)) : 0;
     }
     run += x[i] + x[i + 1] + x[i + 2] + x[i + 3];
   }
@@ -554,11 +511,6 @@ __global__ void __launch_bounds__(kScanThreads) scan_kernel(const int32_t* __res
   }
 }
 
-// kParent: rep holds parent links of the fused merge (a smaller row of the
-// same group, or -1 for the group's first row); the group's first row is
-// found by following them (each link goes to a smaller index, so the walk
-// ends).
-template <bool kParent>
 __global__ void __launch_bounds__(256) finalize_kernel(const int32_t* __restrict__ rep,
                                                        const int32_t* __restrict__ uid, int64_t n,
                                                        const int32_t* __restrict__ n_unique,
@@ -569,403 +521,171 @@ __global__ void __launch_bounds__(256) finalize_kernel(const int32_t* __restrict
   const int64_t nu = *n_unique;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
        i += (int64_t)gridDim.x * blockDim.x) {
-    int32_t r;
-    if constexpr (kParent) {
-      int32_t x = (int32_t)i, p = rep[i];
-      while (p >= 0) {
-        x = p;
-        p = rep[x];
-      }
-      r = x;
-    } else {
-      r = rep[i];
-    }
+    const int32_t r = rep[i];
     inverse[i] = uid[r];
     if (r == (int32_t)i) unique_idx[uid[i]] = (int32_t)i;
     if (i >= nu) unique_idx[i] = 0;     // the tail is a valid row map too
   }
 }
 
-// ---- fused merge: fingerprint + table insert + verify in one pass ----------------------------
-// hs_merge_rows reads every row once.  A CTA has kMrH hash warps; each has
-// four verify warps, one per pass of its tiles.
-//
-// Hash warp: takes the next 128-row tile of the input from a global ticket
-// (tiles go out in row order), ranks the tile's rows by their number of full
-// 32-token chunks and hashes them in four passes of 32 rows of similar
-// length, a row per lane, so a pass lasts about as many rounds as its rows
-// have chunks.  In each round the warp stages one full chunk of every row
-// into a shared-memory ring (kMrStages - 1 rounds ahead of hashing) with
-// coalesced 16-byte cp.async copies (eight lanes per 128-byte chunk; only
-// bytes below each row's length are read), then each lane hashes its row's
-// chunk (FNV-1a, as the fingerprint kernels; a lane whose row has fewer
-// full chunks hashes into a scratch state it drops).  A last round stages
-// and hashes every row's remaining L mod 32 tokens.  The warp writes the
-// pass's fingerprints and hands (row, key, length) to the pass's verify
-// warp; it never waits on global memory itself, so few hash warps with
-// deep staging keep the hash chains busy while the bytes in flight between
-// a row's first read and its comparison stay far below L2's capacity.
-//
-// Verify warp (pass q of each tile): offers its 32 rows to the table, whose
-// slot keeps the smallest row index with that key; the value the slot held
-// before (atomicMin) says what the row must be compared with:
-//   - a smaller row r holds the key: compare the row with r; if equal, the
-//     row links to r;
-//   - the row displaced a larger row x (x came first): compare x with the
-//     row; if equal, x links to the row;
-//   - the slot was empty: nothing to compare yet.
-// Rows of a pass with equal keys are combined first (the smallest inserts,
-// the others compare with it or with the smaller row it found).  Each row is
-// the first element of at most one pair, so each link has one writer, and
-// every link goes to a smaller index.  A lane compares its pair in full, 16
-// bytes at a time with kMrPieces pieces of both rows in flight; both rows
-// were streamed in moments ago or are hot representatives, so they come
-// from L2.  A mismatch (a fingerprint collision) lists the row.
-//
-// After this kernel every row links to an equal smaller row, is a root (-1)
-// or is listed (-2).  The resolve kernel compares each listed row with the
-// final smallest row of its key and regroups the rest exactly (as
-// hs_unique_inverse does); the scan counts the roots and the finalize kernel
-// follows the links to each row's root.
-constexpr int kMrH = 4;                                // hash warps per CTA
-constexpr int kMrPasses = 4;                           // passes per tile = verify warps per hash warp
-constexpr int kMrStages = 8;                           // chunk rounds in flight per hash warp
-constexpr int kMrPieces = 8;                           // piece pairs per verify lane in flight
-constexpr int kMrTile = 32 * kMrPasses;                // rows per tile
-constexpr int kMrThreads = 32 * kMrH * (1 + kMrPasses);
-constexpr int kMrRowBytes = 144;                       // a 128-byte chunk + 16 bytes of padding
-constexpr int kMrStageBytes = 32 * kMrRowBytes;        // one round of a warp's 32 rows
-constexpr size_t kMrSmem = (size_t)kMrH * kMrStages * kMrStageBytes;
-constexpr int kCtrTicket = 3;                          // next tile (fused merge)
-static_assert(kMrThreads <= 1024, "one block");
+// ---- verify over flat piece lists ------------------------------------------------------------
+// Verify of 32 consecutive rows per warp against their representatives (the
+// table's smallest row with the same fingerprint).  The rows that need a
+// comparison (representative another row, lengths equal) are compared as
+// one flat list of 16-byte piece pairs: the warp's pairs are laid end to
+// end (a prefix sum of their piece counts in shared memory), and each lane
+// takes every 32nd piece pair, kVerifyPieces of them in flight per round,
+// so a warp's rows cost about (their bytes / 4 KB) round trips whatever
+// their lengths.  The tokens of a pair's last piece past its length are
+// masked.  Needs 16-byte aligned rows (stride % 4 == 0).
+constexpr int kVerifyPieces = 4;
+constexpr int kVerifyThreads = 256;
 
-struct MrMailbox {                 // per hash warp
-  uint64_t key[kMrPasses][32];     // pass q of the current tile: table key,
-  int32_t row[kMrPasses][32];      // row index (-1: none),
-  int32_t len[kMrPasses][32];      // length clamped to [0, stride]
-  int32_t live[kMrPasses];         // 1: a pass; 0: the hash warp has finished
-  int32_t order[kMrTile];          // the tile's row offsets by full-chunk count
-  int32_t olen[kMrTile];           // and their lengths
-  uint64_t full[kMrPasses];        // mbarrier: pass q published (1 arrival)
-  uint64_t empty[kMrPasses];       // mbarrier: pass q read by its verify warp (1 arrival)
-};
-
-// Bounded wait (every lane) for the phase of parity `parity` of a mailbox
-// mbarrier; false if the wait ran out or the block aborted.
-__device__ __forceinline__ bool mr_wait_phase(uint64_t* bar, uint32_t parity, volatile int* abort,
-                                              unsigned* err) {
-  if (mbar_wait(bar, parity, abort)) return true;
-  set_error(err, kErrTimeout);
-  return false;
-}
-
-// FNV-1a rounds over the 32 staged tokens of a chunk.
-template <bool SMALL>
-__device__ __forceinline__ void mr_hash_chunk(uint32_t& lo, uint32_t& hi, const uint32_t (&w)[32]) {
-#pragma unroll
-  for (int t = 0; t < 32; ++t) {
-    if (SMALL)
-      fnv::hash_word_small(lo, hi, w[t]);
-    else
-      fnv::hash_word_full(lo, hi, w[t]);
-  }
-}
-
-__device__ __forceinline__ void mr_hash_role(const int32_t* __restrict__ tokens, int64_t n,
-                                             int32_t stride, const int32_t* __restrict__ lens,
-                                             uint64_t seed, uint64_t key_mask,
-                                             uint64_t* __restrict__ fp_out, uint32_t* ctr,
-                                             uint32_t stage_base, MrMailbox& mb,
-                                             volatile int* abort, unsigned* err) {
-  const int lane = threadIdx.x & 31, p = lane & 7, sub = lane >> 3;
-  const uint32_t seed_lo = (uint32_t)seed, seed_hi = (uint32_t)(seed >> 32);
-  uint32_t tile = 0;
-  if (lane == 0) tile = atomicAdd(ctr + kCtrTicket, 1u);
-  tile = __shfl_sync(0xffffffffu, tile, 0);
-  for (unsigned tn = 0;; ++tn) {                       // tiles done by this warp
-    const int64_t t0 = (int64_t)tile * kMrTile;
-    if (t0 >= n || *abort) {
-      for (int q = 0; q < kMrPasses; ++q) {            // tell every verify warp to stop
-        if (tn >= 1 && !mr_wait_phase(&mb.empty[q], (tn - 1) & 1u, abort, err)) return;
-        if (lane == 0) {
-          mb.live[q] = 0;
-          mbar_arrive(&mb.full[q]);
-        }
-      }
-      return;
-    }
-    uint32_t next = 0;                                 // the next tile, fetched ahead
-    if (lane == 0) next = atomicAdd(ctr + kCtrTicket, 1u);
-    // lengths of the tile's rows (offset lane + 32 q) and their rank by
-    // (full chunks, offset): unique keys, rows past n rank last
-    int32_t L4[kMrPasses], key4[kMrPasses];
-#pragma unroll
-    for (int q = 0; q < kMrPasses; ++q) {
-      const int64_t r = t0 + lane + 32 * q;
-      L4[q] = r < n ? (lens ? __ldg(lens + r) : stride) : 0;
-      const bool bad = L4[q] < 0 || L4[q] > stride;
-      const int32_t nf = r < n ? min(bad ? 0 : L4[q] >> 5, 0x7ffffe) : 0x7fffff;
-      key4[q] = (nf << 8) | (lane + 32 * q);
-    }
-    int32_t rank4[kMrPasses] = {};
-#pragma unroll 4
-    for (int sl = 0; sl < 32; ++sl) {
-#pragma unroll
-      for (int q2 = 0; q2 < kMrPasses; ++q2) {
-        const int32_t o = __shfl_sync(0xffffffffu, key4[q2], sl);
-#pragma unroll
-        for (int q = 0; q < kMrPasses; ++q) rank4[q] += o < key4[q];
-      }
-    }
-#pragma unroll
-    for (int q = 0; q < kMrPasses; ++q) {
-      mb.order[rank4[q]] = lane + 32 * q;
-      mb.olen[rank4[q]] = L4[q];
-    }
-    __syncwarp();
-    for (int pass = 0; pass < kMrPasses; ++pass) {
-      const int off = mb.order[32 * pass + lane];
-      const int32_t L = mb.olen[32 * pass + lane];
-      const int64_t r = t0 + off;
-      const bool valid = r < n;
-      const bool bad = valid && (L < 0 || L > stride);
-      if (bad) set_error(err, kErrInvalidArg);
-      const int32_t Lcmp = L < 0 ? 0 : (L > stride ? stride : L);
-      const int32_t Lh = bad ? 0 : L;                 // tokens hashed
-      const int nfull = Lh >> 5;
-      const int F = (int)__reduce_max_sync(0xffffffffu, (unsigned)nfull);
-      int32_t Lc[8];                                  // lengths of the rows this lane copies
-      const int32_t* rowc[8];                         // and their first token
-#pragma unroll
-      for (int kk = 0; kk < 8; ++kk) {
-        Lc[kk] = __shfl_sync(0xffffffffu, Lh, 4 * kk + sub);
-        const int oc = __shfl_sync(0xffffffffu, off, 4 * kk + sub);
-        rowc[kk] = tokens + (t0 + oc) * (int64_t)stride;
-      }
-      auto stage = [&](int c) {
-        if (c <= F) {
-          const uint32_t sb = stage_base + (uint32_t)((c % kMrStages) * kMrStageBytes);
-#pragma unroll
-          for (int kk = 0; kk < 8; ++kk) {
-            const int row = 4 * kk + sub;
-            const int32_t Lr = Lc[kk];
-            // full chunk c, or (round F) the row's tail chunk
-            const int32_t t = (c < F ? 32 * c : (Lr & ~31)) + 4 * p;
-            const bool want = c < F ? (32 * c + 32 <= Lr) : (t < Lr);
-            if (want) cp_async16(sb + (uint32_t)(row * kMrRowBytes + 16 * p), rowc[kk] + t);
-          }
-        }
-        cp_async_commit();
-      };
-#pragma unroll
-      for (int c = 0; c < kMrStages - 1; ++c) stage(c);
-      uint32_t lo = seed_lo, hi = seed_hi;
-      for (int c = 0; c <= F; ++c) {
-        stage(c + kMrStages - 1);
-        cp_async_wait<kMrStages - 1>();
-        __syncwarp();
-        const uint32_t src =
-            stage_base + (uint32_t)((c % kMrStages) * kMrStageBytes + lane * kMrRowBytes);
-        uint32_t w[32];
-#pragma unroll
-        for (int q = 0; q < 8; ++q) {
-          const uint4 v = lds128(src + 16 * q);
-          w[4 * q] = v.x;
-          w[4 * q + 1] = v.y;
-          w[4 * q + 2] = v.z;
-          w[4 * q + 3] = v.w;
-        }
-        __syncwarp();   // every lane has read this buffer before it is staged again
-        if (c < F) {
-          const bool mine = c < nfull;                // a full chunk of this lane's row
-          uint32_t any = 0;
-#pragma unroll
-          for (int t = 0; t < 32; ++t) any |= w[t];
-          const bool small = __all_sync(0xffffffffu, !mine || (any >> 16) == 0u);
-          uint32_t lo2 = lo, hi2 = hi;
-          if (small) mr_hash_chunk<true>(lo2, hi2, w);
-          else mr_hash_chunk<false>(lo2, hi2, w);
-          lo = mine ? lo2 : lo;
-          hi = mine ? hi2 : hi;
-        } else {
-          const int32_t m = Lh - 32 * nfull;          // 0 .. 31 tail tokens
-#pragma unroll
-          for (int t = 0; t < 31; ++t)
-            if (t < m) fnv::hash_word(lo, hi, w[t]);
-        }
-      }
-      cp_async_wait_all();
-      const uint64_t fpv = bad ? 0ull : (((uint64_t)hi << 32) | lo);
-      if (valid) fp_out[r] = fpv;
-      // hand the pass to its verify warp once it has read the previous tile's
-      if (tn >= 1 && !mr_wait_phase(&mb.empty[pass], (tn - 1) & 1u, abort, err)) return;
-      mb.key[pass][lane] = fpv & key_mask;
-      mb.row[pass][lane] = valid ? (int32_t)r : -1;
-      mb.len[pass][lane] = Lcmp;
-      if (lane == 0) mb.live[pass] = 1;
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&mb.full[pass]);  // release: the mailbox writes come first
-    }
-    tile = __shfl_sync(0xffffffffu, next, 0);
-  }
-}
-
-// Verify warp of pass q: offers its rows to the table, then compares each
-// row's pair in full (a lane per pair), kMrPieces pieces of both rows in
-// flight (the tokens of the last piece past the length are masked).  The
-// length compared is that of the hash lane's row; the other row's length is
-// loaded beside the first pieces, and unequal lengths mean the rows differ.
-__device__ __forceinline__ void mr_verify_role(const int32_t* __restrict__ tokens, int32_t stride,
-                                               const int32_t* __restrict__ lens, uint64_t* keys,
-                                               uint32_t* idx, int log2T, int32_t* parent,
-                                               int32_t* coll_list, uint32_t* ctr, int q,
-                                               MrMailbox& mb, volatile int* abort,
-                                               unsigned* err) {
-  const int lane = threadIdx.x & 31;
-  for (unsigned tn = 0;; ++tn) {
-    if (!mr_wait_phase(&mb.full[q], tn & 1u, abort, err)) break;
-    if (*reinterpret_cast<volatile int32_t*>(&mb.live[q]) == 0) break;
-    const uint64_t key = mb.key[q][lane];
-    const int32_t r = mb.row[q][lane], Lk = mb.len[q][lane];
-    __syncwarp();
-    if (lane == 0) mbar_arrive(&mb.empty[q]);      // the pass is in registers now
-    const bool valid = r >= 0;
-    const unsigned act = __ballot_sync(0xffffffffu, valid);
-    int32_t a = -1, b = -1;
-    if (valid) {
-      const unsigned peers = __match_any_sync(act, key);
-      const uint32_t rmin = __reduce_min_sync(peers, (uint32_t)r);
-      uint32_t old = 0xffffffffu;
-      if ((uint32_t)r == rmin) {
-        const uint32_t s = insert_key(keys, key, log2T);
-        const uint32_t cur = *reinterpret_cast<volatile uint32_t*>(idx + s);
-        old = cur < (uint32_t)r ? cur : atomicMin(idx + s, (uint32_t)r);
-      }
-      old = __reduce_min_sync(peers, old);
-      if ((uint32_t)r == rmin) {
-        if (old < (uint32_t)r) {                   // a smaller row holds the key
-          a = r;
-          b = (int32_t)old;
-        } else if (old != kNoRow) {                // this row displaced a larger one
-          a = (int32_t)old;
-          b = r;
-        }
-      } else {
-        a = r;
-        b = (int32_t)(old < rmin ? old : rmin);
-      }
-    }
-    if (a < 0) continue;
-    const int32_t la = clamp_len(lens, a, stride, err);
-    const int32_t lb = clamp_len(lens, b, stride, err);
-    const uint4* pa = reinterpret_cast<const uint4*>(tokens + (int64_t)a * stride);
-    const uint4* pb = reinterpret_cast<const uint4*>(tokens + (int64_t)b * stride);
-    const int32_t P = (Lk + 3) >> 2;                 // 16-byte pieces to compare
-    bool differ = false;
-    for (int32_t j0 = 0; j0 < P; j0 += kMrPieces) {
-      uint4 x[kMrPieces], y[kMrPieces];
-#pragma unroll
-      for (int u = 0; u < kMrPieces; ++u) {
-        if (j0 + u < P) {
-          x[u] = __ldg(pa + j0 + u);
-          y[u] = __ldg(pb + j0 + u);
-        }
-      }
-#pragma unroll
-      for (int u = 0; u < kMrPieces; ++u) {
-        const int32_t vt = Lk - 4 * (j0 + u);        // live tokens in the piece
-        if (vt > 0)
-          differ |= (x[u].x != y[u].x) | ((vt > 1) & (x[u].y != y[u].y)) |
-                    ((vt > 2) & (x[u].z != y[u].z)) | ((vt > 3) & (x[u].w != y[u].w));
-      }
-    }
-    if (la == lb && !differ) {
-      parent[a] = b;
-    } else {
-      parent[a] = -2;
-      coll_list[atomicAdd(ctr + kCtrColl, 1u)] = a;
-    }
-  }
-}
-
-__global__ void __launch_bounds__(kMrThreads, 1) merge_rows_kernel(
-    const int32_t* __restrict__ tokens, int64_t n, int32_t stride,
-    const int32_t* __restrict__ lens, uint64_t seed, uint64_t key_mask,
-    uint64_t* __restrict__ fp_out, uint64_t* keys, uint32_t* idx, int log2T, int32_t* parent,
-    int32_t* coll_list, uint32_t* ctr, unsigned* err) {
-  extern __shared__ __align__(128) uint8_t mr_smem[];
-  __shared__ MrMailbox s_mb[kMrH];
-  __shared__ int s_abort;
-  const int tid = threadIdx.x, warp = tid >> 5;
-  for (int i = tid; i < kMrH * kMrPasses; i += blockDim.x) {
-    mbar_init(&s_mb[i / kMrPasses].full[i % kMrPasses], 1);
-    mbar_init(&s_mb[i / kMrPasses].empty[i % kMrPasses], 1);
-    s_mb[i / kMrPasses].live[i % kMrPasses] = 0;
-  }
-  if (tid == 0) s_abort = 0;
-  __syncthreads();
+__global__ void __launch_bounds__(kVerifyThreads) verify_flat_kernel(
+    const uint64_t* __restrict__ fp, uint64_t key_mask, int64_t n,
+    const uint64_t* __restrict__ keys, const uint32_t* __restrict__ idx, int log2T,
+    const int32_t* __restrict__ tokens, int32_t stride, const int32_t* __restrict__ lens,
+    int32_t* __restrict__ rep, int32_t* coll_list, uint32_t* ctr, unsigned* err) {
   pdl_wait();
   pdl_trigger();
-  if (warp < kMrH) {
-    mr_hash_role(tokens, n, stride, lens, seed, key_mask, fp_out, ctr,
-                 smem_u32(mr_smem) + (uint32_t)(warp * kMrStages * kMrStageBytes), s_mb[warp],
-                 &s_abort, err);
-  } else {
-    const int v = warp - kMrH;
-    mr_verify_role(tokens, stride, lens, keys, idx, log2T, parent, coll_list, ctr,
-                   v % kMrPasses, s_mb[v / kMrPasses], &s_abort, err);
-  }
-}
-
-// The listed rows of the fused merge (practically none: fingerprint
-// collisions).  Each is compared with the final smallest row of its key,
-// which is smaller than it; equal rows link to it.  The rest can only equal
-// each other and are regrouped exactly as in hs_unique_inverse (a second
-// key, then peeling), in the scratch rep2; their roots become -1.
-template <bool VEC>
-__global__ void __launch_bounds__(kResolveThreads) merge_resolve_kernel(
-    const uint64_t* __restrict__ fp, uint64_t key_mask, const int32_t* __restrict__ tokens,
-    int32_t stride, const int32_t* __restrict__ lens, int32_t* parent,
-    const int32_t* coll_list, const uint32_t* ctr, uint64_t* keys, uint32_t* idx, int log2T,
-    int32_t* list2, int32_t* rep2, int32_t* list3, unsigned* err) {
-  pdl_wait();
-  pdl_trigger();
-  __shared__ uint32_t s_m2;
-  const uint32_t m = ctr[kCtrColl];
-  if (m == 0) return;
-  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5, nw = blockDim.x >> 5;
-  if (tid == 0) s_m2 = 0;
-  __syncthreads();
-  for (uint32_t b0 = (uint32_t)w * 32u; b0 < m; b0 += (uint32_t)nw * 32u) {
-    const uint32_t c = b0 + lane;
-    const bool valid = c < m;
-    const int64_t a = valid ? coll_list[c] : 0;
+  __shared__ int32_t s_pre[kVerifyThreads / 32][32];
+  __shared__ int32_t s_a[kVerifyThreads / 32][32];
+  __shared__ int32_t s_b[kVerifyThreads / 32][32];
+  __shared__ int32_t s_len[kVerifyThreads / 32][32];
+  const int lane = threadIdx.x & 31, wl = threadIdx.x >> 5;
+  const int64_t warps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  const int64_t w = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  for (int64_t p0 = w * 32; p0 < n; p0 += warps * 32) {
+    const int64_t a = p0 + lane;
+    const bool valid = a < n;
     int64_t r = a;
+    int32_t la = 0, lr = 0;
     if (valid) {
-      const uint32_t v = idx[find_key(keys, fp[a] & key_mask, log2T)];
-      if (v < (uint32_t)a) r = v;
+      const uint32_t v = idx[find_key(keys, __ldg(fp + a) & key_mask, log2T)];
+      if (v < (uint32_t)n) r = v;
+      else set_error(err, kErrInvalidArg);   // not reached: every row was inserted
+      la = clamp_len(lens, a, stride, err);
+      lr = r != a ? clamp_len(lens, r, stride, err) : la;
     }
-    const bool merged = verify_warp<VEC>(tokens, stride, lens, valid, a, r, err);
-    if (valid) {
-      if (merged && r != a) {
-        parent[a] = (int32_t)r;
-      } else {
-        rep2[a] = -1;
-        list2[atomicAdd(&s_m2, 1u)] = (int32_t)a;
+    const bool need = valid && r != a && la == lr;
+    int32_t incl = need ? (la + 3) >> 2 : 0;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += y;
+    }
+    s_pre[wl][lane] = incl;
+    s_a[wl][lane] = (int32_t)a;
+    s_b[wl][lane] = (int32_t)r;
+    s_len[wl][lane] = la;
+    const int32_t total = __shfl_sync(0xffffffffu, incl, 31);
+    __syncwarp();
+    uint32_t differ = 0;                       // bit t: a piece of pair t differs
+    int t = 0;                                 // this lane's current pair (only moves forward)
+    for (int32_t g0 = 0; g0 < total; g0 += 32 * kVerifyPieces) {
+      uint4 x[kVerifyPieces], y[kVerifyPieces];
+      int tt[kVerifyPieces], vt[kVerifyPieces];
+#pragma unroll
+      for (int u = 0; u < kVerifyPieces; ++u) {
+        const int32_t g = g0 + u * 32 + lane;
+        tt[u] = -1;
+        if (g < total) {
+          while (s_pre[wl][t] <= g) ++t;
+          const int32_t j = g - (t > 0 ? s_pre[wl][t - 1] : 0);
+          x[u] = __ldg(reinterpret_cast<const uint4*>(tokens + (int64_t)s_a[wl][t] * stride) + j);
+          y[u] = __ldg(reinterpret_cast<const uint4*>(tokens + (int64_t)s_b[wl][t] * stride) + j);
+          tt[u] = t;
+          vt[u] = s_len[wl][t] - 4 * j;        // live tokens in this piece (>= 1)
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < kVerifyPieces; ++u) {
+        if (tt[u] >= 0) {
+          const bool d = (x[u].x != y[u].x) | ((vt[u] > 1) & (x[u].y != y[u].y)) |
+                         ((vt[u] > 2) & (x[u].z != y[u].z)) | ((vt[u] > 3) & (x[u].w != y[u].w));
+          if (d) differ |= 1u << tt[u];
+        }
       }
     }
+    differ = __reduce_or_sync(0xffffffffu, differ);
+    __syncwarp();                              // shared lists free for the next rows
+    if (valid) {
+      const bool merged = r == a || (need && !((differ >> lane) & 1u));
+      rep[a] = merged ? (int32_t)r : -1;
+      if (!merged) coll_list[atomicAdd(ctr + kCtrColl, 1u)] = (int32_t)a;
+    }
   }
-  __syncthreads();
-  const uint32_t m2 = s_m2;
-  if (m2 == 0) return;
-  const uint32_t m3 =
-      regroup_block<VEC>(fp, tokens, stride, lens, rep2, list2, m2, keys, idx, list3, err);
-  if (m3) peel_block<VEC>(fp, tokens, stride, lens, rep2, list3, m3, err);
-  __syncthreads();
-  for (uint32_t c = tid; c < m2; c += blockDim.x) {
-    const int32_t a = list2[c];
-    const int32_t r = rep2[a];
-    parent[a] = r == a ? -1 : r;
+}
+
+// ---- hs_merge_rows: second pass of the fingerprint, fused with the insert ---------------------
+// One thread per row finishes the fingerprint (the last L mod 32 tokens,
+// from the state the chunk kernel left in fp_out, or the whole row when it
+// is shorter than 32 tokens or the chunk kernel did not run), writes it,
+// and offers (fp & key_mask, row) to the table in the same pass: rows of a
+// warp with equal keys are combined and the smallest index inserts
+// (atomicMin), as insert_kernel does.  An invalid length sets the error
+// word and a zero fingerprint, as hs_fingerprint does.
+__global__ void __launch_bounds__(256) tails_insert_kernel(
+    const int32_t* __restrict__ tokens, int64_t n, int32_t stride,
+    const int32_t* __restrict__ lens, uint64_t seed, bool chunks_ran, uint64_t key_mask,
+    uint64_t* __restrict__ fp_out, uint64_t* keys, uint32_t* idx, int log2T, unsigned* err) {
+  pdl_wait();
+  pdl_trigger();
+  constexpr int T = 32;
+  for (int64_t base = (int64_t)blockIdx.x * blockDim.x; base < n;
+       base += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t r = base + threadIdx.x;
+    const bool valid = r < n;
+    uint64_t f = 0;
+    if (valid) {
+      const int32_t L = lens ? __ldg(lens + r) : stride;
+      if (L < 0 || L > stride) {
+        set_error(err, kErrInvalidArg);
+      } else {
+        const int32_t m = L % T;
+        const bool from_chunks = chunks_ran && L >= T;
+        if (from_chunks && m == 0) {
+          f = fp_out[r];                           // the chunk kernel wrote the final value
+        } else {
+          uint32_t lo = (uint32_t)seed, hi = (uint32_t)(seed >> 32);
+          int32_t t0 = 0;
+          if (from_chunks) {
+            const uint64_t st = fp_out[r];
+            lo = (uint32_t)st;
+            hi = (uint32_t)(st >> 32);
+            t0 = L - m;
+          }
+          // at most 31 tokens remain past the full chunks (fewer than 32 in a
+          // short row): all their 16-byte pieces are loaded before hashing
+          const int32_t* src = tokens + r * (int64_t)stride + t0;
+          const int32_t m2 = L - t0;               // tokens to hash here
+          if (m2 < T) {
+            uint4 v[T / 4];
+#pragma unroll
+            for (int q = 0; q < T / 4; ++q)
+              if (4 * q < m2) v[q] = __ldg(reinterpret_cast<const uint4*>(src + 4 * q));
+#pragma unroll
+            for (int q = 0; q < T / 4; ++q) {
+              if (4 * q < m2) fnv::hash_word(lo, hi, v[q].x);
+              if (4 * q + 1 < m2) fnv::hash_word(lo, hi, v[q].y);
+              if (4 * q + 2 < m2) fnv::hash_word(lo, hi, v[q].z);
+              if (4 * q + 3 < m2) fnv::hash_word(lo, hi, v[q].w);
+            }
+          } else {                                 // a whole row (no chunk pass ran)
+            for (int32_t t = 0; t < m2; t += 4) {  // 16-byte pieces, the last one masked
+              const uint4 v = __ldg(reinterpret_cast<const uint4*>(src + t));
+              fnv::hash_word(lo, hi, v.x);
+              if (t + 1 < m2) fnv::hash_word(lo, hi, v.y);
+              if (t + 2 < m2) fnv::hash_word(lo, hi, v.z);
+              if (t + 3 < m2) fnv::hash_word(lo, hi, v.w);
+            }
+          }
+          f = ((uint64_t)hi << 32) | lo;
+        }
+      }
+      fp_out[r] = f;
+    }
+    insert_row(keys, idx, log2T, valid, f & key_mask, (uint32_t)r);
   }
 }
 
@@ -1154,8 +874,9 @@ hs_status launch_unique_inverse(const uint64_t* fp, const int32_t* tokens, int64
              L.log2T);
   const unsigned vgrid = grid_for(n, 256, sms * 8);   // one warp per 32 rows
   if (vec)
-    launch_pdl(verify_kernel<true>, dim3(vgrid), dim3(256), 0, stream, fp, n, keys, idx, L.log2T,
-               tokens, stride, lens, rep, coll_list, ctr, err);
+    launch_pdl(verify_flat_kernel, dim3(vgrid), dim3(kVerifyThreads), 0, stream, fp, ~0ull, n,
+               (const uint64_t*)keys, (const uint32_t*)idx, L.log2T, tokens, stride, lens, rep,
+               coll_list, ctr, err);
   else
     launch_pdl(verify_kernel<false>, dim3(vgrid), dim3(256), 0, stream, fp, n, keys, idx, L.log2T,
                tokens, stride, lens, rep, coll_list, ctr, err);
@@ -1166,9 +887,9 @@ hs_status launch_unique_inverse(const uint64_t* fp, const int32_t* tokens, int64
     launch_pdl(resolve_kernel<false>, dim3(1), dim3(kResolveThreads), 0, stream, fp, tokens,
                stride, lens, rep, coll_list, ctr, keys, idx, uid, err);
   const int64_t tiles = (n + kScanTile - 1) / kScanTile;
-  launch_pdl(scan_kernel<false>, dim3((unsigned)tiles), dim3(kScanThreads), 0, stream, rep, n, uid, status,
+  launch_pdl(scan_kernel, dim3((unsigned)tiles), dim3(kScanThreads), 0, stream, rep, n, uid, status,
              ctr, n_unique_dev, err, g_scan_wait_limit_ns.load(), g_scan_withhold_tile.load());
-  launch_pdl(finalize_kernel<false>, dim3(grid_for(n, 256, sms * 8)), dim3(256), 0, stream, rep, uid, n,
+  launch_pdl(finalize_kernel, dim3(grid_for(n, 256, sms * 8)), dim3(256), 0, stream, rep, uid, n,
              n_unique_dev, unique_idx, inverse);
   count_launches(5);  // insert, verify, resolve, scan, finalize
   return cuda_fail(cudaGetLastError(), "unique_inverse launch");
@@ -1176,69 +897,65 @@ hs_status launch_unique_inverse(const uint64_t* fp, const int32_t* tokens, int64
 
 hs_status launch_fingerprint(const int32_t*, int64_t, int32_t, const int32_t*, uint64_t,
                              uint64_t*, cudaStream_t);
+hs_status launch_fingerprint_chunks(const int32_t*, int64_t, int32_t, const int32_t*, uint64_t,
+                                    uint64_t*, bool*, cudaStream_t);
 
-// Test hook of the fused merge (hs_debug_merge_key_mask): the table key is
+// Test hook of hs_merge_rows (hs_debug_merge_key_mask): the table key is
 // fp & mask, so a narrow mask forces fingerprint collisions.
 std::atomic<uint64_t> g_merge_key_mask{~0ull};
 
-size_t merge_rows_workspace(int64_t n) {
-  if (n <= 0) return 256;
-  const size_t a = merge_layout(n).total, b = layout(n).total;
-  return a > b ? a : b;
-}
+size_t merge_rows_workspace(int64_t n) { return unique_inverse_workspace(n); }
 
+// hs_merge_rows: the fingerprint's chunk pass, then one pass that finishes
+// the fingerprints and inserts them (no separate insert pass), then the
+// verify, collision resolve, scan and finalize of hs_unique_inverse.
 hs_status launch_merge_rows(const int32_t* tokens, int64_t n, int32_t stride, const int32_t* lens,
                             uint64_t seed, uint64_t* fp_out, int32_t* n_unique_dev,
                             int32_t* unique_idx, int32_t* inverse, void* ws, cudaStream_t stream) {
   const bool vec = ((reinterpret_cast<uintptr_t>(tokens) & 15u) == 0) && (stride % 4 == 0);
+  const uint64_t mask = g_merge_key_mask.load();
   if (n <= kSmallRows || !vec) {   // few rows, or rows not 16-byte aligned: the two calls
-    const hs_status st = launch_fingerprint(tokens, n, stride, lens, seed, fp_out, stream);
+    hs_status st = launch_fingerprint(tokens, n, stride, lens, seed, fp_out, stream);
     if (st != HS_OK) return st;
     return launch_unique_inverse(fp_out, tokens, n, stride, lens, n_unique_dev, unique_idx,
                                  inverse, ws, stream);
   }
   unsigned* err = device_error_word();
   if (!err) return fail(HS_ERR_CUDA, "could not resolve the device error word");
-  static std::atomic<uint64_t> configured{0};
-  const hs_status cst = once_per_device(configured, [] {
-    return cuda_fail(cudaFuncSetAttribute(merge_rows_kernel,
-                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                          (int)kMrSmem),
-                     "merge smem attribute");
-  });
-  if (cst != HS_OK) return cst;
-  const MergeLayout L = merge_layout(n);
+  const Layout L = layout(n);
   char* w = static_cast<char*>(ws);
   uint32_t* ctr = reinterpret_cast<uint32_t*>(w + L.ctr);
   auto* status = reinterpret_cast<unsigned long long*>(w + L.scan_status);
   uint64_t* keys = reinterpret_cast<uint64_t*>(w + L.keys);
   uint32_t* idx = reinterpret_cast<uint32_t*>(w + L.idx);
-  int32_t* parent = reinterpret_cast<int32_t*>(w + L.parent);
+  int32_t* rep = reinterpret_cast<int32_t*>(w + L.rep);
   int32_t* uid = reinterpret_cast<int32_t*>(w + L.uid);
   int32_t* coll_list = reinterpret_cast<int32_t*>(w + L.coll_list);
-  int32_t* list2 = reinterpret_cast<int32_t*>(w + L.list2);
-  int32_t* rep2 = reinterpret_cast<int32_t*>(w + L.rep2);
-  int32_t* list3 = reinterpret_cast<int32_t*>(w + L.list3);
+  const int sms = num_sms();
   cudaError_t e = cudaMemsetAsync(w, 0, L.zero_end, stream);
   if (e != cudaSuccess) return cuda_fail(e, "workspace clear");
   e = cudaMemsetAsync(w + L.zero_end, 0xff, L.ones_end - L.zero_end, stream);
-  if (e != cudaSuccess) return cuda_fail(e, "table clear");
-  const uint64_t mask = g_merge_key_mask.load();
-  const int64_t row_tiles = (n + kMrTile - 1) / kMrTile;
-  const unsigned grid = grid_for(row_tiles, kMrH, num_sms());
-  launch_pdl(merge_rows_kernel, dim3(grid), dim3(kMrThreads), kMrSmem, stream, tokens, n, stride,
-             lens, seed, mask, fp_out, keys, idx, L.log2T, parent, coll_list, ctr, err);
-  launch_pdl(merge_resolve_kernel<true>, dim3(1), dim3(kResolveThreads), 0, stream,
-             (const uint64_t*)fp_out, mask, tokens, stride, lens, parent, (const int32_t*)coll_list,
-             (const uint32_t*)ctr, keys, idx, L.log2T, list2, rep2, list3, err);
+  if (e != cudaSuccess) return cuda_fail(e, "hash table clear");
+  bool ran = false;
+  hs_status st = launch_fingerprint_chunks(tokens, n, stride, lens, seed, fp_out, &ran, stream);
+  if (st != HS_OK) return st;
+  launch_pdl(tails_insert_kernel, dim3(grid_for(n, 256, sms * 16)), dim3(256), 0, stream, tokens,
+             n, stride, lens, seed, ran, mask, fp_out, keys, idx, L.log2T, err);
+  launch_pdl(verify_flat_kernel, dim3(grid_for(n, kVerifyThreads, sms * 8)), dim3(kVerifyThreads),
+             0, stream, (const uint64_t*)fp_out, mask, n, (const uint64_t*)keys,
+             (const uint32_t*)idx, L.log2T, tokens, stride, lens, rep, coll_list, ctr, err);
+  launch_pdl(resolve_kernel<true>, dim3(1), dim3(kResolveThreads), 0, stream,
+             (const uint64_t*)fp_out, tokens, stride, lens, rep, (const int32_t*)coll_list,
+             (const uint32_t*)ctr, keys, idx, uid, err);
   const int64_t tiles = (n + kScanTile - 1) / kScanTile;
-  launch_pdl(scan_kernel<true>, dim3((unsigned)tiles), dim3(kScanThreads), 0, stream,
-             (const int32_t*)parent, n, uid, status, ctr, n_unique_dev, err,
+  launch_pdl(scan_kernel, dim3((unsigned)tiles), dim3(kScanThreads), 0, stream,
+             (const int32_t*)rep, n, uid, status, ctr, n_unique_dev, err,
              g_scan_wait_limit_ns.load(), g_scan_withhold_tile.load());
-  launch_pdl(finalize_kernel<true>, dim3(grid_for(n, 256, num_sms() * 8)), dim3(256), 0, stream,
-             (const int32_t*)parent, (const int32_t*)uid, n, (const int32_t*)n_unique_dev,
+  launch_pdl(finalize_kernel, dim3(grid_for(n, 256, sms * 8)), dim3(256), 0, stream,
+             (const int32_t*)rep, (const int32_t*)uid, n, (const int32_t*)n_unique_dev,
              unique_idx, inverse);
-  count_launches(4);  // merge, resolve, scan, finalize
+  count_launches(5);  // tails+insert, verify, resolve, scan, finalize (the chunk launcher
+                      // counts its own)
   return cuda_fail(cudaGetLastError(), "merge_rows launch");
 }
 

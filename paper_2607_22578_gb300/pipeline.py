@@ -1,12 +1,13 @@
 """The whole embed-and-retrieve stage for one batch of concurrent workflows.
 
 Composition of the C-ABI calls only (no arithmetic here):
-  chunks:  hs_fingerprint -> hs_unique_inverse      (merge duplicate chunk nodes)
+  chunks:  hs_merge_rows                            (fingerprint + merge of duplicate
+                                                     chunk nodes)
   queries: hs_merge_queries                         (merge duplicate query nodes,
              (batches up to HS_MERGE_QUERIES_MAX;    Section 3.3 (I): fingerprint,
-              larger ones: hs_fingerprint ->          unique and gather in one
-              hs_unique_inverse ->                    launch)
-              hs_scatter_results gathering the unique rows)
+              larger ones: hs_merge_rows ->           unique and gather in one
+              hs_scatter_results gathering the        launch)
+              unique rows)
            -> hs_retrieve_topk_fanout               (one retrieval per merged node,
                                                      results written to every
                                                      originating query)
@@ -43,10 +44,10 @@ class EmbedRetrieveStage:
         self.max_queries = int(max_queries)
         mq, mc = self.max_queries, max(int(max_chunk_rows), 1)
         i32 = dict(dtype=torch.int32, device=dev)
-        self.ws_q = torch.empty(_lib.hs_unique_inverse_workspace(mq), dtype=torch.uint8, device=dev)
+        self.ws_q = torch.empty(_lib.hs_merge_rows_workspace(mq), dtype=torch.uint8, device=dev)
         self.ws_r = torch.empty(_lib.hs_retrieve_topk_workspace(mq, self.N, self.d, k),
                                 dtype=torch.uint8, device=dev)
-        self.ws_c = torch.empty(_lib.hs_unique_inverse_workspace(mc), dtype=torch.uint8, device=dev)
+        self.ws_c = torch.empty(_lib.hs_merge_rows_workspace(mc), dtype=torch.uint8, device=dev)
         self.q_out = (torch.empty(1, **i32), torch.empty(mq, **i32), torch.empty(mq, **i32))
         self.c_out = (torch.empty(1, **i32), torch.empty(mc, **i32), torch.empty(mc, **i32))
         self.q_fp = torch.empty(mq, dtype=torch.int64, device=dev)
@@ -88,9 +89,9 @@ class EmbedRetrieveStage:
         """Fingerprint + exact unique of chunk rows.  Returns (n_unique_dev,
         unique_idx, inverse, fp) as device tensors."""
         n = tokens.shape[0]
-        fp = _lib.hs_fingerprint(tokens, lens, fp_out=self.c_fp[:n])
-        nu, uidx, inv = _lib.hs_unique_inverse(fp, tokens, lens, workspace=self.ws_c,
-                                               out=self.c_out)
+        nu_b, uidx_b, inv_b = self.c_out
+        fp, nu, uidx, inv = _lib.hs_merge_rows(
+            tokens, lens, workspace=self.ws_c, out=(self.c_fp[:n], nu_b, uidx_b[:n], inv_b[:n]))
         return nu, uidx, inv, fp
 
     def retrieve(self, queries: torch.Tensor, events: tuple | None = None):
@@ -161,8 +162,8 @@ class EmbedRetrieveStage:
                 queries, out=(self.q_fp[:Q], nu_b, uidx_b[:Q], inv_b[:Q], self.uq[:Q]))
             return nu, inv, uq
         qi32 = queries.view(torch.int32)
-        fp = _lib.hs_fingerprint(qi32, fp_out=self.q_fp[:Q])
-        nu, uidx, inv = _lib.hs_unique_inverse(fp, qi32, workspace=self.ws_q, out=self.q_out)
+        _, nu, uidx, inv = _lib.hs_merge_rows(
+            qi32, workspace=self.ws_q, out=(self.q_fp[:Q], nu_b, uidx_b[:Q], inv_b[:Q]))
         uq = _lib.hs_scatter_results(queries, uidx, dst=self.uq[:Q])
         return nu, inv, uq
 
