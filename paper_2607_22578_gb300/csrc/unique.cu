@@ -937,7 +937,8 @@ hs_status launch_merge_rows(const int32_t* tokens, int64_t n, int32_t stride, co
   e = cudaMemsetAsync(w + L.zero_end, 0xff, L.ones_end - L.zero_end, stream);
   if (e != cudaSuccess) return cuda_fail(e, "hash table clear");
   bool ran = false;
-  hs_status st = launch_fingerprint_chunks(tokens, n, stride, lens, seed, fp_out, &ran, stream);
+  const hs_status st =
+      launch_fingerprint_chunks(tokens, n, stride, lens, seed, fp_out, &ran, stream);
   if (st != HS_OK) return st;
   launch_pdl(tails_insert_kernel, dim3(grid_for(n, 256, sms * 16)), dim3(256), 0, stream, tokens,
              n, stride, lens, seed, ran, mask, fp_out, keys, idx, L.log2T, err);
