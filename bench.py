@@ -403,7 +403,8 @@ def gpu_arm(args, rank: int, local_rank: int, world: int) -> int:
 
     # The other workloads' figures, measured in the same process after the
     # headline (rank 0): the dedup-heavy merge (fingerprint, unique/inverse,
-    # scatter against HBM) and batch-sweep latencies.
+    # scatter against HBM), batch-sweep latencies and the large-corpus
+    # retrieval (k = 100).
     extras = {}
     if rank == 0 and not args.no_extras:
         del graph, feed, stage, corpus, tokens, queries, h_tokens, h_queries
@@ -412,6 +413,9 @@ def gpu_arm(args, rank: int, local_rank: int, world: int) -> int:
         torch.cuda.empty_cache()
         extras["dedup_heavy"] = row_dedup_heavy(args, dev, peaks)
         extras["batch_sweep"] = row_batch_sweep(args, dev, peaks, batches=(1, 64, 512))
+        torch.cuda.empty_cache()
+        extras["large_corpus"] = row_large_corpus(args, dev, peaks)
+        gc.collect()
         torch.cuda.empty_cache()
 
     if rank == 0:
@@ -754,8 +758,8 @@ def row_large_corpus(args, dev, peaks) -> dict:
         cfg["N"] = args.corpus_rows
     w = configs.build_large_corpus(cfg, seed=args.seed)
     corpus, queries = _dev_array(w["corpus"], dev), _dev_array(w["queries"], dev)
-    N, d = w["corpus"].shape
-    Q, k = w["queries"].shape[0], w["k"]
+    N, d = corpus.shape
+    Q, k = queries.shape[0], w["k"]
     del w
     ws = torch.empty(hs.hs_retrieve_topk_workspace(Q, N, d, k), dtype=torch.uint8, device=dev)
     outs = (torch.empty((Q, k), dtype=torch.float32, device=dev),

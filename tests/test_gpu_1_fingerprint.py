@@ -138,3 +138,24 @@ def test_chunk_paths_mixed_tokens(stride, offset):
     out = hs.hs_fingerprint(t, to_dev(lens))
     hs.hs_get_device_error()
     assert (fp_host(out) == oracle.fingerprint(tok, lens)).all()
+
+
+@pytest.mark.parametrize("pattern", [0, 1, 2])
+def test_stream_rows_diagnostic_reads_exactly_the_valid_prefixes(pattern):
+    """hs_debug_stream_rows (the read-ceiling diagnostic) folds the tokens it
+    reads into an xor checksum: the valid prefixes for patterns 0 and 1,
+    the whole padded rows for pattern 2."""
+    rng = np.random.default_rng(pattern)
+    n, stride = 3001, 72
+    tokens = rng.integers(-2**31, 2**31 - 1, size=(n, stride), dtype=np.int64).astype(np.int32)
+    lens = rng.integers(0, stride + 1, size=n).astype(np.int32)
+    ck = torch.zeros(1, dtype=torch.int32, device="cuda")
+    hs.hs_debug_stream_rows(to_dev(tokens), to_dev(lens), pattern, ck, 2)
+    torch.cuda.synchronize()
+    u = tokens.view(np.uint32)
+    if pattern == 2:
+        want = np.bitwise_xor.reduce(u.reshape(-1))
+    else:
+        mask = np.arange(stride)[None, :] < lens[:, None]
+        want = np.bitwise_xor.reduce(np.where(mask, u, 0).reshape(-1))
+    assert int(ck.cpu().numpy().view(np.uint32)[0]) == int(want)
