@@ -537,12 +537,13 @@ __global__ void __launch_bounds__(256) finalize_kernel(const int32_t* __restrict
 // takes every 32nd piece pair, kVerifyPieces of them in flight per round,
 // so a warp's rows cost about (their bytes / 4 KB) round trips whatever
 // their lengths.  The tokens of a pair's last piece past its length are
-// masked.  Needs 16-byte aligned rows (stride % 4 == 0).
+// masked.  Needs 16-byte aligned rows (stride % 4 == 0).  Verifies rows
+// [row0, row_end) of n (row indices, the table and rep are global).
 constexpr int kVerifyPieces = 4;
 constexpr int kVerifyThreads = 256;
 
 __global__ void __launch_bounds__(kVerifyThreads) verify_flat_kernel(
-    const uint64_t* __restrict__ fp, uint64_t key_mask, int64_t n,
+    const uint64_t* __restrict__ fp, uint64_t key_mask, int64_t n, int64_t row0, int64_t row_end,
     const uint64_t* __restrict__ keys, const uint32_t* __restrict__ idx, int log2T,
     const int32_t* __restrict__ tokens, int32_t stride, const int32_t* __restrict__ lens,
     int32_t* __restrict__ rep, int32_t* coll_list, uint32_t* ctr, unsigned* err) {
@@ -555,9 +556,9 @@ __global__ void __launch_bounds__(kVerifyThreads) verify_flat_kernel(
   const int lane = threadIdx.x & 31, wl = threadIdx.x >> 5;
   const int64_t warps = ((int64_t)gridDim.x * blockDim.x) >> 5;
   const int64_t w = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  for (int64_t p0 = w * 32; p0 < n; p0 += warps * 32) {
+  for (int64_t p0 = row0 + w * 32; p0 < row_end; p0 += warps * 32) {
     const int64_t a = p0 + lane;
-    const bool valid = a < n;
+    const bool valid = a < row_end;
     int64_t r = a;
     int32_t la = 0, lr = 0;
     if (valid) {
@@ -624,18 +625,19 @@ __global__ void __launch_bounds__(kVerifyThreads) verify_flat_kernel(
 // and offers (fp & key_mask, row) to the table in the same pass: rows of a
 // warp with equal keys are combined and the smallest index inserts
 // (atomicMin), as insert_kernel does.  An invalid length sets the error
-// word and a zero fingerprint, as hs_fingerprint does.
+// word and a zero fingerprint, as hs_fingerprint does.  Rows [row0,
+// row_end); row0 is a multiple of 32 (warps combine their rows' inserts).
 __global__ void __launch_bounds__(256) tails_insert_kernel(
-    const int32_t* __restrict__ tokens, int64_t n, int32_t stride,
+    const int32_t* __restrict__ tokens, int64_t row0, int64_t row_end, int32_t stride,
     const int32_t* __restrict__ lens, uint64_t seed, bool chunks_ran, uint64_t key_mask,
     uint64_t* __restrict__ fp_out, uint64_t* keys, uint32_t* idx, int log2T, unsigned* err) {
   pdl_wait();
   pdl_trigger();
   constexpr int T = 32;
-  for (int64_t base = (int64_t)blockIdx.x * blockDim.x; base < n;
+  for (int64_t base = row0 + (int64_t)blockIdx.x * blockDim.x; base < row_end;
        base += (int64_t)gridDim.x * blockDim.x) {
     const int64_t r = base + threadIdx.x;
-    const bool valid = r < n;
+    const bool valid = r < row_end;
     uint64_t f = 0;
     if (valid) {
       const int32_t L = lens ? __ldg(lens + r) : stride;
@@ -875,8 +877,8 @@ hs_status launch_unique_inverse(const uint64_t* fp, const int32_t* tokens, int64
   const unsigned vgrid = grid_for(n, 256, sms * 8);   // one warp per 32 rows
   if (vec)
     launch_pdl(verify_flat_kernel, dim3(vgrid), dim3(kVerifyThreads), 0, stream, fp, ~0ull, n,
-               (const uint64_t*)keys, (const uint32_t*)idx, L.log2T, tokens, stride, lens, rep,
-               coll_list, ctr, err);
+               (int64_t)0, n, (const uint64_t*)keys, (const uint32_t*)idx, L.log2T, tokens,
+               stride, lens, rep, coll_list, ctr, err);
   else
     launch_pdl(verify_kernel<false>, dim3(vgrid), dim3(256), 0, stream, fp, n, keys, idx, L.log2T,
                tokens, stride, lens, rep, coll_list, ctr, err);
@@ -941,9 +943,9 @@ hs_status launch_merge_rows(const int32_t* tokens, int64_t n, int32_t stride, co
       launch_fingerprint_chunks(tokens, n, stride, lens, seed, fp_out, &ran, stream);
   if (st != HS_OK) return st;
   launch_pdl(tails_insert_kernel, dim3(grid_for(n, 256, sms * 16)), dim3(256), 0, stream, tokens,
-             n, stride, lens, seed, ran, mask, fp_out, keys, idx, L.log2T, err);
+             (int64_t)0, n, stride, lens, seed, ran, mask, fp_out, keys, idx, L.log2T, err);
   launch_pdl(verify_flat_kernel, dim3(grid_for(n, kVerifyThreads, sms * 8)), dim3(kVerifyThreads),
-             0, stream, (const uint64_t*)fp_out, mask, n, (const uint64_t*)keys,
+             0, stream, (const uint64_t*)fp_out, mask, n, (int64_t)0, n, (const uint64_t*)keys,
              (const uint32_t*)idx, L.log2T, tokens, stride, lens, rep, coll_list, ctr, err);
   launch_pdl(resolve_kernel<true>, dim3(1), dim3(kResolveThreads), 0, stream,
              (const uint64_t*)fp_out, tokens, stride, lens, rep, (const int32_t*)coll_list,
