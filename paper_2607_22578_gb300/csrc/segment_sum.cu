@@ -3,23 +3,22 @@
 // merged into v*.  With the inverse map of the merge, that is a segmented
 // sum: out[u] = sum of phi[i] over the rows i with inverse[i] = u.
 //
-// Groups are arbitrary (a hot row's copies are scattered over the batch), and
-// the hot groups of a Zipf-like merge would serialise any scheme that adds
-// every row, or every warp's partial sum, to the output: the L2 processes
-// updates of one line one at a time.  So the sum is taken in three levels:
-//   1. each warp sums 4 rounds of 32 rows into its own shared-memory table
-//      keyed by group ordinal; within a round, rows of one group are first
-//      combined with shuffles (pairwise trees), so the keys of a round are
-//      distinct and plain adds suffice;
-//   2. a group met once in a warp's tile is added to the output at once (a
-//      cold group: one global fp64 atomic); the groups met more than once
-//      (the hot ones) are merged over the CTA's warps into a CTA table, and
-//      so are the groups with ordinals below 4096: ordinals follow first
+// Groups are arbitrary (a hot row's copies are scattered over the batch).
+// Adding every row to the output with a global atomic would serialise the
+// hot groups in the L2, and a shared-memory hash table per tile costs more
+// than the atomics it saves for the cold groups.  So each CTA sorts its
+// rows into three paths:
+//   1. per round of 32 rows, the lanes of one group are combined with
+//      shuffles (pairwise trees), leaving one partial sum per distinct group;
+//   2. a group with ordinal below kSsDense goes to a dense per-CTA array in
+//      shared memory (fp64 shared atomics).  Ordinals follow first
 //      occurrence, so the frequent groups of a batch mostly have small
-//      ordinals and share the first output lines, which every CTA would
-//      otherwise update;
-//   3. each group of the CTA table takes one global fp64 atomic, so a hot
-//      group costs one update per CTA tile of 1024 rows.
+//      ordinals; the array is added to the output once per CTA, a warp's
+//      32 consecutive ordinals per instruction, zeros skipped;
+//   3. a larger ordinal that occurs more than once in its round (a hot group
+//      that appeared late) claims a slot of a per-CTA hash table (bounded
+//      probing; a full table sends the sum straight to the output), flushed
+//      once per CTA; every other partial sum is one global fp64 atomic.
 // The output is cleared with a memset first.  Additions run in fp64 in no
 // fixed order: for a group of m rows the result is within
 // ((m-1) u / (1 - (m-1) u)) * sum |phi| of the exact sum (u = 2^-53), and
@@ -31,20 +30,13 @@ namespace {
 
 constexpr int kSsThreads = 256;
 constexpr int kSsWarps = kSsThreads / 32;
-constexpr int kSsRounds = 4;                             // warp-rounds per warp tile
+constexpr int kSsRounds = 4;                             // rounds of 32 rows per warp tile
 constexpr int kSsTile = 32 * kSsRounds;                  // rows per warp tile
 constexpr int kSsCtaRows = kSsWarps * kSsTile;           // rows per CTA tile
-constexpr int kSsLog2Slots = 8;
-constexpr int kSsSlots = 1 << kSsLog2Slots;              // slots of a warp table
-constexpr int kSsLog2CtaSlots = kSsLog2Slots + 3;
-constexpr int kSsLowIds = 4096;                          // ordinals always merged per CTA
-constexpr int kSsCtaSlots = 1 << kSsLog2CtaSlots;        // slots of the CTA table
-constexpr size_t kSsSmem = (size_t)(kSsWarps * kSsSlots + kSsCtaSlots) *
-                               (sizeof(double) + sizeof(int32_t)) +
-                           (size_t)kSsWarps * kSsSlots * sizeof(int32_t);
-static_assert(kSsSlots >= 2 * kSsTile && kSsCtaSlots >= 2 * kSsCtaRows,
-              "tables at least twice the rows they hold");
-static_assert(kSsSmem <= 232448, "the warp and CTA tables fit one CTA's shared memory");
+constexpr int kSsDense = 256;                            // ordinals summed densely per CTA
+constexpr int kSsLog2Slots = 9;
+constexpr int kSsSlots = 1 << kSsLog2Slots;              // hash slots for repeated large ordinals
+constexpr int kSsProbes = 32;                            // probes before going to the output
 
 __device__ __forceinline__ uint32_t ss_slot(int32_t g, int log2_slots) {
   return ((uint32_t)g * 0x9E3779B1u) >> (32 - log2_slots);
@@ -70,18 +62,17 @@ __device__ __forceinline__ double sum_peers(unsigned peers, double x, int lane) 
   return x;
 }
 
-// Slot of group g in a table of 2^log2 slots, claimed if new (a free slot
-// always exists: the table has at least twice as many slots as keys).
-__device__ __forceinline__ uint32_t claim_slot(int32_t* keys, int32_t g, int log2) {
-  const uint32_t mask = (1u << log2) - 1u;
-  uint32_t s = ss_slot(g, log2);
+// Slot of group g in the hash table, claimed if new, or -1 when kSsProbes
+// slots in a row hold other groups.
+__device__ __forceinline__ int claim_slot(int32_t* keys, int32_t g) {
+  uint32_t s = ss_slot(g, kSsLog2Slots);
 #pragma unroll 1
-  for (uint32_t probe = 0; probe <= mask; ++probe) {
+  for (int probe = 0; probe < kSsProbes; ++probe) {
     const int32_t k = atomicCAS(keys + s, -1, g);
-    if (k == -1 || k == g) return s;
-    s = (s + 1u) & mask;
+    if (k == -1 || k == g) return (int)s;
+    s = (s + 1u) & (kSsSlots - 1u);
   }
-  return s;   // not reached
+  return -1;
 }
 
 __global__ void __launch_bounds__(kSsThreads) segment_sum_kernel(
@@ -90,18 +81,22 @@ __global__ void __launch_bounds__(kSsThreads) segment_sum_kernel(
     unsigned* err) {
   pdl_wait();
   pdl_trigger();
-  extern __shared__ __align__(16) uint8_t sm[];
+  __shared__ double dense[kSsDense];
+  __shared__ double hsum[kSsSlots];
+  __shared__ int32_t hkey[kSsSlots];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  double* cta_sums = reinterpret_cast<double*>(sm);
-  double* sums = cta_sums + kSsCtaSlots + warp * kSsSlots;
-  int32_t* cta_keys = reinterpret_cast<int32_t*>(cta_sums + kSsCtaSlots + kSsWarps * kSsSlots);
-  int32_t* keys = cta_keys + kSsCtaSlots + warp * kSsSlots;
-  int32_t* rows = cta_keys + kSsCtaSlots + kSsWarps * kSsSlots + warp * kSsSlots;
   int64_t count = max_groups;
   if (count_dev) {
     const int64_t c = __ldg(count_dev);
     count = c < 0 ? 0 : (c > max_groups ? max_groups : c);
   }
+  const int32_t H = (int32_t)(count < kSsDense ? count : kSsDense);
+  for (int s = tid; s < H; s += kSsThreads) dense[s] = 0.0;
+  for (int s = tid; s < kSsSlots; s += kSsThreads) {
+    hkey[s] = -1;
+    hsum[s] = 0.0;
+  }
+  __syncthreads();
   const int64_t tiles = (n + kSsCtaRows - 1) / kSsCtaRows;
   for (int64_t t = blockIdx.x; t < tiles; t += gridDim.x) {
     const int64_t r0 = t * kSsCtaRows + (int64_t)warp * kSsTile;
@@ -121,53 +116,33 @@ __global__ void __launch_bounds__(kSsThreads) segment_sum_kernel(
         }
       }
     }
-    for (int s = tid; s < kSsCtaSlots; s += kSsThreads) {
-      cta_keys[s] = -1;
-      cta_sums[s] = 0.0;
-    }
-#pragma unroll
-    for (int j = 0; j < kSsSlots / 32; ++j) {
-      keys[j * 32 + lane] = -1;
-      sums[j * 32 + lane] = 0.0;
-      rows[j * 32 + lane] = 0;
-    }
-    __syncwarp();
-    // 1. this warp's rows into its own table: per round, the first lane of
-    //    each distinct group adds the group's round sum (keys of a round are
-    //    distinct, rounds are ordered by warp barriers: plain adds suffice)
 #pragma unroll
     for (int j = 0; j < kSsRounds; ++j) {
       const unsigned peers = __match_any_sync(0xffffffffu, g[j]);
       const double x = sum_peers(peers, v[j], lane);
       if (g[j] >= 0 && lane == __ffs(peers) - 1) {
-        const uint32_t s = claim_slot(keys, g[j], kSsLog2Slots);
-        sums[s] += x;
-        rows[s] += __popc(peers);
-      }
-      __syncwarp();
-    }
-    __syncthreads();
-    // 2. groups seen more than once in a warp tile, and groups with small
-    //    ordinals, are merged into the CTA table (a group meets at most one
-    //    entry per warp table: shared fp64 atomics with little contention);
-    //    the rest go straight to the output
-#pragma unroll 1
-    for (int j = 0; j < kSsSlots / 32; ++j) {
-      const int32_t k = keys[j * 32 + lane];
-      if (k >= 0) {
-        if (rows[j * 32 + lane] > 1 || k < kSsLowIds)
-          atomicAdd(cta_sums + claim_slot(cta_keys, k, kSsLog2CtaSlots), sums[j * 32 + lane]);
-        else
-          atomicAdd(out + k, sums[j * 32 + lane]);
+        if (g[j] < H) {
+          atomicAdd(dense + g[j], x);
+        } else {
+          const int s = peers != (1u << lane) ? claim_slot(hkey, g[j]) : -1;
+          if (s >= 0)
+            atomicAdd(hsum + s, x);
+          else
+            atomicAdd(out + g[j], x);
+        }
       }
     }
-    __syncthreads();
-    // 3. one global fp64 atomic per distinct group of the CTA tile
-    for (int s = tid; s < kSsCtaSlots; s += kSsThreads) {
-      const int32_t k = cta_keys[s];
-      if (k >= 0) atomicAdd(out + k, cta_sums[s]);
-    }
-    __syncthreads();
+  }
+  __syncthreads();
+  // Adding a zero changes no output (the output starts at +0), so zero
+  // entries are skipped.
+  for (int s = tid; s < H; s += kSsThreads) {
+    const double x = dense[s];
+    if (x != 0.0) atomicAdd(out + s, x);
+  }
+  for (int s = tid; s < kSsSlots; s += kSsThreads) {
+    const int32_t k = hkey[s];
+    if (k >= 0) atomicAdd(out + k, hsum[s]);
   }
 }
 
@@ -183,18 +158,10 @@ hs_status launch_segment_sum(const double* phi, const int32_t* inverse, int64_t 
     if (e != cudaSuccess) return cuda_fail(e, "output clear");
   }
   if (n == 0) return HS_OK;
-  static std::atomic<uint64_t> configured{0};
-  const hs_status cst = once_per_device(configured, [] {
-    return cuda_fail(cudaFuncSetAttribute(segment_sum_kernel,
-                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                          (int)kSsSmem),
-                     "segment sum smem attribute");
-  });
-  if (cst != HS_OK) return cst;
   const int64_t blocks = (n + kSsCtaRows - 1) / kSsCtaRows;
   const int64_t cap = (int64_t)num_sms() * 4;
   const unsigned grid = (unsigned)(blocks < cap ? blocks : cap);
-  launch_pdl(segment_sum_kernel, dim3(grid), dim3(kSsThreads), kSsSmem, stream, phi, inverse, n,
+  launch_pdl(segment_sum_kernel, dim3(grid), dim3(kSsThreads), 0, stream, phi, inverse, n,
              count_dev, max_groups, out, err);
   count_launches(1);
   return cuda_fail(cudaGetLastError(), "segment sum launch");

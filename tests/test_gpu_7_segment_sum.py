@@ -107,10 +107,15 @@ def test_count_and_bad_entries():
     assert gpu_sum(np.zeros(0), np.zeros(0, np.int32), 4).tolist() == [0, 0, 0, 0]
 
 
-@pytest.mark.parametrize("pattern", ["hot_high_ordinals", "cold_uniform", "identity"])
+@pytest.mark.parametrize("pattern", ["hot_high_ordinals", "cold_uniform", "identity",
+                                     "late_hot", "adjacent_pairs", "dense_only"])
 def test_group_patterns_exact(pattern):
-    """Hot groups with large ordinals (merged per CTA), cold groups spread
-    over many ordinals (added directly) and one row per group."""
+    """Hot groups with large ordinals (merged in the per-CTA hash table),
+    cold groups spread over many ordinals (added directly), one row per
+    group, a hot group first seen after 10,000 others, pairs of adjacent
+    rows (512 repeated groups per 1024-row tile: the hash table fills and
+    the bounded probing sends the rest to the output), and every ordinal
+    below the dense array's 256."""
     n = 300_000
     rng = np.random.default_rng(9)
     if pattern == "hot_high_ordinals":
@@ -119,6 +124,17 @@ def test_group_patterns_exact(pattern):
     elif pattern == "cold_uniform":
         inv = rng.integers(0, 200_000, size=n).astype(np.int32)
         G = 200_000
+    elif pattern == "late_hot":
+        inv = (np.arange(n) % 10_000).astype(np.int32)
+        inv[10_000:] = np.where(rng.random(n - 10_000) < 0.5, 5_000,
+                                rng.integers(0, 10_000, n - 10_000))
+        G = 10_000
+    elif pattern == "adjacent_pairs":
+        inv = (1_000 + np.arange(n) // 2).astype(np.int32)
+        G = 1_000 + n // 2
+    elif pattern == "dense_only":
+        inv = rng.integers(0, 256, size=n).astype(np.int32)
+        G = 256
     else:
         inv = rng.permutation(n).astype(np.int32)
         G = n
