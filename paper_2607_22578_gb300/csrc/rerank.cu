@@ -8,19 +8,25 @@
 // index ascending).
 //
 // One warp per output row.  The work is a gather of k1 corpus rows per
-// query — HBM-bound — so a warp keeps four candidate rows in flight at a
-// time (lane l reads 16-byte pieces l, l + 32, ... of each row) and reduces
-// the four partial dot products with shuffles.  Lane c then holds candidate
-// c's score; its rank is the number of candidates ahead of it in the order
+// query, and with a few thousand output rows every row is resident at once:
+// the kernel's time is the chain of dependent memory round trips of one row,
+// not bandwidth.  So the chain is kept short: the map entry, the candidate
+// ids, then per group of four candidates one round trip in which each lane
+// requests all of its 16-byte pieces (l, l + 32, l + 64, l + 96) of the
+// query row and the four candidate rows before the first product (d <= 1024;
+// longer rows take one round trip per 1024 dimensions).  The four partial
+// dot products are reduced with shuffles.  Lane c then holds candidate c's
+// score; its rank is the number of candidates ahead of it in the order
 // (ties between equal keys by lane), and the lanes of rank < k2 write their
-// entry.
+// entry.  CTAs of two warps spread the rows evenly over the SMs.
 #include "hs_internal.cuh"
 
 namespace hs {
 namespace {
 
-constexpr int kRrThreads = 256;
+constexpr int kRrThreads = 64;
 constexpr int kRrGroup = 4;                  // candidate rows in flight per warp
+constexpr int kRrPieces = 4;                 // 16-byte pieces per lane and row in flight
 
 __device__ __forceinline__ uint64_t rr_key(float s, int32_t id) {
   uint32_t u = __float_as_uint(s);
@@ -80,15 +86,28 @@ __global__ void __launch_bounds__(kRrThreads) rerank_kernel(
         if (c0 + g >= k1) cid[g] = -1;
         acc[g] = 0.0f;
       }
-      for (int v = lane; v < nv; v += 32) {
-        const uint4 a = __ldg(qrow + v);
-        uint4 b[kRrGroup];
+      // Every piece of the group's rows that this lane reads in a round of
+      // kRrPieces pieces is requested before the first product, so a round
+      // costs one memory round trip (one per group for d <= 1024).
+      for (int v0 = 0; v0 < nv; v0 += 32 * kRrPieces) {
+        uint4 a[kRrPieces], b[kRrGroup][kRrPieces];
 #pragma unroll
-        for (int g = 0; g < kRrGroup; ++g)
-          if (cid[g] >= 0) b[g] = __ldg(rc + (int64_t)cid[g] * nv + v);
+        for (int pc = 0; pc < kRrPieces; ++pc) {
+          const int v = v0 + pc * 32 + lane;
+          a[pc] = v < nv ? __ldg(qrow + v) : make_uint4(0u, 0u, 0u, 0u);
 #pragma unroll
-        for (int g = 0; g < kRrGroup; ++g)
-          if (cid[g] >= 0) acc[g] = dot8(a, b[g], acc[g]);
+          for (int g = 0; g < kRrGroup; ++g)
+            b[g][pc] = (cid[g] >= 0 && v < nv) ? __ldg(rc + (int64_t)cid[g] * nv + v)
+                                               : make_uint4(0u, 0u, 0u, 0u);
+        }
+#pragma unroll
+        for (int pc = 0; pc < kRrPieces; ++pc) {
+          if (v0 + pc * 32 + lane < nv) {
+#pragma unroll
+            for (int g = 0; g < kRrGroup; ++g)
+              if (cid[g] >= 0) acc[g] = dot8(a[pc], b[g][pc], acc[g]);
+          }
+        }
       }
 #pragma unroll
       for (int g = 0; g < kRrGroup; ++g) {
