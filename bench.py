@@ -593,6 +593,21 @@ def row_dedup_heavy(args, dev, peaks) -> dict:
     hs.hs_get_device_error()
     assert int(outs[0].item()) == n_u
     t_all = e0.elapsed_time(e1) / K
+    cpu = None
+    if not getattr(args, "no_cpu_baseline", False):
+        # The oracle on the whole workload (a few seconds on one host core):
+        # fingerprint, unique/inverse and the scatter of the 1536-byte rows.
+        import oracle
+        host_payload = payload.cpu().numpy()
+        t0 = time.perf_counter()
+        oracle.fingerprint(w["tokens"], w["lens"])
+        _, oinv = oracle.unique_inverse(w["tokens"], w["lens"])
+        oracle.scatter(host_payload, oinv)
+        t_cpu = time.perf_counter() - t0
+        cpu = {"value": n / t_cpu, "unit": "dedup rows/s", "cores": 1, "kind": "oracle",
+               "cpu": cpu_model(),
+               "sample": "all %d rows, measured: fingerprint + unique/inverse + scatter of "
+                         "%d B rows, one host thread, %.2f s" % (n, W, t_cpu)}
     L = w["lens"].astype(np.int64)
     sizes = np.bincount(gi, minlength=n_u)
     multi = sizes[gi] > 1
@@ -628,7 +643,8 @@ def row_dedup_heavy(args, dev, peaks) -> dict:
                       "re-read of every row in a group of size >= 2 + fp in + unique_idx/inverse "
                       "out (sort scratch is L2-resident and not counted); scatter: unique rows "
                       "once + every destination row + map",
-        "token_bytes_one_pass": tok_bytes}
+        "token_bytes_one_pass": tok_bytes,
+        "cpu_baseline": cpu}
 
 
 def row_read_ceiling(args, dev, peaks) -> dict:
