@@ -75,6 +75,9 @@ def test_tiny_config():
     (17, 3000, 256, 100),     # candidate-buffer path
     (5, 2000, 64, 33),        # smallest buffered k
     (40, 20000, 128, 1024),   # HS_TOPK_MAX_K
+    (600, 100, 64, 12),       # CTA pairs, N < 128: the odd CTA's corpus half is past N
+    (417, 3000, 1024, 32),    # CTA pairs over two query-block groups, k = 32, d = 1024
+    (1000, 4096, 128, 16),    # four query-block groups, ragged last block
 ])
 def test_shapes(nq, N, d, k):
     Q, C = unit_pair(nq, N, d, nq * 7 + N)
