@@ -739,7 +739,11 @@ constexpr int kMaxListsPerLane = 10;
 // Any kout: picks 0..31 are kept one per lane and written together when
 // kout <= 32; for larger kout each pick is written as it is made.  With
 // out_i NULL only the kout-th pick's score is written, to out_s[o].  `only`
-// and `flag_out` are as for merge_kernel.
+// and `flag_out` are as for merge_kernel.  LPL lists per lane at most (the
+// launch's bound on 2 * nsplit / 32, rounded up); slots past the query's
+// list count are skipped warp-uniformly, so the per-round work and the
+// registers follow the lists a launch can have, not the largest count.
+template <int LPL>
 __global__ void __launch_bounds__(256) merge_warp_kernel(const Params p, float* __restrict__ out_s,
                                                          int32_t* __restrict__ out_i,
                                                          int32_t kout, OutRows rows,
@@ -762,14 +766,17 @@ __global__ void __launch_bounds__(256) merge_warp_kernel(const Params p, float* 
     if (only && only[q / BM] == 0u) continue;      // warp-uniform
     const float* __restrict__ ps = p.part_s + (size_t)q * lists * k;
     const int32_t* __restrict__ pi = p.part_i + (size_t)q * lists * k;
-    uint64_t head[kMaxListsPerLane], next[kMaxListsPerLane];
-    int pos[kMaxListsPerLane];
+    uint64_t head[LPL], next[LPL];
+    int pos[LPL];
 #pragma unroll
-    for (int j = 0; j < kMaxListsPerLane; ++j) {
+    for (int j = 0; j < LPL; ++j) {
       const int l = j * 32 + lane;
       pos[j] = 0;
-      head[j] = l < lists ? pack_key(ps[(size_t)l * k], pi[(size_t)l * k]) : 0ull;
-      next[j] = (l < lists && k > 1) ? pack_key(ps[(size_t)l * k + 1], pi[(size_t)l * k + 1]) : 0ull;
+      head[j] = next[j] = 0ull;
+      if (j * 32 < lists) {                        // warp-uniform
+        if (l < lists) head[j] = pack_key(ps[(size_t)l * k], pi[(size_t)l * k]);
+        if (l < lists && k > 1) next[j] = pack_key(ps[(size_t)l * k + 1], pi[(size_t)l * k + 1]);
+      }
     }
     float my_s = -FLT_MAX;
     int32_t my_i = -1;
@@ -778,17 +785,17 @@ __global__ void __launch_bounds__(256) merge_warp_kernel(const Params p, float* 
       uint64_t best = 0ull;
       int bj = 0;
 #pragma unroll
-      for (int j = 0; j < kMaxListsPerLane; ++j)
-        if (head[j] > best) {
+      for (int j = 0; j < LPL; ++j)
+        if (j * 32 < lists && head[j] > best) {    // the first test is warp-uniform
           best = head[j];
           bj = j;
         }
-      uint64_t mx = best;
-#pragma unroll
-      for (int sh = 16; sh > 0; sh >>= 1) {
-        const uint64_t y = __shfl_xor_sync(0xffffffffu, mx, sh);
-        mx = y > mx ? y : mx;
-      }
+      // Warp maximum of the 64-bit keys: the largest high word, then the
+      // largest low word among the lanes holding it (two warp reductions).
+      const uint32_t bhi = (uint32_t)(best >> 32), blo = (uint32_t)best;
+      const uint32_t mhi = __reduce_max_sync(0xffffffffu, bhi);
+      const uint32_t mlo = __reduce_max_sync(0xffffffffu, bhi == mhi ? blo : 0u);
+      const uint64_t mx = ((uint64_t)mhi << 32) | mlo;
       const unsigned win = __ballot_sync(0xffffffffu, best == mx && mx != 0ull);
       last = mx;
       if (kout <= 32) {
@@ -802,7 +809,7 @@ __global__ void __launch_bounds__(256) merge_warp_kernel(const Params p, float* 
       }
       if (win != 0u && lane == __ffs(win) - 1) {
 #pragma unroll
-        for (int j = 0; j < kMaxListsPerLane; ++j)
+        for (int j = 0; j < LPL; ++j)
           if (j == bj) {
             const int l = j * 32 + lane;
             ++pos[j];
@@ -826,7 +833,7 @@ __global__ void __launch_bounds__(256) merge_warp_kernel(const Params p, float* 
     if (flag_out) {
       bool cut = false;
 #pragma unroll
-      for (int j = 0; j < kMaxListsPerLane; ++j) {
+      for (int j = 0; j < LPL; ++j) {
         const int l = j * 32 + lane;
         if (l < lists)
           cut |= pack_key(ps[(size_t)l * k + k - 1], pi[(size_t)l * k + k - 1]) >= last;
@@ -1371,8 +1378,21 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
     if (nr == 0) return HS_OK;
     if (2 * (int64_t)pm.slots <= 32 * kMaxListsPerLane) {
       const int64_t blocks = (nr + 7) / 8;          // one warp per row
-      launch_pdl(merge_warp_kernel, dim3((unsigned)(blocks < sms * 16 ? blocks : sms * 16)),
-                 dim3(256), 0, stream, pm, os, oi, kout, orows, flag_out, only);
+      const dim3 grid((unsigned)(blocks < sms * 16 ? blocks : sms * 16));
+      // lists per query <= 2 * slots (nsplit <= slots): lanes need that / 32
+      const int64_t lpl = (2 * (int64_t)pm.slots + 31) / 32;
+      if (lpl <= 2)
+        launch_pdl(merge_warp_kernel<2>, grid, dim3(256), 0, stream, pm, os, oi, kout, orows,
+                   flag_out, only);
+      else if (lpl <= 3)
+        launch_pdl(merge_warp_kernel<3>, grid, dim3(256), 0, stream, pm, os, oi, kout, orows,
+                   flag_out, only);
+      else if (lpl <= 5)
+        launch_pdl(merge_warp_kernel<5>, grid, dim3(256), 0, stream, pm, os, oi, kout, orows,
+                   flag_out, only);
+      else
+        launch_pdl(merge_warp_kernel<kMaxListsPerLane>, grid, dim3(256), 0, stream, pm, os, oi,
+                   kout, orows, flag_out, only);
       return cuda_fail(cudaGetLastError(), "merge launch");
     }
     const int64_t mgrid = nr < sms * 8 ? nr : sms * 8;
