@@ -78,6 +78,7 @@ def test_tiny_config():
     (600, 100, 64, 12),       # CTA pairs, N < 128: the odd CTA's corpus half is past N
     (417, 3000, 1024, 32),    # CTA pairs over two query-block groups, k = 32, d = 1024
     (1000, 4096, 128, 16),    # four query-block groups, ragged last block
+    (300, 30000, 128, 1024),  # CTA pairs at HS_TOPK_MAX_K: optimistic pass, flags, exact passes
 ])
 def test_shapes(nq, N, d, k):
     Q, C = unit_pair(nq, N, d, nq * 7 + N)
