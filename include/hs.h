@@ -541,6 +541,26 @@ hs_status hs_debug_scan_wait(uint64_t limit_ns, int64_t withhold_tile);
 hs_status hs_debug_merge_key_mask(uint64_t mask);
 
 /*
+ * hs_debug_retrieve_wait — test hook of the retrieval's bounded waits
+ * (failure detection); takes no part in the method.  The main retrieval
+ * kernel (launches with more than 16 addressable queries) gives up a
+ * pipeline wait (shared-memory stage, tensor-memory accumulator) after
+ * limit_ns, sets HS_ERR_TIMEOUT in the device error word and returns: before
+ * its CTA pair frees tensor memory, the even CTA waits (with the same
+ * limit) for every stage copy it armed and every MMA it issued.  With
+ * withhold_first = 1 every CTA skips the copies of its first stage, so that
+ * stage never fills and the waits run out; the outputs of such a call are
+ * unspecified (every write stays inside the outputs and the workspace).
+ *
+ * limit_ns        wait limit in ns, at most 2e9; 0 restores 2 s.
+ * withhold_first  0 or 1.
+ * Settings are process-wide and take effect at the next launch.
+ * Returns HS_ERR_INVALID_ARG for a limit above 2 s or withhold_first
+ * outside {0, 1}.
+ */
+hs_status hs_debug_retrieve_wait(uint64_t limit_ns, int32_t withhold_first);
+
+/*
  * hs_debug_stream_rows — diagnostics: stream the rows' valid prefixes with
  * no hashing, to measure what the row layout itself costs to read; takes no
  * part in the method.

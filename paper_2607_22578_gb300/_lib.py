@@ -105,6 +105,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
             lib.hs_merge_rows.restype = st
             lib.hs_debug_merge_key_mask.argtypes = [u64]
             lib.hs_debug_merge_key_mask.restype = st
+            lib.hs_debug_retrieve_wait.argtypes = [u64, i32]
+            lib.hs_debug_retrieve_wait.restype = st
             lib.hs_debug_stream_rows.argtypes = [P, i64, i32, P, i32, P, i32, P]
             lib.hs_debug_stream_rows.restype = st
             _lib = lib
@@ -220,6 +222,12 @@ def hs_debug_merge_key_mask(mask: int = 0) -> None:
     """Test hook of hs_merge_rows: key the table by fp & mask (0 restores
     all ones; see hs.h)."""
     _check(load().hs_debug_merge_key_mask(int(mask)))
+
+
+def hs_debug_retrieve_wait(limit_ns: int = 0, withhold_first: int = 0) -> None:
+    """Test hook of the retrieval's bounded waits: the wait limit (0: 2 s)
+    and whether every CTA withholds its first stage (see hs.h)."""
+    _check(load().hs_debug_retrieve_wait(int(limit_ns), int(withhold_first)))
 
 
 def hs_unique_inverse_noalloc(fp: torch.Tensor, tokens: torch.Tensor,

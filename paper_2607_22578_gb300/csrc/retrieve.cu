@@ -75,7 +75,7 @@ struct Ring {
   static constexpr size_t smem = 1024 + (size_t)stages * stage_bytes + kBarBytes + kEpiSmem;
 };
 static_assert(Ring<1>::smem <= 232448 && Ring<2>::smem <= 232448, "shared memory per CTA");
-static_assert(8 * (2 * Ring<2>::stages + 4) + 8 <= kBarBytes, "barrier area");
+static_assert(8 * (2 * Ring<2>::stages + 4) + 8 + 8 <= kBarBytes, "barrier area");
 
 struct Params {
   int64_t Qmax, N, tiles;
@@ -101,6 +101,11 @@ struct Params {
   // Optional, one word per query block: a unit whose query blocks are all 0
   // here is skipped (the exact large-k pass re-runs only the flagged blocks).
   const uint32_t* only;
+  // Bounded waits of retrieve_kernel: give up after wait_limit_ns.  With
+  // withhold_first set (a test hook) every CTA skips the loads of its first
+  // stage, so that stage never fills and the waits run out.
+  uint64_t wait_limit_ns;
+  int32_t withhold_first;
 };
 
 // Rows the merge writes: with inv NULL one per query (row q = query q);
@@ -328,7 +333,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* tempty = tfull + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  uint64_t* drain = tempty + 3;          // after tmem_slot and abort_flag: the MMA drain
   uint8_t* epi_smem = smem + kStages * kStageBytes + kBarBytes;
+  const uint64_t lim = p.wait_limit_ns ? p.wait_limit_ns : kWaitLimitNs;
 
   // CTA pair: the even CTA (rank 0) owns the full and tempty barriers that
   // both CTAs' loads and epilogues signal, and issues every MMA.
@@ -342,6 +349,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(tfull + a, 1);
       mbar_init(tempty + a, kEpiWarps * CL);
     }
+    mbar_init(drain, 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -380,6 +388,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint64_t pol_c = policy_evict_first();
       const uint64_t pol_q = policy_evict_last();
       uint32_t stage = 0, phase = 0;
+      int64_t issued = 0;                 // stages armed (or withheld) so far
       for (int64_t u = u0; u < units; u += ustep) {
         if (unit_skipped(p, sp, u, CL)) continue;
         int qb, split;
@@ -387,7 +396,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         unit_coords(sp, p.tiles, u, rank, CL, qb, split, t0, t1);
         for (int64_t t = t0; t < t1; ++t) {
           for (int kb = 0; kb < p.kb_count; ++kb) {
-            if (!mbar_wait(empty + stage, phase ^ 1u, abort_flag)) goto producer_done;
+            if (!mbar_wait_limit(empty + stage, phase ^ 1u, abort_flag, lim)) goto producer_done;
+            if (p.withhold_first && issued == 0) {   // test hook: this stage never fills
+              ++issued;
+              if (++stage == kStages) {
+                stage = 0;
+                phase ^= 1u;
+              }
+              continue;
+            }
+            ++issued;
             // A query block past the last addressable row is loaded from
             // row 0 instead: its scores are masked, and no box lies wholly
             // outside the tensor.
@@ -415,13 +433,28 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       }
-    producer_done:;
+    producer_done:
+      // Before it leaves, the even CTA (whose full barriers count both CTAs'
+      // bytes) waits, bounded, for every stage it armed that may still be in
+      // flight, so no copy lands in shared memory after the CTAs exit, even
+      // when some role gave up.  In a normal run these phases have completed
+      // or complete within the last tile.
+      if (rank == 0) {
+        volatile int keep_going = 0;
+        for (int64_t i = issued > kStages ? issued - kStages : 0; i < issued; ++i) {
+          if (p.withhold_first && i == 0) continue;           // never armed
+          if (!mbar_wait_limit(full + (int)(i % kStages), (uint32_t)((i / kStages) & 1),
+                               &keep_going, lim))
+            break;
+        }
+      }
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0 && rank == 0) {
       constexpr uint32_t idesc = idesc_bf16_f32(BM * CL, BN);
       uint32_t stage = 0, phase = 0, tile_i = 0;
+      bool any_mma = false;
       for (int64_t u = u0; u < units; u += ustep) {
         if (unit_skipped(p, sp, u, CL)) continue;
         int qb, split;
@@ -429,12 +462,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         unit_coords(sp, p.tiles, u, rank, CL, qb, split, t0, t1);
         for (int64_t t = t0; t < t1; ++t, ++tile_i) {
           const uint32_t acc = tile_i & 1u, aphase = (tile_i >> 1) & 1u;
-          if (!mbar_wait(tempty + acc, aphase ^ 1u, abort_flag)) goto mma_done;
+          if (!mbar_wait_limit(tempty + acc, aphase ^ 1u, abort_flag, lim)) goto mma_done;
           tc_fence_after();
           const uint32_t d_tmem = tmem_base + acc * BN;
           for (int kb = 0; kb < p.kb_count; ++kb) {
-            if (!mbar_wait(full + stage, phase, abort_flag)) goto mma_done;
+            if (!mbar_wait_limit(full + stage, phase, abort_flag, lim)) goto mma_done;
             tc_fence_after();
+            any_mma = true;
             const uint64_t a0 = smem_desc_k_sw128(smem_u32(sA + stage * kABytes));
             const uint64_t b0 = smem_desc_k_sw128(smem_u32(sB + stage * kBLocal));
 #pragma unroll
@@ -460,7 +494,18 @@ __global__ void __launch_bounds__(kThreads, 1)
             umma_commit_pair_mc(tfull + acc, 0x3);
         }
       }
-    mma_done:;
+    mma_done:
+      // Every MMA this thread issued completes before the teardown frees
+      // tensor memory, even when some role gave up (one commit to the drain
+      // barrier; in a normal run the last tile's MMAs are all it waits for).
+      if (any_mma) {
+        if (CL == 1)
+          umma_commit(drain);
+        else
+          umma_commit_pair_mc(drain, 0x1);
+        volatile int keep_going = 0;
+        mbar_wait_limit(drain, 0u, &keep_going, lim);
+      }
     }
   } else {
     // ------------------------------------------------------------ epilogue
@@ -522,7 +567,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       for (int64_t t = t0; t < t1; ++t, ++tile_i) {
         const uint32_t acc = tile_i & 1u, aphase = (tile_i >> 1) & 1u;
-        if (!mbar_wait(tfull + acc, aphase, abort_flag)) goto epi_done;
+        if (!mbar_wait_limit(tfull + acc, aphase, abort_flag, lim)) goto epi_done;
         tc_fence_after();
         theta = fmaxf(theta, qf_theta);
         const int64_t col0 = t * BN + half * kHalfCols;
@@ -1210,6 +1255,11 @@ int p2_for(int64_t nsplit, int32_t k) {
   return p2;
 }
 
+// Test hook of the main kernel's bounded waits (hs_debug_retrieve_wait): the
+// wait limit (0: 2 s) and whether every CTA withholds its first stage.
+std::atomic<uint64_t> g_ret_wait_limit_ns{0};
+std::atomic<int> g_ret_withhold{0};
+
 template <int KREG, int CL>
 hs_status configure_kernel() {
   static std::atomic<uint64_t> done{0};
@@ -1354,6 +1404,8 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
   prm.count_dev = count_dev;
   prm.k = k;
   prm.kb_count = (d + BK - 1) / BK;
+  prm.wait_limit_ns = g_ret_wait_limit_ns.load();
+  prm.withhold_first = g_ret_withhold.load();
   prm.part_s = reinterpret_cast<float*>(w);
   prm.part_i = reinterpret_cast<int32_t*>(w + part);
   prm.list_s = reinterpret_cast<float*>(w + 2 * part);
@@ -1496,3 +1548,16 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
 }
 
 }  // namespace hs
+
+/*
+ * Diagnostics only (declared in hs.h as hs_debug_retrieve_wait).
+ */
+extern "C" hs_status hs_debug_retrieve_wait(uint64_t limit_ns, int32_t withhold_first) {
+  hs::clear_last_error();
+  if (limit_ns > hs::kWaitLimitNs) return hs::fail(HS_ERR_INVALID_ARG, "limit above 2 s");
+  if (withhold_first < 0 || withhold_first > 1)
+    return hs::fail(HS_ERR_INVALID_ARG, "withhold_first must be 0 or 1");
+  hs::g_ret_wait_limit_ns.store(limit_ns);
+  hs::g_ret_withhold.store(withhold_first);
+  return HS_OK;
+}

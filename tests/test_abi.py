@@ -62,6 +62,9 @@ def test_host_only_calls_without_gpu():
     assert lib.hs_debug_scan_wait(3_000_000_000, -1) == _lib.HS_ERR_INVALID_ARG
     assert lib.hs_debug_scan_wait(0, -2) == _lib.HS_ERR_INVALID_ARG
     assert lib.hs_debug_scan_wait(0, -1) == _lib.HS_OK
+    assert lib.hs_debug_retrieve_wait(3_000_000_000, 0) == _lib.HS_ERR_INVALID_ARG
+    assert lib.hs_debug_retrieve_wait(0, 2) == _lib.HS_ERR_INVALID_ARG
+    assert lib.hs_debug_retrieve_wait(0, 0) == _lib.HS_OK
 
 
 def test_binding_names_match_header():

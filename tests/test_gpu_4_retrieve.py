@@ -339,3 +339,32 @@ def test_large_k_optimistic_pass_and_exact_fallback(hot):
         check_topk(s[qq], i[qq], os_[r], oi[r], exact, N, k)
     if hot:
         assert set(range(1000, 1100)) & set(i[0].tolist())   # the crowded rows are found
+
+
+def test_pipeline_wait_runs_out_and_reports_timeout():
+    """Failure detection without a fault: with a 1 ms wait limit and every
+    CTA withholding the copies of its first stage, the retrieval kernel's
+    pipeline waits run out.  The even CTA of each pair still waits for the
+    copies it armed before the pair frees tensor memory; the call returns in
+    well under the default 2 s limit, hs_get_device_error reports
+    HS_ERR_TIMEOUT (and clears it), and a normal call on the same stream
+    then meets the parity rule."""
+    import time
+    nq, N, d, k = 300, 8192, 128, 10          # CTA pairs, register lists
+    Q, C = unit_pair(nq, N, d, 21)
+    Qd, Cd = to_dev(Q), to_dev(C)
+    torch.cuda.synchronize()
+    try:
+        hs.hs_debug_retrieve_wait(1_000_000, 1)
+        t0 = time.perf_counter()
+        hs.hs_retrieve_topk(Qd, Cd, k)
+        with pytest.raises(hs.HsError) as e:
+            hs.hs_get_device_error()          # synchronises
+        elapsed = time.perf_counter() - t0
+        assert e.value.status == hs.HS_ERR_TIMEOUT
+        assert elapsed < 1.0, elapsed
+    finally:
+        hs.hs_debug_retrieve_wait(0, 0)
+    hs.hs_get_device_error()                  # cleared
+    gs, gi = gpu_topk(Qd, Cd, k)
+    parity(Q, C, k, gs, gi, range(nq))
