@@ -542,15 +542,17 @@ hs_status hs_debug_merge_key_mask(uint64_t mask);
 
 /*
  * hs_debug_retrieve_wait — test hook of the retrieval's bounded waits
- * (failure detection); takes no part in the method.  The main retrieval
- * kernel (launches with more than 16 addressable queries) gives up a
- * pipeline wait (shared-memory stage, tensor-memory accumulator) after
- * limit_ns, sets HS_ERR_TIMEOUT in the device error word and returns: before
- * its CTA pair frees tensor memory, the even CTA waits (with the same
- * limit) for every stage copy it armed and every MMA it issued.  With
- * withhold_first = 1 every CTA skips the copies of its first stage, so that
- * stage never fills and the waits run out; the outputs of such a call are
- * unspecified (every write stays inside the outputs and the workspace).
+ * (failure detection); takes no part in the method.  Both retrieval kernels
+ * (the main one and, for at most 16 addressable queries, the small-batch
+ * one) give up a pipeline wait (shared-memory stage, query load,
+ * tensor-memory accumulator) after limit_ns, set HS_ERR_TIMEOUT in the
+ * device error word and return: before tensor memory is freed, the CTA
+ * whose barriers count the copies (the even CTA of a pair) waits, with the
+ * same limit, for every copy it armed and every MMA it issued.  With
+ * withhold_first = 1 every CTA skips the copies of its first corpus stage,
+ * so that stage never fills and the waits run out; the outputs of such a
+ * call are unspecified (every write stays inside the outputs and the
+ * workspace).
  *
  * limit_ns        wait limit in ns, at most 2e9; 0 restores 2 s.
  * withhold_first  0 or 1.

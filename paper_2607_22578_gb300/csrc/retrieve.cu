@@ -998,7 +998,7 @@ constexpr size_t SQ_EPI_BYTES = (size_t)SQ_N * (SQ_CAP + 32) * 8 + SQ_N * 8;
 constexpr size_t SQ_SMEM = 1024 + (size_t)SQ_MAXKB * SQ_QBYTES + (size_t)SQ_STAGES * SQ_ABYTES +
                            256 + SQ_EPI_BYTES;
 static_assert(SQ_SMEM <= 232448, "small-batch kernel shared memory");
-static_assert(8 * (2 * SQ_STAGES + 1 + 2 * SQ_TBUF) + 8 <= 256, "small-batch barrier area");
+static_assert(8 * (2 * SQ_STAGES + 1 + 2 * SQ_TBUF) + 8 + 8 <= 256, "small-batch barrier area");
 
 __global__ void __launch_bounds__(SQ_THREADS, 1)
     retrieve_small_kernel(const __grid_constant__ CUtensorMap tmap_q,
@@ -1017,6 +1017,8 @@ __global__ void __launch_bounds__(SQ_THREADS, 1)
   uint64_t* tempty = tfull + SQ_TBUF;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + SQ_TBUF);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  uint64_t* drain = tempty + SQ_TBUF + 1;    // after tmem_slot and abort_flag: the MMA drain
+  const uint64_t lim = p.wait_limit_ns ? p.wait_limit_ns : kWaitLimitNs;
   uint64_t* lists = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(bars) + 256);  // [16][32]
   uint64_t* cands = lists + SQ_N * 32;                                                    // [16][128]
   float* theta = reinterpret_cast<float*>(cands + SQ_N * SQ_CAP);                          // [16]
@@ -1033,6 +1035,7 @@ __global__ void __launch_bounds__(SQ_THREADS, 1)
       mbar_init(tfull + b, 1);
       mbar_init(tempty + b, 4);
     }
+    mbar_init(drain, 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -1068,9 +1071,19 @@ __global__ void __launch_bounds__(SQ_THREADS, 1)
       for (int kb = 0; kb < p.kb_count; ++kb)
         tma_load_2d(sQ + kb * SQ_QBYTES, &tmap_q, qfull, kb * BK, 0);
       uint32_t stage = 0, phase = 0;
+      int64_t issued = 0;                 // corpus stages armed (or withheld) so far
       for (int64_t t = t0; t < t1; ++t) {
         for (int kb = 0; kb < p.kb_count; ++kb) {
-          if (!mbar_wait(empty + stage, phase ^ 1u, abort_flag)) goto sq_producer_done;
+          if (!mbar_wait_limit(empty + stage, phase ^ 1u, abort_flag, lim)) goto sq_producer_done;
+          if (p.withhold_first && issued == 0) {   // test hook: this stage never fills
+            ++issued;
+            if (++stage == SQ_STAGES) {
+              stage = 0;
+              phase ^= 1u;
+            }
+            continue;
+          }
+          ++issued;
           mbar_arrive_expect_tx(full + stage, SQ_ABYTES);
           tma_load_2d_hint(sA + stage * SQ_ABYTES, &tmap_c, full + stage, kb * BK,
                            (int32_t)(t * SQ_BM), pol_c);
@@ -1080,23 +1093,40 @@ __global__ void __launch_bounds__(SQ_THREADS, 1)
           }
         }
       }
-    sq_producer_done:;
+    sq_producer_done:
+      // Before it leaves, the producer waits, bounded, for the query copies
+      // and every corpus stage it armed that may still be in flight, so no
+      // copy lands in shared memory after the CTA exits, even when some role
+      // gave up (in a normal run these phases have completed or complete
+      // within the last tile).
+      {
+        volatile int keep_going = 0;
+        mbar_wait_limit(qfull, 0u, &keep_going, lim);
+        for (int64_t i = issued > SQ_STAGES ? issued - SQ_STAGES : 0; i < issued; ++i) {
+          if (p.withhold_first && i == 0) continue;           // never armed
+          if (!mbar_wait_limit(full + (int)(i % SQ_STAGES), (uint32_t)((i / SQ_STAGES) & 1),
+                               &keep_going, lim))
+            break;
+        }
+      }
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0 && Q > 0) {
       constexpr uint32_t idesc = idesc_bf16_f32(SQ_BM, SQ_N);
       uint32_t stage = 0, phase = 0, tile_i = 0;
-      if (!mbar_wait(qfull, 0u, abort_flag)) goto sq_mma_done;
+      bool any_mma = false;
+      if (!mbar_wait_limit(qfull, 0u, abort_flag, lim)) goto sq_mma_done;
       tc_fence_after();
       for (int64_t t = t0; t < t1; ++t, ++tile_i) {
         const uint32_t b = tile_i % SQ_TBUF, bphase = (tile_i / SQ_TBUF) & 1u;
-        if (!mbar_wait(tempty + b, bphase ^ 1u, abort_flag)) goto sq_mma_done;
+        if (!mbar_wait_limit(tempty + b, bphase ^ 1u, abort_flag, lim)) goto sq_mma_done;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + b * SQ_N;
         for (int kb = 0; kb < p.kb_count; ++kb) {
-          if (!mbar_wait(full + stage, phase, abort_flag)) goto sq_mma_done;
+          if (!mbar_wait_limit(full + stage, phase, abort_flag, lim)) goto sq_mma_done;
           tc_fence_after();
+          any_mma = true;
           const uint64_t a0 = smem_desc_k_sw128(smem_u32(sA + stage * SQ_ABYTES));
           const uint64_t b0 = smem_desc_k_sw128(smem_u32(sQ + kb * SQ_QBYTES));
 #pragma unroll
@@ -1111,7 +1141,14 @@ __global__ void __launch_bounds__(SQ_THREADS, 1)
         }
         umma_commit(tfull + b);
       }
-    sq_mma_done:;
+    sq_mma_done:
+      // Every MMA this thread issued completes before the teardown frees
+      // tensor memory (one commit to the drain barrier).
+      if (any_mma) {
+        umma_commit(drain);
+        volatile int keep_going = 0;
+        mbar_wait_limit(drain, 0u, &keep_going, lim);
+      }
     }
   } else {
     // ------------------------------------------------------------ epilogue
@@ -1124,7 +1161,7 @@ __global__ void __launch_bounds__(SQ_THREADS, 1)
       const uint32_t b = tile_i % SQ_TBUF, bphase = (tile_i / SQ_TBUF) & 1u;
       // On a timeout every later wait fails at once; the named barriers
       // below stay paired because all four warps walk every tile.
-      const bool ok = mbar_wait(tfull + b, bphase, abort_flag);
+      const bool ok = mbar_wait_limit(tfull + b, bphase, abort_flag, lim);
       tc_fence_after();
       uint32_t r[16];
       tmem_ld_32x32b_x16(tmem_base + lane_addr + b * SQ_N, r);

@@ -341,16 +341,17 @@ def test_large_k_optimistic_pass_and_exact_fallback(hot):
         assert set(range(1000, 1100)) & set(i[0].tolist())   # the crowded rows are found
 
 
-def test_pipeline_wait_runs_out_and_reports_timeout():
+@pytest.mark.parametrize("nq", [300, 8])    # CTA pairs; the small-batch kernel
+def test_pipeline_wait_runs_out_and_reports_timeout(nq):
     """Failure detection without a fault: with a 1 ms wait limit and every
-    CTA withholding the copies of its first stage, the retrieval kernel's
-    pipeline waits run out.  The even CTA of each pair still waits for the
-    copies it armed before the pair frees tensor memory; the call returns in
-    well under the default 2 s limit, hs_get_device_error reports
-    HS_ERR_TIMEOUT (and clears it), and a normal call on the same stream
-    then meets the parity rule."""
+    CTA withholding the copies of its first corpus stage, the retrieval
+    kernel's pipeline waits run out.  The CTA that counts the copies still
+    waits for those it armed, and for its MMAs, before tensor memory is
+    freed; the call returns in well under the default 2 s limit,
+    hs_get_device_error reports HS_ERR_TIMEOUT (and clears it), and a
+    normal call on the same stream then meets the parity rule."""
     import time
-    nq, N, d, k = 300, 8192, 128, 10          # CTA pairs, register lists
+    N, d, k = 8192, 128, 10
     Q, C = unit_pair(nq, N, d, 21)
     Qd, Cd = to_dev(Q), to_dev(C)
     torch.cuda.synchronize()
