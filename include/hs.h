@@ -17,6 +17,8 @@
  *   hs_cache_lookup / hs_cache_insert   a device-resident result cache
  * and the scheduling weight of the merged nodes:
  *   hs_segment_sum           priority contribution of each fused node (Eq. 3)
+ * and a batch's copies between host buffers and the device:
+ *   hs_memcpy_async
  *
  * Conventions shared by every call
  *   - Pointers named *_dev or documented as device pointers must be device
@@ -500,6 +502,19 @@ hs_status hs_segment_sum(const double* phi, const int32_t* inverse, int64_t n_ro
  * takes precedence over HS_ERR_INVALID_ARG).
  */
 hs_status hs_get_device_error(hs_stream_t stream);
+
+/*
+ * hs_memcpy_async — copy `bytes` bytes from src to dst on `stream`: host
+ * to device, device to host or device to device, the direction taken from
+ * the pointers (unified addressing).  This is how a caller moves a batch's
+ * inputs from host buffers into the device buffers the other calls take,
+ * and its results back; with pinned host memory the copy is asynchronous
+ * and overlaps kernels on other streams.  The caller owns both buffers and
+ * keeps them alive until the copy has run.  bytes == 0 does nothing.
+ * Returns HS_ERR_INVALID_ARG for a NULL pointer with bytes > 0, and
+ * HS_ERR_CUDA if the runtime rejects the copy.
+ */
+hs_status hs_memcpy_async(void* dst, const void* src, size_t bytes, hs_stream_t stream);
 
 /*
  * hs_launch_count — diagnostics: number of kernels this library has launched

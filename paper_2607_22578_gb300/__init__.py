@@ -7,7 +7,7 @@ from ._lib import (HS_ERR_CUDA, HS_ERR_INVALID_ARG, HS_ERR_TIMEOUT, HS_ERR_UNSUP
                    HS_TOPK_MAX_K, HsError, hs_debug_merge_key_mask, hs_debug_retrieve_wait,
                    hs_debug_scan_wait,
                    hs_debug_stream_rows, hs_fingerprint, hs_merge_rows, hs_merge_rows_workspace, hs_get_device_error,
-                   hs_launch_count, hs_merge_queries, hs_retrieve_topk, hs_retrieve_topk_fanout,
+                   hs_launch_count, hs_memcpy_async, hs_merge_queries, hs_retrieve_topk, hs_retrieve_topk_fanout,
                    hs_retrieve_topk_n, hs_retrieve_topk_workspace, hs_scatter_results,
                    hs_rerank_topk, hs_segment_sum, ResultCache, hs_cache_bytes, hs_cache_init, hs_cache_insert,
                    hs_cache_lookup, hs_cache_stats,
@@ -22,7 +22,7 @@ __all__ = [
     "hs_unique_inverse_workspace", "hs_retrieve_topk", "hs_retrieve_topk_n",
     "hs_retrieve_topk_fanout", "hs_merge_queries", "hs_retrieve_topk_workspace",
     "hs_scatter_results", "hs_rerank_topk", "hs_segment_sum", "ResultCache",
-    "hs_cache_bytes", "hs_cache_init", "hs_cache_lookup", "hs_cache_insert", "hs_cache_stats", "hs_get_device_error", "hs_launch_count",
+    "hs_cache_bytes", "hs_cache_init", "hs_cache_lookup", "hs_cache_insert", "hs_cache_stats", "hs_get_device_error", "hs_launch_count", "hs_memcpy_async",
     "hs_debug_scan_wait", "hs_debug_stream_rows", "hs_debug_merge_key_mask",
     "hs_debug_retrieve_wait", "hs_merge_rows",
     "hs_merge_rows_workspace", "hs_version",

@@ -107,6 +107,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
             lib.hs_debug_merge_key_mask.restype = st
             lib.hs_debug_retrieve_wait.argtypes = [u64, i32]
             lib.hs_debug_retrieve_wait.restype = st
+            lib.hs_memcpy_async.argtypes = [P, P, sz, P]
+            lib.hs_memcpy_async.restype = st
             lib.hs_debug_stream_rows.argtypes = [P, i64, i32, P, i32, P, i32, P]
             lib.hs_debug_stream_rows.restype = st
             _lib = lib
@@ -222,6 +224,21 @@ def hs_debug_merge_key_mask(mask: int = 0) -> None:
     """Test hook of hs_merge_rows: key the table by fp & mask (0 restores
     all ones; see hs.h)."""
     _check(load().hs_debug_merge_key_mask(int(mask)))
+
+
+def hs_memcpy_async(dst: torch.Tensor, src: torch.Tensor, stream=None) -> torch.Tensor:
+    """Copy src into dst (equal byte sizes, contiguous; host, pinned host or
+    device on either side) on `stream` through the C ABI.  Returns dst."""
+    if not dst.is_contiguous() or not src.is_contiguous():
+        raise ValueError("dst and src must be contiguous")
+    nbytes = dst.numel() * dst.element_size()
+    if nbytes != src.numel() * src.element_size():
+        raise ValueError("dst and src differ in size")
+    if not (dst.is_cuda or src.is_cuda):
+        raise ValueError("one side must be on the GPU")
+    _check(load().hs_memcpy_async(ctypes.c_void_p(dst.data_ptr()), ctypes.c_void_p(src.data_ptr()),
+                                  nbytes, _stream(stream)))
+    return dst
 
 
 def hs_debug_retrieve_wait(limit_ns: int = 0, withhold_first: int = 0) -> None:

@@ -467,4 +467,15 @@ hs_status hs_get_device_error(hs_stream_t stream) {
   return HS_OK;
 }
 
+hs_status hs_memcpy_async(void* dst, const void* src, size_t bytes, hs_stream_t stream) {
+  clear_msg();
+  if (bytes == 0) return HS_OK;
+  if (!dst || !src) return fail(HS_ERR_INVALID_ARG, "NULL pointer");
+  // One copy, its direction from unified addressing (pinned or pageable
+  // host memory, or device memory, on either side).
+  return cuda_fail(cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDefault,
+                                   reinterpret_cast<cudaStream_t>(stream)),
+                   "copy");
+}
+
 }  // extern "C"

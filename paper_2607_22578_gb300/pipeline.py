@@ -309,8 +309,8 @@ class HostFeed:
         if self.used[b]:
             self.copy_stream.wait_event(self.freed[b])
         with torch.cuda.stream(self.copy_stream):
-            self.d_tok[b].copy_(h_tokens, non_blocking=True)
-            self.d_q[b].view(torch.int16).copy_(h_queries.view(torch.int16), non_blocking=True)
+            _lib.hs_memcpy_async(self.d_tok[b], h_tokens, self.copy_stream)
+            _lib.hs_memcpy_async(self.d_q[b], h_queries, self.copy_stream)
             self.copied[b].record(self.copy_stream)
         main.wait_event(self.copied[b])
         if self.graphs is not None:
@@ -318,9 +318,9 @@ class HostFeed:
         else:
             _, (s, i, nu) = self.stage.step(self.d_tok[b], self.d_q[b])
         self.freed[b].record(main)
-        self.h_s[b].copy_(s, non_blocking=True)
-        self.h_i[b].copy_(i, non_blocking=True)
-        self.h_nu[b].copy_(nu, non_blocking=True)
+        _lib.hs_memcpy_async(self.h_s[b], s, main)
+        _lib.hs_memcpy_async(self.h_i[b], i, main)
+        _lib.hs_memcpy_async(self.h_nu[b], nu, main)
         self.done[b].record(main)
         self.used[b] = True
         return b

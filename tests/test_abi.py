@@ -65,6 +65,8 @@ def test_host_only_calls_without_gpu():
     assert lib.hs_debug_retrieve_wait(3_000_000_000, 0) == _lib.HS_ERR_INVALID_ARG
     assert lib.hs_debug_retrieve_wait(0, 2) == _lib.HS_ERR_INVALID_ARG
     assert lib.hs_debug_retrieve_wait(0, 0) == _lib.HS_OK
+    assert lib.hs_memcpy_async(None, None, 0, None) == _lib.HS_OK
+    assert lib.hs_memcpy_async(None, None, 16, None) == _lib.HS_ERR_INVALID_ARG
 
 
 def test_binding_names_match_header():

@@ -75,3 +75,26 @@ def test_overlap_rejected():
     with pytest.raises(hs.HsError):
         hs.hs_scatter_results(buf[:32].view(2, 16), to_dev(np.array([0, 1], np.int32)),
                               dst=buf[16:48].view(2, 16))
+
+
+def test_memcpy_async_round_trips_host_and_device():
+    """hs_memcpy_async (the C ABI's copy between host buffers and the
+    device): pinned host -> device -> device -> pageable host, bytes
+    unchanged; zero bytes is a no-op."""
+    import numpy as np
+    import torch
+    rng = np.random.default_rng(12)
+    src = torch.from_numpy(rng.integers(0, 255, size=(1000, 1536), dtype=np.uint8)).pin_memory()
+    d0 = torch.empty_like(src, device="cuda")
+    d1 = torch.empty_like(d0)
+    back = torch.empty_like(src)                     # pageable
+    s = torch.cuda.Stream()
+    hs.hs_memcpy_async(d0, src, s)
+    hs.hs_memcpy_async(d1, d0, s)
+    hs.hs_memcpy_async(back, d1, s)
+    s.synchronize()
+    assert torch.equal(back, src)
+    empty = torch.empty(0, dtype=torch.uint8)
+    hs.hs_memcpy_async(torch.empty(0, dtype=torch.uint8, device="cuda"), empty, s)
+    with pytest.raises(ValueError):
+        hs.hs_memcpy_async(d0[:10], src, s)
