@@ -12,7 +12,7 @@ resident 1,048,576 x 768 bf16 corpus, k = 10):
 ``value`` is merged (unique) queries retrieved per second over all GPUs,
 with inputs resident in HBM; ``e2e`` is the same metric through the public
 API with the step's inputs copied from pinned host memory and its results
-copied back inside the timed region.
+copied back (``hs_memcpy_async`` of the C ABI) inside the timed region.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gb300|reference]
 
