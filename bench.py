@@ -617,6 +617,9 @@ def row_dedup_heavy(args, dev, peaks) -> dict:
     sc_bytes = n_u * W + n * W + 4 * n
     ss_bytes = 8 * n + 4 * n + 8 * n_u
     merge = _roof(fp_bytes + un_bytes, None, t_mr, peaks)
+    # the lower bound: one pass over the valid tokens (+ lens, fp, outputs)
+    merge["frac_hbm_one_pass"] = ((tok_bytes + 4 * n + 8 * n + 8 * n) / (t_mr / 1e3) / 1e9
+                                  / peaks["hbm_gbs"])
     return {
         "workload": "dedup_heavy: 400,000 rows x 512 int32 (lens U[64,512], Zipf(1.1) over "
                     "100,000 distinct) -> %d unique; scatter %d B per row" % (n_u, W),
@@ -634,7 +637,9 @@ def row_dedup_heavy(args, dev, peaks) -> dict:
             "hs_segment_sum": _roof(ss_bytes, None, t_ss, peaks)},
         "merge_bytes_note": "hs_merge_rows: the method bytes of the two calls it combines "
                             "(one pass over the valid tokens + the verify re-read of every row "
-                            "in a group of size >= 2, + lens, fp, outputs)",
+                            "in a group of size >= 2, + lens, fp, outputs); frac_hbm_one_pass "
+                            "counts the lower bound, one pass over the valid tokens + lens, fp "
+                            "and outputs",
         "segment_sum_note": "priority contribution per merged node (Eq. 3) over the same "
                             "inverse map, timed after the step and not part of its value; bytes: "
                             "phi (fp64) + inverse in, one fp64 per merged node out; the output "
