@@ -439,7 +439,7 @@ def gpu_arm(args, rank: int, local_rank: int, world: int) -> int:
             "roofline": {
                 "bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                 "frac": achieved / peak, "traffic": traffic,
-                "kernel": "hs_retrieve_topk (retrieve_kernel + merge_kernel), %.3f ms/launch"
+                "kernel": "hs_retrieve_topk (retrieve_kernel + merge_warp_kernel), %.3f ms/launch"
                           % ret_ms,
                 "algorithmic": "2 * %d merged queries * %d rows * %d dims = %.4g FLOP/launch"
                                % (n_u, N, d, flops),

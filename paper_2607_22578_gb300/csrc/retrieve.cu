@@ -37,7 +37,8 @@
 // lanes.  For k > 32 a 16-entry candidate buffer per thread in shared memory
 // is sorted and merged into a sorted list in global scratch whenever a
 // buffer fills.  Each unit writes its k best per (query, half); K7 merges the
-// lists of each query with a bitonic sort of packed (score, index) keys.
+// sorted lists of each query: one warp per query takes the largest head of
+// its lists k times (packed (score, index) keys).
 #include <float.h>
 
 #include <algorithm>
@@ -59,7 +60,7 @@ constexpr uint32_t kABytes = BM * BK * 2;
 constexpr uint32_t kBBytes = BN * BK * 2;
 constexpr uint32_t kTmemCols = 2 * BN;
 constexpr int kCap = 16;              // candidate buffer per thread (large-k path)
-constexpr int kMergeMax = 16384;      // lists * k bound for K7
+constexpr int kMergeMax = 16384;      // bound on lists * k per query (the merge's candidates)
 constexpr size_t kBarBytes = 256;
 constexpr size_t kEpiSmem = (size_t)kEpi * 32 * 4;  // 32 KB: staging or candidate buffer
 static_assert((size_t)kCap * kEpi * 8 == kEpiSmem, "candidate buffer size");
@@ -783,8 +784,14 @@ constexpr int kMaxListsPerLane = 10;
 
 // Any kout: picks 0..31 are kept one per lane and written together when
 // kout <= 32; for larger kout each pick is written as it is made.  With
-// out_i NULL only the kout-th pick's score is written, to out_s[o].  `only`
-// and `flag_out` are as for merge_kernel.  LPL lists per lane at most (the
+// out_i NULL only the kout-th pick's score is written, to out_s[o] (the
+// floor of the second large-k pass).  With `only` set, rows whose query
+// block is not flagged there are skipped.  With `flag_out` set, a query's
+// block is flagged when one of its lists may have cut off a member of the
+// top kout: a full list whose last (k-th) entry is not below the union's
+// kout-th pick.  A list whose last entry is below it holds every row of its
+// range that can be in the top kout, so with no list flagged the union's
+// first kout entries are exact.  LPL lists per lane at most (the
 // launch's bound on 2 * nsplit / 32, rounded up); slots past the query's
 // list count are skipped warp-uniformly, so the per-round work and the
 // registers follow the lists a launch can have, not the largest count.
@@ -885,86 +892,6 @@ __global__ void __launch_bounds__(256) merge_warp_kernel(const Params p, float* 
       }
       if (__any_sync(0xffffffffu, cut) && lane == 0) atomicOr(flag_out + q / BM, 1u);
     }
-  }
-}
-
-// Lists of p.k entries per (query, split, half) -> the kout best per query.
-// With out_i NULL only the kout-th best score of each query is written, to
-// out_s[q] (the floor of the second large-k pass).  With `only` set, rows
-// whose query block is not flagged there are skipped.  With `flag_out` set,
-// a query's block is flagged when one of its lists may have cut off a member
-// of the top kout: a full list whose last (k-th) entry is not below the
-// union's kout-th best.  A list whose last entry is below that score holds
-// every row of its range that can be in the top kout, so with no list
-// flagged the union's first kout entries are exact.
-__global__ void __launch_bounds__(256) merge_kernel(const Params p, float* __restrict__ out_s,
-                                                    int32_t* __restrict__ out_i, int32_t kout,
-                                                    OutRows rows, uint32_t* flag_out,
-                                                    const uint32_t* only) {
-  pdl_wait();
-  pdl_trigger();
-  extern __shared__ uint64_t keys[];
-  const int64_t Q = query_count(p);
-  const SplitPlan sp = split_plan(Q, p.tiles, p.k, p.slots, p.cl);
-  const int k = p.k;
-  const int lists = 2 * sp.nsplit;
-  const int m = lists * k;
-  int p2 = 1;
-  while (p2 < m) p2 <<= 1;
-  const float* __restrict__ part_s = p.part_s;
-  const int32_t* __restrict__ part_i = p.part_i;
-  const int64_t R = rows.inv ? rows.n_out : Q;
-  for (int64_t o = blockIdx.x; o < R; o += gridDim.x) {
-    const int64_t q = rows.inv ? (int64_t)__ldg(rows.inv + o) : o;
-    if (q < 0 || q >= Q) {                         // block-uniform
-      if (threadIdx.x == 0) set_error(p.err, kErrInvalidArg);
-      continue;
-    }
-    if (only && only[q / BM] == 0u) continue;      // block-uniform
-    const float* ps = part_s + (size_t)q * m;
-    const int32_t* pi = part_i + (size_t)q * m;
-    for (int e = threadIdx.x; e < p2; e += blockDim.x) keys[e] = e < m ? pack_key(ps[e], pi[e]) : 0ull;
-    __syncthreads();
-    // Bitonic sort, descending.
-    for (int size = 2; size <= p2; size <<= 1) {
-      for (int stride = size >> 1; stride > 0; stride >>= 1) {
-        for (int t = threadIdx.x; t < (p2 >> 1); t += blockDim.x) {
-          const int lo = 2 * t - (t & (stride - 1));
-          const int hi = lo + stride;
-          const bool desc = (lo & size) == 0;
-          const uint64_t a = keys[lo], b = keys[hi];
-          if ((a < b) == desc) {
-            keys[lo] = b;
-            keys[hi] = a;
-          }
-        }
-        __syncthreads();
-      }
-    }
-    if (flag_out) {
-      const uint64_t kth = kout - 1 < m ? keys[kout - 1] : 0ull;
-      bool cut = false;
-      for (int l = threadIdx.x; l < lists; l += blockDim.x)
-        cut |= pack_key(ps[(size_t)l * k + k - 1], pi[(size_t)l * k + k - 1]) >= kth;
-      if (__syncthreads_or(cut) && threadIdx.x == 0) atomicOr(flag_out + q / BM, 1u);
-    }
-    if (!out_i) {
-      if (threadIdx.x == 0) {
-        float s = -FLT_MAX;
-        int32_t idx = -1;
-        if (kout - 1 < m) unpack_key(keys[kout - 1], s, idx);
-        out_s[o] = s;
-      }
-    } else {
-      for (int j = threadIdx.x; j < kout; j += blockDim.x) {
-        float s = -FLT_MAX;
-        int32_t idx = -1;
-        if (j < m) unpack_key(keys[j], s, idx);
-        out_s[(size_t)o * kout + j] = s;
-        out_i[(size_t)o * kout + j] = idx;
-      }
-    }
-    __syncthreads();
   }
 }
 
@@ -1286,12 +1213,6 @@ bool make_map(CUtensorMap* map, const uint16_t* base, int64_t rows, int32_t d, u
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-int p2_for(int64_t nsplit, int32_t k) {
-  int p2 = 1;
-  while (p2 < 2 * nsplit * k) p2 <<= 1;
-  return p2;
-}
-
 // Test hook of the main kernel's bounded waits (hs_debug_retrieve_wait): the
 // wait limit (0: 2 s) and whether every CTA withholds its first stage.
 std::atomic<uint64_t> g_ret_wait_limit_ns{0};
@@ -1366,11 +1287,14 @@ hs_status launch_variant(const uint16_t* corpus, int64_t N, int32_t d, const CUt
   hs_status st = configure_kernel<KREG, 1>();
   if (st != HS_OK) return st;
   int cl = 1;
-  int64_t slots = sms;
+  // Unit executors: at most 16 * kMaxListsPerLane, so every query's lists
+  // (2 per split, nsplit <= slots) fit the warp merge.
+  int64_t slots = std::min<int64_t>(sms, 16 * kMaxListsPerLane);
   if (qblocks_max >= 2) {
     st = configure_kernel<KREG, 2>();
     if (st != HS_OK) return st;
-    const int64_t pairs = std::min<int64_t>(max_pairs<KREG>(), sms / 2);
+    const int64_t pairs = std::min<int64_t>(std::min<int64_t>(max_pairs<KREG>(), sms / 2),
+                                            16 * kMaxListsPerLane);
     if (pairs >= 1) {
       cl = 2;
       slots = pairs;
@@ -1465,7 +1389,12 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
                    uint32_t* flag_out = nullptr, const uint32_t* only = nullptr) -> hs_status {
     const int64_t nr = orows.inv ? orows.n_out : Qmax;
     if (nr == 0) return HS_OK;
-    if (2 * (int64_t)pm.slots <= 32 * kMaxListsPerLane) {
+    // Every plan caps its executors (slots) at 16 * kMaxListsPerLane, so a
+    // query has at most 32 * kMaxListsPerLane lists: the warp merge takes
+    // every launch.
+    if (2 * (int64_t)pm.slots > 32 * kMaxListsPerLane)
+      return fail(HS_ERR_UNSUPPORTED, "more lists per query than the merge takes");
+    {
       const int64_t blocks = (nr + 7) / 8;          // one warp per row
       const dim3 grid((unsigned)(blocks < sms * 16 ? blocks : sms * 16));
       // lists per query <= 2 * slots (nsplit <= slots): lanes need that / 32
@@ -1484,19 +1413,6 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
                    kout, orows, flag_out, only);
       return cuda_fail(cudaGetLastError(), "merge launch");
     }
-    const int64_t mgrid = nr < sms * 8 ? nr : sms * 8;
-    const size_t msmem = (size_t)p2_for(max_splits(sms, pm.tiles, pm.k), pm.k) * 8;
-    static std::atomic<size_t> merge_configured[kMaxDeviceOrdinals];   // per device
-    const int dev = device_ordinal();
-    if (msmem > 48 * 1024 && (dev < 0 || msmem > merge_configured[dev].load())) {
-      cudaError_t e = cudaFuncSetAttribute(merge_kernel,
-                                           cudaFuncAttributeMaxDynamicSharedMemorySize, (int)msmem);
-      if (e != cudaSuccess) return cuda_fail(e, "merge smem attribute");
-      if (dev >= 0) merge_configured[dev].store(msmem);
-    }
-    launch_pdl(merge_kernel, dim3((unsigned)mgrid), dim3(256), msmem, stream, pm, os, oi, kout,
-               orows, flag_out, only);
-    return cuda_fail(cudaGetLastError(), "merge launch");
   };
   hs_status st;
   if (small) {
@@ -1514,7 +1430,7 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
     if (cst != HS_OK) return cst;
     // Lists per query = 2 * nsplit of the plan the merge kernel recomputes
     // (one query block, one group: nsplit = min(slots, tiles, 8192 / k)).
-    prm.slots = (int32_t)std::max<int64_t>(1, sms / 2);
+    prm.slots = (int32_t)std::max<int64_t>(1, std::min<int64_t>(sms / 2, 16 * kMaxListsPerLane));
     prm.cl = 1;
     const SplitPlan sp = split_plan(1, tiles, k, prm.slots, 1);
     const int64_t grid = 2 * (int64_t)sp.nsplit;
@@ -1580,7 +1496,7 @@ hs_status launch_retrieve_topk(const uint16_t* queries, int64_t Qmax, const int3
   if (st != HS_OK) return st;
   st = merge(prm, k, scores_out, ids_out, rows, nullptr, prm.only);
   if (st != HS_OK) return st;
-  count_launches(R > 0 ? 2 : 1);  // retrieve_kernel + merge_kernel
+  count_launches(R > 0 ? 2 : 1);  // retrieve_kernel + merge_warp_kernel
   return HS_OK;
 }
 
